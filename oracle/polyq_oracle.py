@@ -1,0 +1,444 @@
+"""PolyQ reference oracle: a plain, slow, fp64 CPU restatement of the method.
+
+TEST INFRASTRUCTURE ONLY.  Only ``tests/``, ``__graft_entry__.smoke()`` and the
+``cpu_baseline`` / ``--impl reference`` legs of ``bench.py`` may import this
+module.  The product (the C-ABI library under ``paper_2607_14618_gb300``) never
+imports, links or calls it, and this module shares no code with it.
+
+What is restated here (PolyQ, arXiv 2607.14618):
+
+* §3.1  activation-aware per-channel error proxy (E_16 = 0); the proxy is
+        instantiated from the channel saliency ``a_k * ||W[:,k]||`` (reading
+        R3 below).
+* §3.2  layer-wise fractional budget, the residual budget
+        ``Delta = round(B*K) - b_min*K``, the gain-per-bit ``G_{b->b'}`` and the
+        greedy max-heap waterfilling.
+* §3.4 / §3.1 group-wise uniform quantisation at each channel's width
+        (reading R1: asymmetric, fp16 scale/zero per output row per
+        64-channel group; 16-bit channels stored as fp16).
+* §4.1  channel permutation/clustering ``O = (A P^T)(P W)``: only the
+        clustered weight is materialised; the activation is gathered.
+* §4.2  bit-homogeneous blocks (one segment per width per row).
+* §4.3  the merge rule ``O' = A (W P^T)(P W')``: the producer emits its
+        outputs in the consumer's basis, so the consumer's gather becomes the
+        identity.
+* §5.3  the per-token reorder-traffic model (A16 read+write bytes of explicit
+        activation shuffles).
+
+Readings taken where the paper is silent (the same list is in the design doc):
+
+R1 quantiser: per (row n, block, 64-position group of the clustered order),
+   lo=min w, hi=max w, qmax=2^b-1, s=fp16_rn((hi-lo)/qmax), if s==0 then
+   s=fp16_rn(max(|lo|,|hi|,2^-14)); z=clamp(rint(-lo/s),0,qmax);
+   q=clamp(rint(w/s)+z,0,qmax); dequant w'=(q-z)*s.  rint = half-to-even.
+   16-bit channels: w' = fp16_rn(w).  |W| must be finite and <= 65504.
+R2 saliency: sal_k = a_k * sqrt(sum_n W[n,k]^2), the sum taken in fp64 in row
+   order n = 0..N-1.
+R3 allocation (WATERFILL_SALIENCY): E_b[k] = (sal_k/(2^b-1))^2 for b<16,
+   E_16 = 0; max-heap keyed by (gain desc, channel index asc); a popped step
+   that does not fit the residual budget is dropped (the channel stops).
+   SALIENCY_LADDER (option): channels in descending saliency each climb the
+   palette while the next step fits.
+R4 permutation: blocks in ascending width; inside a block ascending channel.
+R5 packing: per (row, block) an LSB-first bitstream (code p at bits
+   [p*b, p*b+b), little-endian bytes), zero-padded to a multiple of 16 bytes;
+   16-bit segments are little-endian fp16 padded with +0.0.  A row is the
+   concatenation of its segments in block order.  meta[n][g] = (scale, zero)
+   as two fp16, groups ordered by block then position.
+R6 merge: a producer basis beta means emitted[i] = y_orig[beta[i]]; the
+   consumer gather is r = beta^-1 o P_c, i.e. xs[p] = x_emitted[r[p]].
+"""
+from __future__ import annotations
+
+import heapq
+import math
+
+import numpy as np
+
+PALETTE = (2, 3, 4, 8, 16)
+GROUP = 64
+FP16_MAX = 65504.0
+WATERFILL_SALIENCY = 0
+SALIENCY_LADDER = 1
+
+
+# ---------------------------------------------------------------------------
+# scalar helpers
+# ---------------------------------------------------------------------------
+def fp16_rn(v):
+    """Round fp64 values to the nearest fp16 (ties to even), returned as fp64.
+
+    NumPy converts float64 -> float16 directly (no float32 step), so this is a
+    single correctly rounded conversion."""
+    return np.asarray(v, dtype=np.float64).astype(np.float16).astype(np.float64)
+
+
+def _check_weights(W):
+    W = np.asarray(W)
+    if W.ndim != 2:
+        raise ValueError("W must be 2-D [N][K]")
+    if not np.all(np.isfinite(W)) or (W.size and np.max(np.abs(W)) > FP16_MAX):
+        raise ValueError("W must be finite with |W| <= 65504 (R1)")
+    return W
+
+
+# ---------------------------------------------------------------------------
+# §3.1 (R1): group-wise asymmetric uniform quantiser
+# ---------------------------------------------------------------------------
+def quantize_group(w, b):
+    """Quantise one group of weights (1-D, fp64) to ``b`` bits (R1, §3.1/§3.4).
+
+    Returns (s, z, q): the fp16-representable scale and zero (as floats) and
+    the integer codes."""
+    w = np.asarray(w, dtype=np.float64)
+    qmax = (1 << b) - 1
+    lo = float(w.min())
+    hi = float(w.max())
+    s = float(fp16_rn((hi - lo) / qmax))
+    if s == 0.0:
+        s = float(fp16_rn(max(abs(lo), abs(hi), 2.0 ** -14)))
+    z = float(min(max(np.rint(-lo / s), 0.0), float(qmax)))
+    q = np.clip(np.rint(w / s) + z, 0.0, float(qmax)).astype(np.int64)
+    return s, z, q
+
+
+def quantize_rows(Wb, b):
+    """Quantise a block ``Wb`` (N x K_b, fp64) group by group along columns.
+
+    Each row and each run of 64 consecutive columns (the last run may be
+    shorter) is one group.  Same arithmetic as :func:`quantize_group`,
+    evaluated for all rows of a group at once.  Returns (scale[N,G],
+    zero[N,G], codes[N,K_b])."""
+    N, Kb = Wb.shape
+    qmax = float((1 << b) - 1)
+    ng = -(-Kb // GROUP)
+    S = np.zeros((N, ng))
+    Z = np.zeros((N, ng))
+    Q = np.zeros((N, Kb), dtype=np.int64)
+    for g in range(ng):
+        cols = slice(g * GROUP, min((g + 1) * GROUP, Kb))
+        w = Wb[:, cols]
+        lo = w.min(axis=1)
+        hi = w.max(axis=1)
+        s = fp16_rn((hi - lo) / qmax)
+        fb = s == 0.0
+        if np.any(fb):
+            alt = np.maximum(np.maximum(np.abs(lo), np.abs(hi)), 2.0 ** -14)
+            s = np.where(fb, fp16_rn(alt), s)
+        z = np.clip(np.rint(-lo / s), 0.0, qmax)
+        q = np.clip(np.rint(w / s[:, None]) + z[:, None], 0.0, qmax)
+        S[:, g] = s
+        Z[:, g] = z
+        Q[:, cols] = q.astype(np.int64)
+    return S, Z, Q
+
+
+# ---------------------------------------------------------------------------
+# §3.1 / §3.2 (R2, R3): saliency, error proxy, greedy waterfilling
+# ---------------------------------------------------------------------------
+def saliency(W, act_absmean):
+    """sal_k = a_k * sqrt(sum_n W[n,k]^2) in fp64, rows summed in order (R2)."""
+    W = np.asarray(W)
+    acc = np.zeros(W.shape[1], dtype=np.float64)
+    for n in range(W.shape[0]):
+        row = W[n].astype(np.float64)
+        acc = acc + row * row
+    return np.asarray(act_absmean, dtype=np.float64) * np.sqrt(acc)
+
+
+def proxy_error(sal_k, b):
+    """E_b[k] from saliency: (sal/(2^b-1))^2, and E_16 = 0 (§3.1, R3)."""
+    if b == 16:
+        return 0.0
+    e = sal_k / float((1 << b) - 1)
+    return e * e
+
+
+def gain(sal_k, b, b_next):
+    """Gain per extra bit G_{b->b'} = (E_b - E_b') / (b' - b) (§3.2)."""
+    return (proxy_error(sal_k, b) - proxy_error(sal_k, b_next)) / float(b_next - b)
+
+
+def palette_from_mask(mask):
+    pal = tuple(b for b in PALETTE if mask & (1 << b))
+    if not pal:
+        raise ValueError("empty palette")
+    return pal
+
+
+def residual_budget(B, K, b_min):
+    """Delta = round(B*K) - b_min*K, round half up (§3.2)."""
+    return int(math.floor(B * K + 0.5)) - b_min * K
+
+
+def allocate_bits(sal, B, palette=PALETTE, rule=WATERFILL_SALIENCY):
+    """Per-channel widths under the average budget B (§3.2, R3).
+
+    Every channel starts at the smallest palette width; upgrades to the next
+    palette width are taken greedily by gain per bit from a max-heap until
+    the residual budget is spent or no step fits."""
+    sal = [float(v) for v in sal]
+    K = len(sal)
+    pal = tuple(sorted(palette))
+    b_min = pal[0]
+    nxt = {pal[i]: pal[i + 1] for i in range(len(pal) - 1)}
+    bits = [b_min] * K
+    delta = residual_budget(B, K, b_min)
+    if delta <= 0 or len(pal) == 1:
+        return np.array(bits, dtype=np.int64)
+    if rule == SALIENCY_LADDER:
+        order = sorted(range(K), key=lambda k: (-sal[k], k))
+        for k in order:
+            if delta == 0:
+                break
+            while bits[k] in nxt and nxt[bits[k]] - bits[k] <= delta:
+                delta -= nxt[bits[k]] - bits[k]
+                bits[k] = nxt[bits[k]]
+        return np.array(bits, dtype=np.int64)
+    heap = [(-gain(sal[k], b_min, nxt[b_min]), k, nxt[b_min]) for k in range(K)]
+    heapq.heapify(heap)
+    while delta > 0 and heap:
+        _, k, b_new = heapq.heappop(heap)
+        cost = b_new - bits[k]
+        if cost > delta:
+            continue  # can never fit later: Delta only shrinks
+        bits[k] = b_new
+        delta -= cost
+        if b_new in nxt:
+            heapq.heappush(heap, (-gain(sal[k], b_new, nxt[b_new]), k, nxt[b_new]))
+    return np.array(bits, dtype=np.int64)
+
+
+# ---------------------------------------------------------------------------
+# §4.1 / §4.2 (R4, R5): permutation, blocks, packing
+# ---------------------------------------------------------------------------
+def cluster_perm(bits):
+    """perm[p] = original channel at clustered position p (R4, §4.1)."""
+    bits = np.asarray(bits)
+    return np.argsort(bits, kind="stable").astype(np.int64)
+
+
+def seg_bytes(b, kb):
+    raw = kb * 2 if b == 16 else (kb * b + 7) // 8
+    return -(-raw // 16) * 16
+
+
+def make_blocks(bits):
+    """Block table: one entry per width present, ascending (§4.2)."""
+    bits = np.asarray(bits)
+    blocks = []
+    pos = 0
+    off = 0
+    goff = 0
+    for b in PALETTE:
+        kb = int(np.sum(bits == b))
+        if kb == 0:
+            continue
+        ng = 0 if b == 16 else -(-kb // GROUP)
+        sb = seg_bytes(b, kb)
+        blocks.append(dict(bits=b, n_ch=kb, pos0=pos, seg_off=off,
+                           seg_bytes=sb, grp_off=goff, n_grp=ng))
+        pos += kb
+        off += sb
+        goff += ng
+    return blocks, off, goff
+
+
+def pack_codes(codes, b, nbytes):
+    """LSB-first bitstream of ``codes`` (N x K_b) padded to ``nbytes`` (R5)."""
+    N, Kb = codes.shape
+    planes = (codes[:, :, None] >> np.arange(b)[None, None, :]) & 1
+    stream = planes.reshape(N, Kb * b).astype(np.uint8)
+    pad = nbytes * 8 - Kb * b
+    stream = np.concatenate([stream, np.zeros((N, pad), np.uint8)], axis=1)
+    return np.packbits(stream, axis=1, bitorder="little")
+
+
+def unpack_codes_from_bytes(seg, b, kb):
+    """Inverse of :func:`pack_codes` for one block segment (N x bytes)."""
+    bitsarr = np.unpackbits(seg, axis=1, bitorder="little")[:, : kb * b]
+    bitsarr = bitsarr.reshape(seg.shape[0], kb, b).astype(np.int64)
+    return (bitsarr << np.arange(b)[None, None, :]).sum(axis=2)
+
+
+def pack_layer(W, act_absmean, B, palette=PALETTE, rule=WATERFILL_SALIENCY,
+               bits=None):
+    """Allocation, permutation and packing of one linear layer.
+
+    ``W`` is [N][K] (out x in) float32, ``act_absmean`` the per-input-channel
+    activation magnitude.  ``bits`` may force a width map (tests).  Returns a
+    dict describing the layer in the R5 format."""
+    W = _check_weights(W)
+    N, K = W.shape
+    if bits is None:
+        sal = saliency(W, act_absmean)
+        bits = allocate_bits(sal, B, palette, rule)
+    bits = np.asarray(bits, dtype=np.int64)
+    perm = cluster_perm(bits)
+    blocks, S, G = make_blocks(bits)
+    packed = np.zeros((N, S), dtype=np.uint8)
+    meta = np.zeros((N, G, 2), dtype=np.uint16)
+    for blk in blocks:
+        b, kb, p0 = blk["bits"], blk["n_ch"], blk["pos0"]
+        Wb = W[:, perm[p0:p0 + kb]].astype(np.float64)
+        o, sb = blk["seg_off"], blk["seg_bytes"]
+        if b == 16:
+            h = np.ascontiguousarray(Wb.astype(np.float16)).view("<u2").view(np.uint8)
+            packed[:, o:o + h.shape[1]] = h
+            continue
+        sc, ze, q = quantize_rows(Wb, b)
+        packed[:, o:o + sb] = pack_codes(q, b, sb)
+        g0, ng = blk["grp_off"], blk["n_grp"]
+        meta[:, g0:g0 + ng, 0] = sc.astype(np.float16).view(np.uint16)
+        meta[:, g0:g0 + ng, 1] = ze.astype(np.float16).view(np.uint16)
+    return dict(N=N, K=K, bits=bits, perm=perm, blocks=blocks, row_stride=S,
+                n_groups=G, packed=packed, meta=meta,
+                out_perm=np.arange(N, dtype=np.int64), B=float(B))
+
+
+def realized_budget(layer):
+    """B_real = mean width over the input channels (§3.3)."""
+    return float(np.mean(layer["bits"]))
+
+
+def unpack_codes(layer):
+    """Integer codes [N][K] in clustered order from the packed bytes.
+
+    For 16-bit positions the value is the fp16 bit pattern."""
+    N, K = layer["N"], layer["K"]
+    out = np.zeros((N, K), dtype=np.int64)
+    for blk in layer["blocks"]:
+        b, kb, p0 = blk["bits"], blk["n_ch"], blk["pos0"]
+        o, sb = blk["seg_off"], blk["seg_bytes"]
+        seg = layer["packed"][:, o:o + sb]
+        if b == 16:
+            out[:, p0:p0 + kb] = seg[:, : 2 * kb].copy().view("<u2").astype(np.int64)
+        else:
+            out[:, p0:p0 + kb] = unpack_codes_from_bytes(seg, b, kb)
+    return out
+
+
+def dequant(layer):
+    """Dequantised clustered weights W'[N][K] (fp64) from the packed bytes:
+    (q - z) * s for b < 16, the stored fp16 value for b = 16 (R1)."""
+    N, K = layer["N"], layer["K"]
+    codes = unpack_codes(layer)
+    Wd = np.zeros((N, K), dtype=np.float64)
+    meta = layer["meta"]
+    for blk in layer["blocks"]:
+        b, kb, p0 = blk["bits"], blk["n_ch"], blk["pos0"]
+        c = codes[:, p0:p0 + kb]
+        if b == 16:
+            Wd[:, p0:p0 + kb] = c.astype(np.uint16).view(np.float16).astype(np.float64)
+            continue
+        g0 = blk["grp_off"]
+        for g in range(blk["n_grp"]):
+            cols = slice(g * GROUP, min((g + 1) * GROUP, kb))
+            s = meta[:, g0 + g, 0].view(np.float16).astype(np.float64)
+            z = meta[:, g0 + g, 1].view(np.float16).astype(np.float64)
+            Wd[:, p0 + cols.start:p0 + cols.stop] = (c[:, cols] - z[:, None]) * s[:, None]
+    return Wd
+
+
+def gather_index(layer, producer_basis=None):
+    """r[p]: index into the producer-emitted activation for clustered
+    position p (R6).  With the natural basis this is ``perm``."""
+    perm = layer["perm"]
+    if producer_basis is None:
+        return perm.copy()
+    return permute_merge(producer_basis, perm)
+
+
+def linear(layer, x, gather=None):
+    """y[b][n'] = sum_p x[b][r[p]] * W'[row(n')][p] in fp64 (§4.1, R6).
+
+    ``x`` is [batch][K] (the activation in its producer's basis, values exact
+    in fp64), ``gather`` is r (default: ``perm``, natural producer basis).
+    Rows come out in the layer's current output basis (``out_perm``)."""
+    x = np.atleast_2d(np.asarray(x, dtype=np.float64))
+    r = layer["perm"] if gather is None else np.asarray(gather)
+    xs = x[:, r]
+    return xs @ dequant(layer).T
+
+
+def linear_natural(layer, x):
+    """The same product written without the permutation: W' is scattered
+    back to original channel order and x is used as is (§4.1 identity)."""
+    x = np.atleast_2d(np.asarray(x, dtype=np.float64))
+    Wc = dequant(layer)
+    Wn = np.zeros_like(Wc)
+    Wn[:, layer["perm"]] = Wc
+    return x @ Wn.T
+
+
+# ---------------------------------------------------------------------------
+# §4.3 (R6): permutation merge
+# ---------------------------------------------------------------------------
+def _check_perm(p, n):
+    p = np.asarray(p, dtype=np.int64)
+    if p.shape != (n,) or not np.array_equal(np.sort(p), np.arange(n)):
+        raise ValueError("not a permutation of 0..n-1")
+    return p
+
+
+def permute_merge(producer_basis, consumer_perm):
+    """r = beta^-1 o P_c: r[p] = beta^-1[consumer_perm[p]] (§4.3, R6)."""
+    n = len(consumer_perm)
+    beta = _check_perm(producer_basis, n)
+    pc = _check_perm(consumer_perm, n)
+    inv = np.empty(n, dtype=np.int64)
+    inv[beta] = np.arange(n)
+    return inv[pc]
+
+
+def permute_rows(layer, row_perm):
+    """Make the layer emit output i = y_orig[out_perm[row_perm[i]]] by moving
+    whole packed rows and their metadata (§4.3: compile-time permutation of
+    the producer's output channels)."""
+    rp = _check_perm(row_perm, layer["N"])
+    out = dict(layer)
+    out["packed"] = layer["packed"][rp].copy()
+    out["meta"] = layer["meta"][rp].copy()
+    out["out_perm"] = layer["out_perm"][rp].copy()
+    return out
+
+
+# ---------------------------------------------------------------------------
+# §5.3: reorder-traffic model
+# ---------------------------------------------------------------------------
+def reorder_traffic_bytes(gathered_k, n_layers):
+    """Per-token A16 read+write bytes of explicit activation shuffles: each
+    shuffled activation of K channels costs 2 bytes read + 2 bytes written
+    per channel (§5.3)."""
+    return 4 * int(sum(gathered_k)) * int(n_layers)
+
+
+def llama_layer_linears(hidden, ffn):
+    """(name, N, K) of the seven linears of one Llama-style decoder layer."""
+    return [("q", hidden, hidden), ("k", hidden, hidden), ("v", hidden, hidden),
+            ("o", hidden, hidden), ("gate", ffn, hidden), ("up", ffn, hidden),
+            ("down", hidden, ffn)]
+
+
+# ---------------------------------------------------------------------------
+# decode-step reference for a Llama-shaped stack (the per-layer graph)
+# ---------------------------------------------------------------------------
+def bf16_rn(v):
+    """Round fp64 to bf16 (ties to even) via fp32, returned as fp64.
+
+    Used only where the decode-step graph stores an activation in bf16; the
+    fp64 -> fp32 -> bf16 order is the graph's definition, not a shortcut."""
+    f = np.asarray(v, dtype=np.float64).astype(np.float32)
+    u = f.view(np.uint32).astype(np.uint64)
+    r = ((u + 0x7FFF + ((u >> 16) & 1)) >> 16) << 16
+    return r.astype(np.uint32).view(np.float32).astype(np.float64)
+
+
+def rmsnorm(s, eps=1e-6):
+    s = np.asarray(s, dtype=np.float64)
+    return s / np.sqrt(np.mean(s * s, axis=-1, keepdims=True) + eps)
+
+
+def silu(v):
+    v = np.asarray(v, dtype=np.float64)
+    return v / (1.0 + np.exp(-v))
