@@ -1,0 +1,210 @@
+/*
+ * polyq.h - C ABI of the PolyQ mixed-bit linear layer for GB300 (sm_103a).
+ *
+ * PolyQ (arXiv 2607.14618) gives every input channel of a linear layer
+ * y = x W^T a width from {2,3,4,8,16} under a fractional average budget B
+ * (Section 3), permutes the channels into bit-homogeneous blocks (Section 4.1
+ * and 4.2) and folds consumer permutations into producer output rows
+ * (Section 4.3).  This library packs a layer on the host and runs the layer
+ * on the GPU.
+ *
+ * Conventions for every call:
+ *   - Return value: 0 (POLYQ_OK) on success, a negative POLYQ_E* code
+ *     otherwise; polyq_last_error() then returns a message (thread-local,
+ *     valid until the next call on the same thread).
+ *   - The caller owns every buffer passed in.  Host buffers are read during
+ *     the call only.  Device buffers must stay valid until the work queued on
+ *     `stream` has finished.
+ *   - GPU entry points never allocate device memory and never synchronise:
+ *     they validate arguments on the host, then enqueue kernels on `stream`
+ *     (a cudaStream_t passed as void*; NULL = legacy default stream) and
+ *     return.  Launch errors are reported as POLYQ_ECUDA.
+ *   - Device pointers must be 16-byte aligned unless stated otherwise.
+ *
+ * Packed format of one layer (host and device identical):
+ *   widths   bits[K]        (original channel order)
+ *   perm     int32 perm[K]: clustered position p holds original channel
+ *            perm[p]; blocks in ascending width, channels ascending in a
+ *            block (Section 4.1: only P_W W is materialised).
+ *   blocks   at most 5, one per width present, ascending.
+ *   packed   uint8 [N][row_stride]: per row the concatenation of one segment
+ *            per block.  A b<16 segment is an LSB-first bitstream (code p of
+ *            the block at bits [p*b, p*b+b), little-endian bytes); a 16-bit
+ *            segment holds little-endian fp16 weights.  Segments are padded
+ *            with zeros to a multiple of 16 bytes.
+ *   meta     uint32 [N][n_groups]: per row and per 64-position group of a
+ *            b<16 block (groups ordered by block, then position; the last
+ *            group of a block may be shorter) the fp16 scale in bits 0..15
+ *            and the fp16 zero point (an integer) in bits 16..31.
+ *   Dequantised weight: w' = (q - zero) * scale for b<16; the fp16 value for
+ *   b=16.  Quantiser: lo/hi = min/max of the group, scale =
+ *   fp16_rn((hi-lo)/(2^b-1)) (if 0: fp16_rn(max(|lo|,|hi|,2^-14))),
+ *   zero = clamp(rint(-lo/scale), 0, 2^b-1), q = clamp(rint(w/scale)+zero).
+ */
+#ifndef POLYQ_H
+#define POLYQ_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define POLYQ_OK 0
+#define POLYQ_EINVAL (-1)       /* bad argument, shape, alignment, permutation */
+#define POLYQ_ENOMEM (-2)       /* host allocation failed / workspace too small */
+#define POLYQ_ECUDA (-3)        /* a CUDA runtime call or launch failed */
+#define POLYQ_EUNSUPPORTED (-4) /* option or size this build does not handle */
+#define POLYQ_ETIMEOUT (-5)     /* a bounded device-side wait gave up */
+
+#define POLYQ_MAX_BLOCKS 5
+#define POLYQ_GROUP 64
+
+#define POLYQ_ALLOC_WATERFILL 0 /* Section 3.2 max-heap waterfilling (default) */
+#define POLYQ_ALLOC_LADDER 1    /* descending saliency, each channel climbs */
+
+/* Options of polyq_pack.  Zero-initialise, then set what you need;
+ * polyq_pack_opts_default() gives the defaults. */
+typedef struct {
+  int32_t group_size;        /* must be 64 */
+  uint32_t palette_mask;     /* bit b set: width b allowed (b in 2,3,4,8,16);
+                                0 means all five */
+  int32_t alloc_rule;        /* POLYQ_ALLOC_WATERFILL or POLYQ_ALLOC_LADDER */
+  int32_t snap_quanta;       /* must be 0 (quanta matching not built) */
+  int32_t n_threads;         /* host threads, 0 = hardware concurrency */
+  const uint8_t* forced_bits;/* optional [K] width map; skips allocation */
+} polyq_pack_opts;
+
+/* One bit-homogeneous block (Section 4.2). */
+typedef struct {
+  int32_t bits;      /* 2, 3, 4, 8 or 16 */
+  int32_t n_ch;      /* channels in the block (K_b) */
+  int32_t pos0;      /* first clustered position */
+  int32_t seg_off;   /* byte offset of the block's segment inside a row */
+  int32_t seg_bytes; /* segment bytes per row (multiple of 16) */
+  int32_t grp_off;   /* first meta group of the block */
+  int32_t n_grp;     /* ceil(n_ch/64) for b<16, 0 for b=16 */
+} polyq_block;
+
+typedef struct {
+  int64_t N, K;          /* out x in */
+  int64_t row_stride;    /* bytes per packed row */
+  int64_t n_groups;      /* meta entries per row */
+  int32_t n_blocks;
+  polyq_block blocks[POLYQ_MAX_BLOCKS];
+  double budget;         /* requested B */
+  double b_real;         /* realised mean width (Section 3.3, B_real) */
+  int64_t packed_bytes;  /* N * row_stride */
+  int64_t meta_bytes;    /* N * n_groups * 4 */
+} polyq_info;
+
+/* A packed layer resident on the device.  Filled by polyq_dev_layer_fill()
+ * (or by hand).  The library only reads it. */
+typedef struct {
+  const uint8_t* packed;  /* device [N][row_stride], 16-byte aligned */
+  const uint32_t* meta;   /* device [N][n_groups], 16-byte aligned */
+  const int32_t* gather;  /* device [K]: xs[p] = x[gather[p]]; NULL = identity
+                             (a merged edge, Section 4.3) */
+  int64_t N, K, row_stride, n_groups;
+  int32_t n_blocks;
+  polyq_block blocks[POLYQ_MAX_BLOCKS];
+} polyq_dev_layer;
+
+typedef struct polyq_layer polyq_layer; /* opaque host-side packed layer */
+
+const char* polyq_last_error(void);
+void polyq_pack_opts_default(polyq_pack_opts* opts);
+
+/* Allocate widths, cluster and pack one layer (Sections 3.1, 3.2, 4.1, 4.2).
+ * W: host fp32 [N][K] row-major (out x in), finite, |W| <= 65504.
+ * act_absmean: host fp32 [K], per-input-channel activation magnitude used for
+ * the saliency a_k * ||W[:,k]||_2 (Section 3.1 error proxy, E_16 = 0).
+ * budget_bits: average width B in [2, 16] (Section 3.2).
+ * Greedy waterfilling: all channels start at the narrowest palette width,
+ * Delta = round(B*K) - b_min*K, upgrades popped from a max-heap by gain per
+ * extra bit (ties: lower channel first); a step that does not fit is dropped.
+ * On success *out owns a new layer (free with polyq_free). */
+int polyq_pack(const float* W, int64_t N, int64_t K, const float* act_absmean,
+               double budget_bits, const polyq_pack_opts* opts,
+               polyq_layer** out);
+
+void polyq_free(polyq_layer* layer);
+
+/* Shape, blocks and byte counts of a packed layer. */
+int polyq_layer_info(const polyq_layer* layer, polyq_info* out);
+
+/* Copy the packed layer into caller buffers (each may be NULL to skip):
+ * packed [N*row_stride] bytes, meta [N*n_groups] uint32, perm [K] int32,
+ * bits [K] uint8 (original channel order), out_perm [N] int32 (the layer
+ * emits output i = y_original[out_perm[i]]). */
+int polyq_layer_export(const polyq_layer* layer, uint8_t* packed,
+                       uint32_t* meta, int32_t* perm, uint8_t* bits,
+                       int32_t* out_perm);
+
+/* Section 4.3 merge, producer side: permute whole output rows (packed bytes
+ * and meta) so that afterwards the layer emits
+ * new_output[i] = old_output[row_perm[i]].  row_perm: host int32 [N], a
+ * permutation.  Passing a consumer's perm makes the producer emit in the
+ * consumer's clustered basis, so the consumer's gather becomes identity. */
+int polyq_layer_permute_rows(polyq_layer* layer, const int32_t* row_perm);
+
+/* Section 4.3 merge rule, index side: gather_out[p] =
+ * producer_basis^-1[consumer_perm[p]] where the producer emits
+ * emitted[i] = y[producer_basis[i]].  All arrays host int32 [n]; both inputs
+ * must be permutations.  The consumer then reads xs[p] = emitted[gather[p]]. */
+int polyq_permute_merge(const int32_t* producer_basis,
+                        const int32_t* consumer_perm, int64_t n,
+                        int32_t* gather_out);
+
+/* Fill a device-layer descriptor from a host layer and the device copies of
+ * its packed bytes and meta (uploaded by the caller from polyq_layer_export)
+ * and an optional device gather vector (NULL = identity). */
+int polyq_dev_layer_fill(const polyq_layer* layer, const uint8_t* packed_dev,
+                         const uint32_t* meta_dev, const int32_t* gather_dev,
+                         polyq_dev_layer* out);
+
+/* Device scratch bytes polyq_linear_gemv needs for this layer and batch. */
+int polyq_gemv_workspace_bytes(const polyq_dev_layer* layer, int batch,
+                               size_t* bytes);
+
+/* Decode GEMV (Section 4.1 factorisation; Section 4.2 blocks in one launch):
+ *   y[b][n] = residual[b][n] + sum_p x[b][gather[p]] * W'[n][p]
+ * x: device bf16 [batch][K] (the activation in its producer's basis);
+ * batch in 1..4; y: device fp32 [batch][N]; residual: device fp32
+ * [batch][N] or NULL (y may alias residual); workspace: device scratch of at
+ * least polyq_gemv_workspace_bytes(), 256-byte aligned, not shared with any
+ * concurrently running call.  Accumulation is fp32. */
+int polyq_linear_gemv(const polyq_dev_layer* layer, const void* x, int batch,
+                      float* y, const float* residual, void* workspace,
+                      size_t workspace_bytes, void* stream);
+
+/* Device scratch bytes polyq_linear_gemm needs for this layer and M. */
+int polyq_gemm_workspace_bytes(const polyq_dev_layer* layer, int64_t M,
+                               size_t* bytes);
+
+/* Prefill GEMM (the same product for M tokens, Section 5.4 prefill):
+ *   Y[m][n] = sum_p X[m][gather[p]] * W'[n][p]
+ * X: device bf16 [M][K]; Y: device fp32 [M][N]; workspace as for the GEMV.
+ * Weights are dequantised to fp16 tiles in shared memory and multiplied on
+ * the tcgen05 tensor cores with fp32 accumulation in tensor memory.  X is
+ * gathered and converted to fp16 first, so |X| must stay within the fp16
+ * range (65504); the product is then within fp16 rounding of each weight. */
+int polyq_linear_gemm(const polyq_dev_layer* layer, const void* X, int64_t M,
+                      float* Y, void* workspace, size_t workspace_bytes,
+                      void* stream);
+
+/* Test aid: unpack the integer codes of every row into codes [N][K]
+ * (device uint16, clustered order; for 16-bit channels the fp16 bit pattern).
+ * Must equal the host-side codes bit for bit. */
+int polyq_unpack_codes(const polyq_dev_layer* layer, uint16_t* codes,
+                       void* stream);
+
+/* Utility: round a double to the nearest fp16 (ties to even); returns the
+ * fp16 bit pattern.  The packer's scale rounding. */
+uint16_t polyq_f64_to_f16(double v);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* POLYQ_H */

@@ -1,0 +1,283 @@
+"""ctypes binding of ``libpolyq.so`` (the C ABI declared in include/polyq.h).
+
+Argument marshalling only: every step of the layer runs in the library.
+PyTorch supplies device memory and the current CUDA stream.  Importing this
+module fails loudly when the library has not been built.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libpolyq.so")
+
+POLYQ_OK = 0
+POLYQ_EINVAL = -1
+POLYQ_ENOMEM = -2
+POLYQ_ECUDA = -3
+POLYQ_EUNSUPPORTED = -4
+POLYQ_ETIMEOUT = -5
+MAX_BLOCKS = 5
+GROUP = 64
+ALLOC_WATERFILL = 0
+ALLOC_LADDER = 1
+
+if not os.path.exists(LIB_PATH):
+    raise ImportError(f"{LIB_PATH} is missing: build it with paper_2607_14618_gb300.build.build_library()")
+_lib = C.CDLL(LIB_PATH)
+
+
+class PolyqError(RuntimeError):
+    def __init__(self, code, msg):
+        super().__init__(f"[{code}] {msg}")
+        self.code = code
+
+
+class PackOpts(C.Structure):
+    _fields_ = [("group_size", C.c_int32), ("palette_mask", C.c_uint32),
+                ("alloc_rule", C.c_int32), ("snap_quanta", C.c_int32),
+                ("n_threads", C.c_int32), ("forced_bits", C.POINTER(C.c_uint8))]
+
+
+class Block(C.Structure):
+    _fields_ = [("bits", C.c_int32), ("n_ch", C.c_int32), ("pos0", C.c_int32),
+                ("seg_off", C.c_int32), ("seg_bytes", C.c_int32), ("grp_off", C.c_int32),
+                ("n_grp", C.c_int32)]
+
+    def as_dict(self):
+        return {f: getattr(self, f) for f, _ in self._fields_}
+
+
+class Info(C.Structure):
+    _fields_ = [("N", C.c_int64), ("K", C.c_int64), ("row_stride", C.c_int64),
+                ("n_groups", C.c_int64), ("n_blocks", C.c_int32),
+                ("blocks", Block * MAX_BLOCKS), ("budget", C.c_double), ("b_real", C.c_double),
+                ("packed_bytes", C.c_int64), ("meta_bytes", C.c_int64)]
+
+
+class DevLayer(C.Structure):
+    _fields_ = [("packed", C.c_void_p), ("meta", C.c_void_p), ("gather", C.c_void_p),
+                ("N", C.c_int64), ("K", C.c_int64), ("row_stride", C.c_int64),
+                ("n_groups", C.c_int64), ("n_blocks", C.c_int32),
+                ("blocks", Block * MAX_BLOCKS)]
+
+
+_P = C.c_void_p
+_SIGS = {
+    "polyq_last_error": (C.c_char_p, []),
+    "polyq_pack_opts_default": (None, [C.POINTER(PackOpts)]),
+    "polyq_pack": (C.c_int, [_P, C.c_int64, C.c_int64, _P, C.c_double, C.POINTER(PackOpts),
+                             C.POINTER(C.c_void_p)]),
+    "polyq_free": (None, [_P]),
+    "polyq_layer_info": (C.c_int, [_P, C.POINTER(Info)]),
+    "polyq_layer_export": (C.c_int, [_P, _P, _P, _P, _P, _P]),
+    "polyq_layer_permute_rows": (C.c_int, [_P, _P]),
+    "polyq_permute_merge": (C.c_int, [_P, _P, C.c_int64, _P]),
+    "polyq_dev_layer_fill": (C.c_int, [_P, _P, _P, _P, C.POINTER(DevLayer)]),
+    "polyq_gemv_workspace_bytes": (C.c_int, [C.POINTER(DevLayer), C.c_int, C.POINTER(C.c_size_t)]),
+    "polyq_linear_gemv": (C.c_int, [C.POINTER(DevLayer), _P, C.c_int, _P, _P, _P, C.c_size_t, _P]),
+    "polyq_gemm_workspace_bytes": (C.c_int, [C.POINTER(DevLayer), C.c_int64,
+                                             C.POINTER(C.c_size_t)]),
+    "polyq_linear_gemm": (C.c_int, [C.POINTER(DevLayer), _P, C.c_int64, _P, _P, C.c_size_t, _P]),
+    "polyq_unpack_codes": (C.c_int, [C.POINTER(DevLayer), _P, _P]),
+    "polyq_f64_to_f16": (C.c_uint16, [C.c_double]),
+}
+for _name, (_res, _args) in _SIGS.items():
+    _fn = getattr(_lib, _name)
+    _fn.restype = _res
+    _fn.argtypes = _args
+
+
+def exported_symbols():
+    """Names of the C-ABI entry points this binding expects."""
+    return list(_SIGS)
+
+
+def _check(rc):
+    if rc != POLYQ_OK:
+        raise PolyqError(rc, _lib.polyq_last_error().decode())
+
+
+def last_error():
+    return _lib.polyq_last_error().decode()
+
+
+def f64_to_f16(v: float) -> int:
+    return int(_lib.polyq_f64_to_f16(float(v)))
+
+
+def permute_merge(producer_basis, consumer_perm):
+    """gather[p] = producer_basis^-1[consumer_perm[p]] (merge rule, index side)."""
+    b = np.ascontiguousarray(producer_basis, dtype=np.int32)
+    c = np.ascontiguousarray(consumer_perm, dtype=np.int32)
+    if b.shape != c.shape or b.ndim != 1:
+        raise ValueError("shape mismatch")
+    out = np.empty_like(c)
+    _check(_lib.polyq_permute_merge(b.ctypes.data, c.ctypes.data, c.shape[0], out.ctypes.data))
+    return out
+
+
+def _palette_mask(palette):
+    m = 0
+    for b in palette:
+        m |= 1 << int(b)
+    return m
+
+
+class HostLayer:
+    """A packed layer owned by the library (host memory)."""
+
+    def __init__(self, handle):
+        self._h = C.c_void_p(handle)
+
+    @classmethod
+    def pack(cls, W, act_absmean=None, budget=3.0, forced_bits=None,
+             rule=ALLOC_WATERFILL, palette=(2, 3, 4, 8, 16), n_threads=0):
+        W = np.ascontiguousarray(W, dtype=np.float32)
+        if W.ndim != 2:
+            raise ValueError("W must be [N][K]")
+        N, K = W.shape
+        opts = PackOpts()
+        _lib.polyq_pack_opts_default(C.byref(opts))
+        opts.alloc_rule = int(rule)
+        opts.palette_mask = _palette_mask(palette)
+        opts.n_threads = int(n_threads)
+        keep = None
+        if forced_bits is not None:
+            keep = np.ascontiguousarray(forced_bits, dtype=np.uint8)
+            if keep.shape != (K,):
+                raise ValueError("forced_bits must be [K]")
+            opts.forced_bits = keep.ctypes.data_as(C.POINTER(C.c_uint8))
+        a = None
+        if act_absmean is not None:
+            a = np.ascontiguousarray(act_absmean, dtype=np.float32)
+            if a.shape != (K,):
+                raise ValueError("act_absmean must be [K]")
+        h = C.c_void_p()
+        _check(_lib.polyq_pack(W.ctypes.data, N, K, a.ctypes.data if a is not None else None,
+                               float(budget), C.byref(opts), C.byref(h)))
+        return cls(h.value)
+
+    def __del__(self):
+        if getattr(self, "_h", None) and self._h.value:
+            _lib.polyq_free(self._h)
+            self._h = C.c_void_p()
+
+    def info(self) -> dict:
+        inf = Info()
+        _check(_lib.polyq_layer_info(self._h, C.byref(inf)))
+        d = {f: getattr(inf, f) for f, _ in Info._fields_ if f != "blocks"}
+        d["blocks"] = [inf.blocks[i].as_dict() for i in range(inf.n_blocks)]
+        return d
+
+    def export(self) -> dict:
+        inf = self.info()
+        N, K, S, G = inf["N"], inf["K"], inf["row_stride"], inf["n_groups"]
+        packed = np.empty((N, S), np.uint8)
+        meta = np.empty((N, G), np.uint32)
+        perm = np.empty(K, np.int32)
+        bits = np.empty(K, np.uint8)
+        out_perm = np.empty(N, np.int32)
+        _check(_lib.polyq_layer_export(self._h, packed.ctypes.data, meta.ctypes.data,
+                                       perm.ctypes.data, bits.ctypes.data, out_perm.ctypes.data))
+        return dict(info=inf, packed=packed, meta=meta, perm=perm, bits=bits, out_perm=out_perm)
+
+    def permute_rows(self, row_perm):
+        rp = np.ascontiguousarray(row_perm, dtype=np.int32)
+        _check(_lib.polyq_layer_permute_rows(self._h, rp.ctypes.data))
+
+
+class DeviceLayer:
+    """Device copy of a packed layer (torch tensors) and its descriptor."""
+
+    def __init__(self, host: HostLayer, device="cuda", gather=None, identity_gather=False):
+        import torch
+        ex = host.export()
+        self.info = ex["info"]
+        self.perm = ex["perm"]
+        self.out_perm = ex["out_perm"]
+        self.packed = torch.from_numpy(ex["packed"]).to(device)
+        self.meta = torch.from_numpy(ex["meta"].view(np.int32)).to(device)
+        if identity_gather:
+            self.gather = None
+        else:
+            g = ex["perm"] if gather is None else np.ascontiguousarray(gather, np.int32)
+            self.gather = torch.from_numpy(np.ascontiguousarray(g, np.int32)).to(device)
+        self.desc = DevLayer()
+        _check(_lib.polyq_dev_layer_fill(
+            host._h, self.packed.data_ptr(), self.meta.data_ptr() if self.meta.numel() else None,
+            self.gather.data_ptr() if self.gather is not None else None, C.byref(self.desc)))
+        self.N = self.info["N"]
+        self.K = self.info["K"]
+
+    def packed_bytes(self):
+        return self.info["packed_bytes"] + self.info["meta_bytes"]
+
+
+def _stream_ptr(stream):
+    import torch
+    s = torch.cuda.current_stream() if stream is None else stream
+    return C.c_void_p(s.cuda_stream)
+
+
+def gemv_workspace_bytes(layer: DeviceLayer, batch: int) -> int:
+    n = C.c_size_t()
+    _check(_lib.polyq_gemv_workspace_bytes(C.byref(layer.desc), int(batch), C.byref(n)))
+    return n.value
+
+
+def linear_gemv(layer: DeviceLayer, x, y=None, residual=None, workspace=None, stream=None):
+    """y[b][n] = residual[b][n] + sum_p x[b][gather[p]] W'[n][p] (device tensors)."""
+    import torch
+    if x.dtype != torch.bfloat16 or not x.is_cuda or x.dim() != 2 or x.shape[1] != layer.K:
+        raise ValueError("x must be a CUDA bf16 tensor [batch][K]")
+    x = x.contiguous()
+    batch = x.shape[0]
+    if y is None:
+        y = torch.empty((batch, layer.N), dtype=torch.float32, device=x.device)
+    ws_need = gemv_workspace_bytes(layer, batch)
+    if workspace is None and ws_need:
+        workspace = torch.empty(ws_need, dtype=torch.uint8, device=x.device)
+    ws_ptr = workspace.data_ptr() if workspace is not None else None
+    ws_len = workspace.numel() if workspace is not None else 0
+    _check(_lib.polyq_linear_gemv(C.byref(layer.desc), x.data_ptr(), batch, y.data_ptr(),
+                                  residual.data_ptr() if residual is not None else None,
+                                  ws_ptr, ws_len, _stream_ptr(stream)))
+    return y
+
+
+def gemm_workspace_bytes(layer: DeviceLayer, M: int) -> int:
+    n = C.c_size_t()
+    _check(_lib.polyq_gemm_workspace_bytes(C.byref(layer.desc), int(M), C.byref(n)))
+    return n.value
+
+
+def linear_gemm(layer: DeviceLayer, X, Y=None, workspace=None, stream=None):
+    """Y[m][n] = sum_p X[m][gather[p]] W'[n][p] (device tensors)."""
+    import torch
+    if X.dtype != torch.bfloat16 or not X.is_cuda or X.dim() != 2 or X.shape[1] != layer.K:
+        raise ValueError("X must be a CUDA bf16 tensor [M][K]")
+    X = X.contiguous()
+    M = X.shape[0]
+    if Y is None:
+        Y = torch.empty((M, layer.N), dtype=torch.float32, device=X.device)
+    ws_need = gemm_workspace_bytes(layer, M)
+    if workspace is None and ws_need:
+        workspace = torch.empty(ws_need, dtype=torch.uint8, device=X.device)
+    ws_ptr = workspace.data_ptr() if workspace is not None else None
+    ws_len = workspace.numel() if workspace is not None else 0
+    _check(_lib.polyq_linear_gemm(C.byref(layer.desc), X.data_ptr(), M, Y.data_ptr(),
+                                  ws_ptr, ws_len, _stream_ptr(stream)))
+    return Y
+
+
+def unpack_codes(layer: DeviceLayer, stream=None):
+    """Device-unpacked integer codes [N][K] (clustered order) as numpy uint16."""
+    import torch
+    out = torch.empty((layer.N, layer.K), dtype=torch.int16, device=layer.packed.device)
+    _check(_lib.polyq_unpack_codes(C.byref(layer.desc), out.data_ptr(), _stream_ptr(stream)))
+    torch.cuda.synchronize()
+    return out.cpu().numpy().view(np.uint16)

@@ -1,0 +1,205 @@
+"""Host-side parity: the library's packer (C++) against the oracle (NumPy),
+bit for bit, plus the C-ABI surface and argument validation.  No GPU."""
+import ctypes as C
+import os
+import re
+
+import numpy as np
+import pytest
+
+from oracle import polyq_oracle as O
+from paper_2607_14618_gb300 import synth
+
+HEADER = os.path.join(os.path.dirname(os.path.dirname(__file__)), "include", "polyq.h")
+
+
+def _declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(polyq_[a-z0-9_]+)\s*\(", text)))
+
+
+def test_library_exports_every_declared_symbol(polyq_lib):
+    names = _declared_functions()
+    assert len(names) >= 15
+    lib = C.CDLL(polyq_lib.LIB_PATH)
+    for n in names:
+        assert hasattr(lib, n), n
+    assert set(names) <= set(polyq_lib.exported_symbols())
+
+
+def test_f64_to_f16_matches_numpy(polyq_lib):
+    rng = np.random.default_rng(0)
+    vals = list(rng.normal(0, 1, 2000) * 10.0 ** rng.integers(-9, 5, 2000))
+    vals += [0.0, -0.0, 1.0, 65504.0, 65519.99, 2.0 ** -24, 2.0 ** -25, 3 * 2.0 ** -26,
+             2.0 ** -14, 2.0 ** -14 - 2.0 ** -25, 1 + 2.0 ** -11, 1 + 2.0 ** -11 + 2.0 ** -40,
+             1 + 3 * 2.0 ** -11, 6.1e-5, 0.0123]
+    for v in vals:
+        got = polyq_lib.f64_to_f16(v)
+        ref = int(np.array([v], np.float64).astype(np.float16).view(np.uint16)[0])
+        assert got == ref, (v, hex(got), hex(ref))
+
+
+def _compare(host, ref):
+    ex = host.export()
+    inf = ex["info"]
+    assert inf["N"] == ref["N"] and inf["K"] == ref["K"]
+    assert np.array_equal(ex["bits"], ref["bits"].astype(np.uint8))
+    assert np.array_equal(ex["perm"], ref["perm"].astype(np.int32))
+    assert inf["row_stride"] == ref["row_stride"] and inf["n_groups"] == ref["n_groups"]
+    assert inf["blocks"] == ref["blocks"]
+    assert np.array_equal(ex["packed"], ref["packed"])
+    meta_ref = ref["meta"][:, :, 0].astype(np.uint32) | (ref["meta"][:, :, 1].astype(np.uint32) << 16)
+    assert np.array_equal(ex["meta"], meta_ref)
+    assert inf["b_real"] == O.realized_budget(ref)
+
+
+@pytest.mark.parametrize("N,K,B,seed", [
+    (2048, 2048, 3.0, 1001),   # the 2048 x 2048, B = 3.0 decode layer
+    (64, 5120, 4.5, 2001),
+    (48, 5120, 6.0, 3003),
+    (96, 1000, 2.0, 5),
+    (33, 777, 2.7, 6),
+    (7, 129, 16.0, 7),
+    (5, 64, 3.3, 8),
+])
+def test_pack_matches_oracle(polyq_lib, N, K, B, seed):
+    W, a = synth.layer_weights(N, K, seed)
+    host = polyq_lib.HostLayer.pack(W, a, B)
+    _compare(host, O.pack_layer(W, a, B))
+
+
+@pytest.mark.parametrize("seed", [11, 12, 13])
+def test_pack_forced_widths_matches_oracle(polyq_lib, seed):
+    rng = np.random.default_rng(seed)
+    K = int(rng.integers(5, 700))
+    N = int(rng.integers(1, 40))
+    W, a = synth.layer_weights(N, K, seed)
+    bits = synth.random_codes_layer_bits(K, seed)
+    host = polyq_lib.HostLayer.pack(W, a, 3.0, forced_bits=bits)
+    _compare(host, O.pack_layer(W, a, 3.0, bits=bits))
+
+
+def test_pack_edge_weights_match_oracle(polyq_lib):
+    # constant groups, zeros, tiny and large magnitudes, fp16 subnormal scales
+    W = np.zeros((6, 200), np.float32)
+    W[1] = 1e-7
+    W[2] = np.linspace(-3e-6, 5e-6, 200, dtype=np.float32)
+    W[3] = 60000.0
+    W[4, ::3] = -65504.0
+    W[5] = np.random.default_rng(1).normal(0, 100, 200).astype(np.float32)
+    a = np.ones(200, np.float32)
+    bits = synth.random_codes_layer_bits(200, 4)
+    host = polyq_lib.HostLayer.pack(W, a, 3.0, forced_bits=bits)
+    _compare(host, O.pack_layer(W, a, 3.0, bits=bits))
+
+
+def test_ladder_and_palette_match_oracle(polyq_lib):
+    W, a = synth.layer_weights(40, 900, 21)
+    host = polyq_lib.HostLayer.pack(W, a, 3.4, rule=polyq_lib.ALLOC_LADDER)
+    ref_bits = O.allocate_bits(O.saliency(W, a), 3.4, rule=O.SALIENCY_LADDER)
+    assert np.array_equal(host.export()["bits"], ref_bits.astype(np.uint8))
+    host = polyq_lib.HostLayer.pack(W, a, 3.4, palette=(2, 4, 8))
+    ref_bits = O.allocate_bits(O.saliency(W, a), 3.4, palette=(2, 4, 8))
+    assert np.array_equal(host.export()["bits"], ref_bits.astype(np.uint8))
+
+
+def test_thread_count_does_not_change_result(polyq_lib):
+    W, a = synth.layer_weights(300, 1500, 9)
+    e1 = polyq_lib.HostLayer.pack(W, a, 3.7, n_threads=1).export()
+    e8 = polyq_lib.HostLayer.pack(W, a, 3.7, n_threads=8).export()
+    for k in ("packed", "meta", "perm", "bits"):
+        assert np.array_equal(e1[k], e8[k])
+
+
+def test_permute_merge_matches_oracle(polyq_lib):
+    rng = np.random.default_rng(3)
+    for n in (1, 5, 1000):
+        beta, pc = rng.permutation(n), rng.permutation(n)
+        assert np.array_equal(polyq_lib.permute_merge(beta, pc), O.permute_merge(beta, pc))
+    with pytest.raises(polyq_lib.PolyqError) as ei:
+        polyq_lib.permute_merge([0, 0, 2], [0, 1, 2])
+    assert ei.value.code == polyq_lib.POLYQ_EINVAL
+
+
+def test_permute_rows_matches_oracle(polyq_lib):
+    Wp, ap = synth.layer_weights(150, 80, 41)
+    host = polyq_lib.HostLayer.pack(Wp, ap, 3.0)
+    ref = O.pack_layer(Wp, ap, 3.0)
+    rp = np.random.default_rng(0).permutation(150)
+    host.permute_rows(rp)
+    ref = O.permute_rows(ref, rp)
+    _compare(host, ref)
+    assert np.array_equal(host.export()["out_perm"], ref["out_perm"])
+    with pytest.raises(polyq_lib.PolyqError):
+        host.permute_rows(np.zeros(150, np.int32))
+
+
+def test_pack_rejects_bad_arguments(polyq_lib):
+    W, a = synth.layer_weights(4, 16, 1)
+    for B in (1.9, 16.5, float("nan")):
+        with pytest.raises(polyq_lib.PolyqError) as ei:
+            polyq_lib.HostLayer.pack(W, a, B)
+        assert ei.value.code == polyq_lib.POLYQ_EINVAL
+    Wbad = W.copy()
+    Wbad[0, 0] = np.inf
+    with pytest.raises(polyq_lib.PolyqError):
+        polyq_lib.HostLayer.pack(Wbad, a, 3.0)
+    Wbad[0, 0] = 70000.0
+    with pytest.raises(polyq_lib.PolyqError):
+        polyq_lib.HostLayer.pack(Wbad, a, 3.0)
+    with pytest.raises(polyq_lib.PolyqError):
+        polyq_lib.HostLayer.pack(W, a, 3.0, forced_bits=np.full(16, 5))
+    with pytest.raises(polyq_lib.PolyqError):
+        polyq_lib.HostLayer.pack(W, a, 3.0, palette=(5,))
+
+
+def _desc_from(polyq_lib, host):
+    """A descriptor with fake (never dereferenced) aligned device addresses."""
+    d = polyq_lib.DevLayer()
+    rc = polyq_lib._lib.polyq_dev_layer_fill(host._h, C.c_void_p(0x100000), C.c_void_p(0x200000),
+                                            None, C.byref(d))
+    assert rc == 0
+    return d
+
+
+def test_corrupt_descriptors_rejected_before_launch(polyq_lib):
+    """Host-side fault injection: every corrupted descriptor is refused with
+    POLYQ_EINVAL before any device work is queued."""
+    W, a = synth.layer_weights(8, 300, 2)
+    host = polyq_lib.HostLayer.pack(W, a, 3.0, forced_bits=synth.random_codes_layer_bits(300, 2))
+    L = polyq_lib._lib
+
+    def gemv(d, batch=1):
+        return L.polyq_linear_gemv(C.byref(d), C.c_void_p(0x300000), batch, C.c_void_p(0x400000),
+                                   None, None, 0, None)
+
+    def mutate(f):
+        d = _desc_from(polyq_lib, host)
+        f(d)
+        return d
+
+    cases = [
+        lambda d: setattr(d, "row_stride", d.row_stride + 8),
+        lambda d: setattr(d, "K", d.K + 1),
+        lambda d: setattr(d, "N", 0),
+        lambda d: setattr(d, "n_blocks", 0),
+        lambda d: setattr(d, "n_blocks", 6),
+        lambda d: setattr(d, "packed", 0x100001),
+        lambda d: setattr(d, "meta", None),
+        lambda d: setattr(d.blocks[1], "bits", 5),
+        lambda d: setattr(d.blocks[2], "n_ch", d.blocks[2].n_ch + 1),
+        lambda d: setattr(d.blocks[0], "seg_bytes", d.blocks[0].seg_bytes + 16),
+        lambda d: setattr(d.blocks[3], "grp_off", 0),
+        lambda d: setattr(d, "n_groups", d.n_groups - 1),
+    ]
+    for f in cases:
+        d = mutate(f)
+        assert gemv(d) == polyq_lib.POLYQ_EINVAL, polyq_lib.last_error()
+        codes_rc = L.polyq_unpack_codes(C.byref(d), C.c_void_p(0x500000), None)
+        assert codes_rc == polyq_lib.POLYQ_EINVAL
+    d = _desc_from(polyq_lib, host)
+    assert gemv(d, batch=0) == polyq_lib.POLYQ_EUNSUPPORTED
+    assert gemv(d, batch=5) == polyq_lib.POLYQ_EUNSUPPORTED
+    assert L.polyq_linear_gemv(C.byref(d), None, 1, C.c_void_p(0x400000), None, None, 0,
+                               None) == polyq_lib.POLYQ_EINVAL
