@@ -1,0 +1,402 @@
+"""Benchmark of the PolyQ mixed-bit linear layer on GB300.
+
+Default workload (one step): the seven decode linears of a Llama2-13B-shaped
+layer (q, k, v, o 5120x5120; gate, up 13824x5120; down 5120x13824), batch 1,
+average budget 3.0 bits, synthetic seeded weights and activations.  Each step
+runs the seven GEMVs through the library; the weights rotate over several
+device copies of the layer so that no step finds its weights in L2.
+
+Output: one JSON line (rank 0).  ``value`` is whole-job packed-layer bytes
+moved per second (TB/s) with inputs resident in HBM; ``e2e`` is the same
+metric through the public API with host<->device copies of each step's
+activations and results inside the timed region.
+
+``--impl reference`` times the CPU oracle on the host cores instead (a
+bounded sample of the same workload per step).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "mixed-bit GEMV HBM TB/s (% of peak) at 3.0b avg; prefill GEMM TFLOPS (% peak)"
+LLAMA = [("q", 5120, 5120), ("k", 5120, 5120), ("v", 5120, 5120), ("o", 5120, 5120),
+         ("gate", 13824, 5120), ("up", 13824, 5120), ("down", 5120, 13824)]
+WORKLOAD = ("llama2-13b decode linears q,k,v,o 5120x5120, gate,up 13824x5120, "
+            "down 5120x13824; batch 1; B=3.0")
+
+
+def _peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d.get("hbm_gbs", 6800.0), d.get("bf16_tflops", 1900.0), \
+            d.get("bf16_tflops_sustained", 1700.0), "measured"
+    return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi samples (200 ms) taken while the timed region runs."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.p = None
+
+    def __enter__(self):
+        try:
+            self.p = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.Q}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.p = None
+        return self
+
+    def __exit__(self, *a):
+        self.rows = []
+        if self.p is None:
+            return
+        self.p.terminate()
+        try:
+            out, _ = self.p.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.p.kill()
+            out, _ = self.p.communicate()
+        for line in out.splitlines():
+            f = [c.strip() for c in line.split(",")]
+            if len(f) >= 9:
+                self.rows.append(f)
+
+    def summary(self):
+        if not getattr(self, "rows", None):
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        sm = [float(r[1]) for r in self.rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in self.rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in self.rows for i in range(4)
+                          if r[5 + i].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons,
+                "samples": len(self.rows)}
+
+
+def _dist():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def build_layers(polyq, synth, budget, copies, device):
+    """Pack the seven linears once (seeded), upload, and clone on device."""
+    layers, xs, bytes_per_step = [], [], 0
+    hosts = []
+    for i, (name, N, K) in enumerate(LLAMA):
+        W, a = synth.layer_weights(N, K, synth.seed_for(2, i))
+        host = polyq.HostLayer.pack(W, a, budget)
+        dev = polyq.DeviceLayer(host, device)
+        xb, _ = synth.activations(a, 1, synth.seed_for(2, i))
+        xs.append(xb)
+        hosts.append((name, host.info()))
+        layers.append([dev] + [dev.clone() for _ in range(copies - 1)])
+        del W
+    return layers, xs, hosts
+
+
+def layer_bytes(info, batch):
+    """Algorithmic bytes of one GEMV launch: packed codes (incl. segment
+    padding) + scale/zero metadata + gathered activations + gather indices +
+    outputs."""
+    return (info["packed_bytes"] + info["meta_bytes"] + batch * info["K"] * 2
+            + info["K"] * 4 + batch * info["N"] * 4)
+
+
+def run_polyq(args):
+    import torch
+    import torch.distributed as dist
+
+    ws, rank, local = _dist()
+    if ws > 1:
+        dist.init_process_group("nccl", init_method="env://")
+    torch.cuda.set_device(local)
+    device = torch.device("cuda", local)
+    from paper_2607_14618_gb300 import build as _b
+    if rank == 0:
+        _b.build_library()
+    if ws > 1:
+        dist.barrier()
+    from paper_2607_14618_gb300 import polyq, synth
+
+    hbm, tf_burst, tf_sus, peak_kind = _peaks()
+    batch = args.batch
+    layers, xs_np, infos = build_layers(polyq, synth, args.budget, args.copies, device)
+    L2 = torch.cuda.get_device_properties(device).L2_cache_size
+    n_lin = len(LLAMA)
+    per_lin_bytes = [layer_bytes(inf, batch) for _, inf in infos]
+    step_bytes = sum(per_lin_bytes)
+    copy_bytes = sum(inf["packed_bytes"] + inf["meta_bytes"] for _, inf in infos)
+    xs = [torch.from_numpy(np.repeat(x, batch, 0).view(np.int16)).to(device).view(torch.bfloat16)
+          for x in xs_np]
+    ys = [torch.empty((batch, N), dtype=torch.float32, device=device) for _, N, _ in LLAMA]
+    wsz = max(polyq.gemv_workspace_bytes(layers[i][0], batch) for i in range(n_lin))
+    wbuf = torch.zeros(max(wsz, 256), dtype=torch.uint8, device=device)
+    kernels_per_gemv = polyq.gemv_launches_per_call(layers[0][0], batch)
+
+    stream = torch.cuda.Stream(device)
+    graphs, evs = [], []
+    torch.cuda.synchronize()
+    with torch.cuda.stream(stream):
+        for i in range(n_lin):  # warm the launch path once before capture
+            polyq.linear_gemv(layers[i][0], xs[i], y=ys[i], workspace=wbuf, stream=stream)
+    stream.synchronize()
+    for c in range(args.copies):
+        g = torch.cuda.CUDAGraph()
+        e = [torch.cuda.Event(enable_timing=True) for _ in range(n_lin + 1)]
+        with torch.cuda.graph(g, stream=stream):
+            e[0].record(stream)
+            for i in range(n_lin):
+                polyq.linear_gemv(layers[i][c], xs[i], y=ys[i], workspace=wbuf, stream=stream)
+                e[i + 1].record(stream)
+        graphs.append(g)
+        evs.append(e)
+    torch.cuda.synchronize()
+
+    for s in range(args.warmup):
+        graphs[s % args.copies].replay()
+    torch.cuda.synchronize()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    if ws > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        t0.record(stream)
+        for s in range(args.steps):
+            graphs[s % args.copies].replay()
+        t1.record(stream)
+        torch.cuda.synchronize()
+    if ws > 1:
+        dist.barrier()
+    ms = t0.elapsed_time(t1)
+    # per-launch durations: the last replay of each copy inside the timed region
+    lin_ms = [[evs[c][i].elapsed_time(evs[c][i + 1]) for c in range(min(args.copies, args.steps))]
+              for i in range(n_lin)]
+    if ws > 1:
+        t = torch.tensor([ms], device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    ms_step = ms / args.steps
+    value_tbs = ws * step_bytes * args.steps / (ms * 1e-3) / 1e12
+
+    # roofline of the dominant kernel (the GEMV): algorithmic bytes / duration
+    avg_ms = [statistics.mean(v) for v in lin_ms]
+    ach = sum(per_lin_bytes) / (sum(avg_ms) * 1e-3) / 1e9
+    roof = {"bound": "hbm", "achieved": round(ach, 1), "peak": hbm, "unit": "GB/s",
+            "frac": round(ach / hbm, 4), "traffic": None, "peak_kind": peak_kind,
+            "kernel": "polyq_linear_gemv", "per_linear_us": {LLAMA[i][0]: round(1e3 * avg_ms[i], 2)
+                                                            for i in range(n_lin)}}
+
+    # end to end through the public API: pinned host x -> device, GEMVs, y -> host
+    e2e = None
+    if not args.no_e2e:
+        hx = [torch.from_numpy(np.repeat(x, batch, 0).view(np.int16)).pin_memory() for x in xs_np]
+        hy = [torch.empty((batch, N), dtype=torch.float32).pin_memory() for _, N, _ in LLAMA]
+        dx = [torch.empty((batch, K), dtype=torch.int16, device=device) for _, _, K in LLAMA]
+        h2d = sum(t.numel() * 2 for t in hx)
+        d2h = sum(t.numel() * 4 for t in hy)
+        e_steps = max(3, min(args.steps, 50))
+        with torch.cuda.stream(stream):
+            for s in range(args.warmup + e_steps):
+                if s == args.warmup:
+                    stream.synchronize()
+                    ta = time.perf_counter()
+                c = s % args.copies
+                for i in range(n_lin):
+                    dx[i].copy_(hx[i], non_blocking=True)
+                    polyq.linear_gemv(layers[i][c], dx[i].view(torch.bfloat16), y=ys[i],
+                                      workspace=wbuf, stream=stream)
+                    hy[i].copy_(ys[i], non_blocking=True)
+                stream.synchronize()
+            tb = time.perf_counter()
+        e2e = {"value": round(step_bytes * e_steps / (tb - ta) / 1e12, 4), "unit": "TB/s",
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": e_steps,
+               "ms_per_step": round(1e3 * (tb - ta) / e_steps, 4)}
+
+    gemm = None
+    if not args.no_gemm:
+        gemm = bench_gemm(polyq, synth, torch, device, stream, args, tf_burst, tf_sus)
+
+    if rank == 0:
+        cpu = None if (args.no_cpu_baseline or ws > 1) else cpu_baseline(args.cpu_seconds)
+        out = {
+            "metric": METRIC, "value": round(value_tbs, 4), "unit": "TB/s", "n_gpus": ws,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_step, 5),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic",
+            "config": {"workload": WORKLOAD, "budget_bits": args.budget, "batch": batch,
+                       "parallelism": f"replicas{ws}" if ws > 1 else "single-gpu",
+                       "layer_copies": args.copies,
+                       "l2": f"weights rotate over {args.copies} device copies "
+                             f"({copy_bytes * args.copies / 2**20:.0f} MiB > L2 "
+                             f"{L2 / 2**20:.0f} MiB)",
+                       "bytes_per_step": step_bytes,
+                       "b_real": {n: round(inf["b_real"], 5) for n, inf in infos},
+                       "graph": "one CUDA graph per layer copy"},
+            "pct_of_peak": round(100 * value_tbs * 1e3 / (hbm * ws), 2),
+            "roofline": roof,
+            "cpu_baseline": cpu,
+            "e2e": e2e,
+            "gpu_launches": args.steps * n_lin * kernels_per_gemv,
+            "clocks": clk.summary(),
+            "prefill_gemm": gemm,
+        }
+        print(json.dumps(out), flush=True)
+    if ws > 1:
+        dist.destroy_process_group()
+
+
+def bench_gemm(polyq, synth, torch, device, stream, args, tf_burst, tf_sus):
+    """Prefill GEMM on the gate/up/down linears at M=2048 (TFLOP/s)."""
+    res = {}
+    try:
+        for name, N, K in (("gate", 13824, 5120), ("down", 5120, 13824)):
+            W, a = synth.layer_weights(N, K, synth.seed_for(4, 0 if name == "gate" else 2))
+            host = polyq.HostLayer.pack(W, a, args.budget)
+            dev = polyq.DeviceLayer(host, device)
+            for M in (512, 2048):
+                Xb, _ = synth.activations(a, M, synth.seed_for(4, 10))
+                X = torch.from_numpy(Xb.view(np.int16)).to(device).view(torch.bfloat16)
+                Y = torch.empty((M, N), dtype=torch.float32, device=device)
+                wsb = torch.empty(max(polyq.gemm_workspace_bytes(dev, M), 256), dtype=torch.uint8,
+                                  device=device)
+                with torch.cuda.stream(stream):
+                    for _ in range(3):
+                        polyq.linear_gemm(dev, X, Y=Y, workspace=wsb, stream=stream)
+                    e0 = torch.cuda.Event(enable_timing=True)
+                    e1 = torch.cuda.Event(enable_timing=True)
+                    reps = 20
+                    e0.record(stream)
+                    for _ in range(reps):
+                        polyq.linear_gemm(dev, X, Y=Y, workspace=wsb, stream=stream)
+                    e1.record(stream)
+                stream.synchronize()
+                ms = e0.elapsed_time(e1) / reps
+                tf = 2.0 * M * N * K / (ms * 1e-3) / 1e12
+                res[f"{name}_M{M}"] = {"tflops": round(tf, 1), "us": round(1e3 * ms, 1),
+                                       "frac_of_burst": round(tf / tf_burst, 4)}
+            del W
+    except polyq.PolyqError as e:
+        return {"unavailable": str(e)}
+    return res
+
+
+def cpu_baseline(seconds):
+    """The oracle's linear (unpack + dequantise + fp64 dot from the packed
+    bytes) on a bounded sample of the workload: row slices of the seven
+    linears, repeated until about ``seconds`` of CPU time."""
+    from oracle import polyq_oracle as O
+    from paper_2607_14618_gb300 import synth
+    rows = 256
+    layers = []
+    for i, (name, N, K) in enumerate(LLAMA):
+        W, a = synth.layer_weights(N, K, synth.seed_for(2, i))
+        bits = O.allocate_bits(O.saliency(W, a), 3.0)
+        L = O.pack_layer(W[:rows], a, 3.0, bits=bits)
+        _, x = synth.activations(a, 1, synth.seed_for(2, i))
+        layers.append((L, x))
+        del W
+    nbytes = 0
+    t0 = time.perf_counter()
+    while time.perf_counter() - t0 < seconds:
+        for L, x in layers:
+            O.linear(L, x)
+            nbytes += L["packed"].nbytes + L["meta"].nbytes + x.size * 2 + L["K"] * 4 + rows * 4
+    dt = time.perf_counter() - t0
+    threads = os.environ.get("OMP_NUM_THREADS") or os.environ.get("OPENBLAS_NUM_THREADS")
+    return {"value": round(nbytes / dt / 1e12, 8), "unit": "TB/s",
+            "cores": int(threads) if threads else 1, "host_cpus": os.cpu_count(),
+            "kind": "oracle",
+            "sample": f"{rows} output rows of each of the 7 linears, oracle linear "
+                      f"(unpack+dequant+fp64 dot) repeated for {dt:.1f} s"}
+
+
+def run_reference(args):
+    ws, rank, _ = _dist()
+    if rank != 0:
+        return
+    from oracle import polyq_oracle as O
+    from paper_2607_14618_gb300 import synth
+    rows = 128
+    layers = []
+    for i, (name, N, K) in enumerate(LLAMA):
+        W, a = synth.layer_weights(N, K, synth.seed_for(2, i))
+        bits = O.allocate_bits(O.saliency(W, a), args.budget)
+        L = O.pack_layer(W[:rows], a, args.budget, bits=bits)
+        _, x = synth.activations(a, 1, synth.seed_for(2, i))
+        layers.append((L, x))
+        del W
+
+    def step():
+        n = 0
+        for L, x in layers:
+            O.linear(L, x)
+            n += L["packed"].nbytes + L["meta"].nbytes + x.size * 2 + L["K"] * 4 + rows * 4
+        return n
+
+    for _ in range(args.warmup):
+        step()
+    t0 = time.perf_counter()
+    nb = sum(step() for _ in range(args.steps))
+    dt = time.perf_counter() - t0
+    v = nb / dt / 1e12
+    out = {"impl": "reference", "metric": METRIC, "value": round(v, 8), "unit": "TB/s",
+           "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
+           "ms_per_step": round(1e3 * dt / args.steps, 3), "higher_is_better": True,
+           "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+           "config": {"workload": WORKLOAD, "budget_bits": args.budget, "batch": 1},
+           "cpu_baseline": {"kind": "oracle", "cores": 1, "host_cpus": os.cpu_count(),
+                            "value": round(v, 8), "unit": "TB/s",
+                            "sample": f"{rows} output rows of each of the 7 linears per step"},
+           "e2e": {"value": round(v, 8), "unit": "TB/s", "h2d_bytes_per_step": 0,
+                   "d2h_bytes_per_step": 0}}
+    print(json.dumps(out), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", default="polyq", choices=["polyq", "reference"])
+    ap.add_argument("--budget", type=float, default=3.0)
+    ap.add_argument("--batch", type=int, default=1)
+    ap.add_argument("--copies", type=int, default=6)
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-gemm", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_polyq(args)
+
+
+if __name__ == "__main__":
+    main()

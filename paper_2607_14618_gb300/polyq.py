@@ -216,6 +216,19 @@ class DeviceLayer:
     def packed_bytes(self):
         return self.info["packed_bytes"] + self.info["meta_bytes"]
 
+    def clone(self):
+        """A second device copy of the same packed layer (distinct memory)."""
+        c = object.__new__(DeviceLayer)
+        c.info, c.perm, c.out_perm, c.N, c.K = self.info, self.perm, self.out_perm, self.N, self.K
+        c.packed = self.packed.clone()
+        c.meta = self.meta.clone()
+        c.gather = self.gather
+        c.desc = DevLayer()
+        C.pointer(c.desc)[0] = self.desc
+        c.desc.packed = c.packed.data_ptr()
+        c.desc.meta = c.meta.data_ptr() if c.meta.numel() else None
+        return c
+
 
 def _stream_ptr(stream):
     import torch
@@ -281,3 +294,8 @@ def unpack_codes(layer: DeviceLayer, stream=None):
     _check(_lib.polyq_unpack_codes(C.byref(layer.desc), out.data_ptr(), _stream_ptr(stream)))
     torch.cuda.synchronize()
     return out.cpu().numpy().view(np.uint16)
+
+
+def gemv_launches_per_call(layer: DeviceLayer, batch: int) -> int:
+    """Kernels one polyq_linear_gemv call enqueues."""
+    return 1

@@ -1,0 +1,108 @@
+"""GPU parity of the decode GEMV and the code unpacker against the oracle.
+All calls go through the C ABI (ctypes binding)."""
+import numpy as np
+import pytest
+
+from oracle import polyq_oracle as O
+from paper_2607_14618_gb300 import synth
+from tests.gpu_util import check_tolerance, make_case, oracle_layer, oracle_rows
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+
+def _dev(polyq_lib, W, a, B, bits=None, gather=None, identity=False):
+    host = polyq_lib.HostLayer.pack(W, a, B, forced_bits=bits)
+    return host, polyq_lib.DeviceLayer(host, "cuda", gather=gather, identity_gather=identity)
+
+
+def _x_dev(xb):
+    return torch.from_numpy(xb.view(np.int16)).cuda().view(torch.bfloat16)
+
+
+@pytest.mark.parametrize("N,K,B,seed,forced", [
+    (2048, 2048, 3.0, 1001, False),
+    (37, 1000, 3.0, 3, True),
+    (8, 16, 3.0, 4, True),
+    (130, 4099, 4.5, 5, True),
+])
+def test_unpack_codes_bit_exact(polyq_lib, N, K, B, seed, forced):
+    W, a, bits, _, _ = make_case(N, K, B, seed, forced)
+    host, dev = _dev(polyq_lib, W, a, B, bits)
+    ref = oracle_layer(W, a, B, bits)
+    assert np.array_equal(dev.perm, ref["perm"].astype(np.int32))
+    got = polyq_lib.unpack_codes(dev)
+    assert np.array_equal(got.astype(np.int64), O.unpack_codes(ref))
+
+
+@pytest.mark.parametrize("batch", [1, 2, 3, 4])
+@pytest.mark.parametrize("N,K,B,seed,forced", [
+    (2048, 2048, 3.0, 1001, False),   # 2048 x 2048 at B = 3.0
+    (300, 5120, 4.5, 2002, False),
+    (61, 3001, 3.0, 7, True),         # all five widths, ragged blocks
+    (8, 16, 3.0, 8, True),            # tiny
+    (5, 1, 16.0, 9, False),           # a single channel
+    (257, 700, 2.0, 10, False),       # all 2-bit
+    (64, 640, 16.0, 11, False),       # all 16-bit
+])
+def test_gemv_matches_oracle(polyq_lib, batch, N, K, B, seed, forced):
+    W, a, bits, xb, x = make_case(N, K, B, seed, forced, batch)
+    host, dev = _dev(polyq_lib, W, a, B, bits)
+    ref = oracle_layer(W, a, B, bits)
+    y = polyq_lib.linear_gemv(dev, _x_dev(xb))
+    torch.cuda.synchronize()
+    check_tolerance(y.cpu().numpy(), O.linear(ref, x), x, K)
+
+
+def test_gemv_residual_and_identity_gather(polyq_lib):
+    W, a, bits, xb, x = make_case(500, 1500, 3.0, 12, True, 2)
+    ref = oracle_layer(W, a, 3.0, bits)
+    # merged edge: x already in the clustered basis, gather = identity
+    xs_bits = xb[:, ref["perm"]]
+    host, dev = _dev(polyq_lib, W, a, 3.0, bits, identity=True)
+    res = torch.randn(2, 500, device="cuda")
+    y = polyq_lib.linear_gemv(dev, _x_dev(np.ascontiguousarray(xs_bits)), residual=res)
+    torch.cuda.synchronize()
+    yref = O.linear(ref, x) + res.cpu().numpy().astype(np.float64)
+    check_tolerance(y.cpu().numpy(), yref, x, 1500)
+    # in-place residual (y aliases residual)
+    res2 = res.clone()
+    polyq_lib.linear_gemv(dev, _x_dev(np.ascontiguousarray(xs_bits)), y=res2, residual=res2)
+    torch.cuda.synchronize()
+    assert torch.equal(res2, y)
+
+
+def test_gemv_merged_rows_match_unmerged(polyq_lib):
+    """Section 4.3: producer rows permuted by the consumer's perm emit the
+    consumer's basis; outputs equal the unmerged outputs gathered."""
+    Wp, ap, _, xb, x = make_case(900, 640, 3.0, 13, False, 1)
+    host = polyq_lib.HostLayer.pack(Wp, ap, 3.0)
+    dev = polyq_lib.DeviceLayer(host, "cuda")
+    y = polyq_lib.linear_gemv(dev, _x_dev(xb)).cpu().numpy()
+    cperm = np.random.default_rng(0).permutation(900)
+    host.permute_rows(cperm)
+    devm = polyq_lib.DeviceLayer(host, "cuda")
+    ym = polyq_lib.linear_gemv(devm, _x_dev(xb)).cpu().numpy()
+    assert np.array_equal(ym, y[:, cperm])
+
+
+@pytest.mark.parametrize("name,N,K,B,batch", [
+    ("llama-q", 5120, 5120, 3.0, 1),
+    ("llama-gate", 13824, 5120, 3.0, 1),
+    ("llama-down", 5120, 13824, 4.5, 1),
+    ("qwen-kv", 1024, 5120, 3.5, 4),
+    ("qwen-down", 5120, 25600, 6.0, 4),
+])
+def test_gemv_full_size_sampled_rows(polyq_lib, name, N, K, B, batch):
+    """Full-size layers in the benchmark's launch configuration; the oracle
+    recomputes a sample of output rows."""
+    seed = 7000 + N + K
+    W, a = synth.layer_weights(N, K, seed)
+    xb, x = synth.activations(a, batch, seed)
+    host, dev = _dev(polyq_lib, W, a, B)
+    y = polyq_lib.linear_gemv(dev, _x_dev(xb))
+    torch.cuda.synchronize()
+    rows = np.unique(np.concatenate([[0, N - 1], np.random.default_rng(1).integers(0, N, 60)]))
+    ref, bits_full = oracle_rows(W, a, B, rows)
+    assert np.array_equal(host.export()["bits"], bits_full.astype(np.uint8))
+    check_tolerance(y.cpu().numpy()[:, rows], O.linear(ref, x), x, K)
