@@ -97,16 +97,20 @@ typedef struct {
   double b_real;         /* realised mean width (Section 3.3, B_real) */
   int64_t packed_bytes;  /* N * row_stride */
   int64_t meta_bytes;    /* N * n_groups * 4 */
+  int64_t meta_stride;   /* device meta row stride in entries: n_groups
+                            rounded up to a multiple of 4 (16-byte rows) */
 } polyq_info;
 
 /* A packed layer resident on the device.  Filled by polyq_dev_layer_fill()
  * (or by hand).  The library only reads it. */
 typedef struct {
   const uint8_t* packed;  /* device [N][row_stride], 16-byte aligned */
-  const uint32_t* meta;   /* device [N][n_groups], 16-byte aligned */
+  const uint32_t* meta;   /* device [N][meta_stride], 16-byte aligned; entries
+                             past n_groups in a row are ignored */
   const int32_t* gather;  /* device [K]: xs[p] = x[gather[p]]; NULL = identity
                              (a merged edge, Section 4.3) */
   int64_t N, K, row_stride, n_groups;
+  int64_t meta_stride;    /* entries per meta row, multiple of 4, >= n_groups */
   int32_t n_blocks;
   polyq_block blocks[POLYQ_MAX_BLOCKS];
 } polyq_dev_layer;
@@ -135,12 +139,14 @@ void polyq_free(polyq_layer* layer);
 int polyq_layer_info(const polyq_layer* layer, polyq_info* out);
 
 /* Copy the packed layer into caller buffers (each may be NULL to skip):
- * packed [N*row_stride] bytes, meta [N*n_groups] uint32, perm [K] int32,
- * bits [K] uint8 (original channel order), out_perm [N] int32 (the layer
- * emits output i = y_original[out_perm[i]]). */
+ * packed [N*row_stride] bytes, meta [N*meta_stride] uint32 (rows padded
+ * with zero entries; meta_stride >= n_groups, use n_groups for the compact
+ * host format or polyq_info.meta_stride for the device layout), perm [K]
+ * int32, bits [K] uint8 (original channel order), out_perm [N] int32 (the
+ * layer emits output i = y_original[out_perm[i]]). */
 int polyq_layer_export(const polyq_layer* layer, uint8_t* packed,
-                       uint32_t* meta, int32_t* perm, uint8_t* bits,
-                       int32_t* out_perm);
+                       uint32_t* meta, int64_t meta_stride, int32_t* perm,
+                       uint8_t* bits, int32_t* out_perm);
 
 /* Section 4.3 merge, producer side: permute whole output rows (packed bytes
  * and meta) so that afterwards the layer emits
@@ -158,8 +164,9 @@ int polyq_permute_merge(const int32_t* producer_basis,
                         int32_t* gather_out);
 
 /* Fill a device-layer descriptor from a host layer and the device copies of
- * its packed bytes and meta (uploaded by the caller from polyq_layer_export)
- * and an optional device gather vector (NULL = identity). */
+ * its packed bytes and meta (uploaded by the caller from polyq_layer_export
+ * with meta_stride = polyq_info.meta_stride) and an optional device gather
+ * vector (NULL = identity). */
 int polyq_dev_layer_fill(const polyq_layer* layer, const uint8_t* packed_dev,
                          const uint32_t* meta_dev, const int32_t* gather_dev,
                          polyq_dev_layer* out);

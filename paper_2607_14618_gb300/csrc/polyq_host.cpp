@@ -416,15 +416,26 @@ extern "C" int polyq_layer_info(const polyq_layer* L, polyq_info* out) {
   out->b_real = (double)sum / (double)L->K;
   out->packed_bytes = L->N * L->S;
   out->meta_bytes = L->N * L->G * 4;
+  out->meta_stride = (L->G + 3) / 4 * 4;
   return POLYQ_OK;
 }
 
 extern "C" int polyq_layer_export(const polyq_layer* L, uint8_t* packed, uint32_t* meta,
-                                  int32_t* perm, uint8_t* bits, int32_t* out_perm) {
+                                  int64_t meta_stride, int32_t* perm, uint8_t* bits,
+                                  int32_t* out_perm) {
   polyq_clear_error();
   if (!L) return polyq_set_error(POLYQ_EINVAL, "polyq_layer_export: NULL layer");
+  if (meta && meta_stride < L->G)
+    return polyq_set_error(POLYQ_EINVAL, "polyq_layer_export: meta_stride %lld < n_groups %lld",
+                           (long long)meta_stride, (long long)L->G);
   if (packed) std::memcpy(packed, L->packed.data(), L->packed.size());
-  if (meta) std::memcpy(meta, L->meta.data(), L->meta.size() * 4);
+  if (meta) {
+    for (int64_t n = 0; n < L->N; ++n) {
+      uint32_t* dst = meta + n * meta_stride;
+      if (L->G) std::memcpy(dst, L->meta.data() + n * L->G, L->G * 4);
+      for (int64_t g = L->G; g < meta_stride; ++g) dst[g] = 0u;
+    }
+  }
   if (perm) std::memcpy(perm, L->perm.data(), L->perm.size() * 4);
   if (bits) std::memcpy(bits, L->bits.data(), L->bits.size());
   if (out_perm) std::memcpy(out_perm, L->out_perm.data(), L->out_perm.size() * 4);
@@ -478,6 +489,7 @@ extern "C" int polyq_dev_layer_fill(const polyq_layer* L, const uint8_t* packed_
   out->K = L->K;
   out->row_stride = L->S;
   out->n_groups = L->G;
+  out->meta_stride = (L->G + 3) / 4 * 4;
   out->n_blocks = (int32_t)L->blocks.size();
   for (size_t i = 0; i < L->blocks.size(); ++i) out->blocks[i] = L->blocks[i];
   return POLYQ_OK;
@@ -510,5 +522,8 @@ int polyq_check_dev_layer(const polyq_dev_layer* L, const char* who) {
   if (pos != L->K || off != L->row_stride || goff != L->n_groups)
     return polyq_set_error(POLYQ_EINVAL, "%s: block table does not cover the layer", who);
   if (L->n_groups > 0 && !L->meta) return polyq_set_error(POLYQ_EINVAL, "%s: meta is NULL", who);
+  if (L->meta_stride < L->n_groups || L->meta_stride % 4)
+    return polyq_set_error(POLYQ_EINVAL, "%s: meta_stride must be a multiple of 4 >= n_groups",
+                           who);
   return POLYQ_OK;
 }

@@ -55,13 +55,14 @@ class Info(C.Structure):
     _fields_ = [("N", C.c_int64), ("K", C.c_int64), ("row_stride", C.c_int64),
                 ("n_groups", C.c_int64), ("n_blocks", C.c_int32),
                 ("blocks", Block * MAX_BLOCKS), ("budget", C.c_double), ("b_real", C.c_double),
-                ("packed_bytes", C.c_int64), ("meta_bytes", C.c_int64)]
+                ("packed_bytes", C.c_int64), ("meta_bytes", C.c_int64),
+                ("meta_stride", C.c_int64)]
 
 
 class DevLayer(C.Structure):
     _fields_ = [("packed", C.c_void_p), ("meta", C.c_void_p), ("gather", C.c_void_p),
                 ("N", C.c_int64), ("K", C.c_int64), ("row_stride", C.c_int64),
-                ("n_groups", C.c_int64), ("n_blocks", C.c_int32),
+                ("n_groups", C.c_int64), ("meta_stride", C.c_int64), ("n_blocks", C.c_int32),
                 ("blocks", Block * MAX_BLOCKS)]
 
 
@@ -73,7 +74,7 @@ _SIGS = {
                              C.POINTER(C.c_void_p)]),
     "polyq_free": (None, [_P]),
     "polyq_layer_info": (C.c_int, [_P, C.POINTER(Info)]),
-    "polyq_layer_export": (C.c_int, [_P, _P, _P, _P, _P, _P]),
+    "polyq_layer_export": (C.c_int, [_P, _P, _P, C.c_int64, _P, _P, _P]),
     "polyq_layer_permute_rows": (C.c_int, [_P, _P]),
     "polyq_permute_merge": (C.c_int, [_P, _P, C.c_int64, _P]),
     "polyq_dev_layer_fill": (C.c_int, [_P, _P, _P, _P, C.POINTER(DevLayer)]),
@@ -173,15 +174,18 @@ class HostLayer:
         d["blocks"] = [inf.blocks[i].as_dict() for i in range(inf.n_blocks)]
         return d
 
-    def export(self) -> dict:
+    def export(self, meta_stride=None) -> dict:
+        """Host copies; meta rows have ``meta_stride`` entries (default: the
+        compact n_groups; pass info()['meta_stride'] for the device layout)."""
         inf = self.info()
         N, K, S, G = inf["N"], inf["K"], inf["row_stride"], inf["n_groups"]
+        ms = G if meta_stride is None else int(meta_stride)
         packed = np.empty((N, S), np.uint8)
-        meta = np.empty((N, G), np.uint32)
+        meta = np.empty((N, ms), np.uint32)
         perm = np.empty(K, np.int32)
         bits = np.empty(K, np.uint8)
         out_perm = np.empty(N, np.int32)
-        _check(_lib.polyq_layer_export(self._h, packed.ctypes.data, meta.ctypes.data,
+        _check(_lib.polyq_layer_export(self._h, packed.ctypes.data, meta.ctypes.data, ms,
                                        perm.ctypes.data, bits.ctypes.data, out_perm.ctypes.data))
         return dict(info=inf, packed=packed, meta=meta, perm=perm, bits=bits, out_perm=out_perm)
 
@@ -195,7 +199,7 @@ class DeviceLayer:
 
     def __init__(self, host: HostLayer, device="cuda", gather=None, identity_gather=False):
         import torch
-        ex = host.export()
+        ex = host.export(meta_stride=host.info()["meta_stride"])
         self.info = ex["info"]
         self.perm = ex["perm"]
         self.out_perm = ex["out_perm"]
@@ -297,5 +301,6 @@ def unpack_codes(layer: DeviceLayer, stream=None):
 
 
 def gemv_launches_per_call(layer: DeviceLayer, batch: int) -> int:
-    """Kernels one polyq_linear_gemv call enqueues."""
-    return 1
+    """Kernels one polyq_linear_gemv call enqueues (activation pre-pass and
+    the streaming kernel)."""
+    return 2

@@ -52,6 +52,11 @@ def _compare(host, ref):
     meta_ref = ref["meta"][:, :, 0].astype(np.uint32) | (ref["meta"][:, :, 1].astype(np.uint32) << 16)
     assert np.array_equal(ex["meta"], meta_ref)
     assert inf["b_real"] == O.realized_budget(ref)
+    ms = inf["meta_stride"]
+    assert ms % 4 == 0 and ms >= inf["n_groups"]
+    padded = host.export(meta_stride=ms)["meta"]
+    assert np.array_equal(padded[:, :inf["n_groups"]], meta_ref)
+    assert np.all(padded[:, inf["n_groups"]:] == 0)
 
 
 @pytest.mark.parametrize("N,K,B,seed", [
@@ -192,6 +197,8 @@ def test_corrupt_descriptors_rejected_before_launch(polyq_lib):
         lambda d: setattr(d.blocks[0], "seg_bytes", d.blocks[0].seg_bytes + 16),
         lambda d: setattr(d.blocks[3], "grp_off", 0),
         lambda d: setattr(d, "n_groups", d.n_groups - 1),
+        lambda d: setattr(d, "meta_stride", d.meta_stride + 1),
+        lambda d: setattr(d, "meta_stride", d.n_groups - 1),
     ]
     for f in cases:
         d = mutate(f)
