@@ -34,6 +34,8 @@ LLAMA = [("q", 5120, 5120), ("k", 5120, 5120), ("v", 5120, 5120), ("o", 5120, 51
          ("gate", 13824, 5120), ("up", 13824, 5120), ("down", 5120, 13824)]
 WORKLOAD = ("llama2-13b decode linears q,k,v,o 5120x5120, gate,up 13824x5120, "
             "down 5120x13824; batch 1; B=3.0")
+# launches of one decoder layer: q/k/v and gate/up read the same input
+GROUPS = [(0, 1, 2), (3,), (4, 5), (6,)]
 
 
 def _peaks():
@@ -60,7 +62,7 @@ class ClockSampler:
         try:
             self.p = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.Q}",
-                 "--format=csv,noheader,nounits", "-lms", "200"],
+                 "--format=csv,noheader,nounits", "-lms", "100"],
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
         except OSError:
             self.p = None
@@ -102,17 +104,21 @@ def _dist():
 
 
 def build_layers(polyq, synth, budget, copies, device):
-    """Pack the seven linears once (seeded), upload, and clone on device."""
-    layers, xs, bytes_per_step = [], [], 0
+    """Pack the seven linears once (seeded), upload, and clone on device.
+    Linears of one launch group share their input activation."""
+    layers, xs = [], [None] * len(LLAMA)
     hosts = []
     for i, (name, N, K) in enumerate(LLAMA):
         W, a = synth.layer_weights(N, K, synth.seed_for(2, i))
         host = polyq.HostLayer.pack(W, a, budget)
         dev = polyq.DeviceLayer(host, device)
-        xb, _ = synth.activations(a, 1, synth.seed_for(2, i))
-        xs.append(xb)
         hosts.append((name, host.info()))
         layers.append([dev] + [dev.clone() for _ in range(copies - 1)])
+        for grp in GROUPS:
+            if grp[0] == i:
+                xb, _ = synth.activations(a, 1, synth.seed_for(2, i))
+                for k in grp:
+                    xs[k] = xb
         del W
     return layers, xs, hosts
 
@@ -152,23 +158,27 @@ def run_polyq(args):
     xs = [torch.from_numpy(np.repeat(x, batch, 0).view(np.int16)).to(device).view(torch.bfloat16)
           for x in xs_np]
     ys = [torch.empty((batch, N), dtype=torch.float32, device=device) for _, N, _ in LLAMA]
-    wsz = max(polyq.gemv_workspace_bytes(layers[i][0], batch) for i in range(n_lin))
+    wsz = max(polyq.gemv_group_workspace_bytes([layers[i][0] for i in grp], batch)
+              for grp in GROUPS)
     wbuf = torch.zeros(max(wsz, 256), dtype=torch.uint8, device=device)
-    kernels_per_gemv = polyq.gemv_launches_per_call(layers[0][0], batch)
+    kernels_per_call = polyq.gemv_launches_per_call(layers[0][0], batch)
+
+    def run_step(c):
+        for grp in GROUPS:
+            polyq.linear_gemv_group([layers[i][c] for i in grp], [xs[i] for i in grp],
+                                    ys=[ys[i] for i in grp], workspace=wbuf, stream=stream)
 
     stream = torch.cuda.Stream(device)
     torch.cuda.synchronize()
     with torch.cuda.stream(stream):
-        for i in range(n_lin):  # warm the launch path once before capture
-            polyq.linear_gemv(layers[i][0], xs[i], y=ys[i], workspace=wbuf, stream=stream)
+        run_step(0)  # warm the launch path once before capture
     stream.synchronize()
-    graphs = []      # one graph per layer copy: the seven GEMVs of a step
+    graphs = []      # one graph per layer copy: the four launches of a step
     lin_graphs = []  # one graph per (linear, copy): per-launch diagnostics
     for c in range(args.copies):
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, stream=stream):
-            for i in range(n_lin):
-                polyq.linear_gemv(layers[i][c], xs[i], y=ys[i], workspace=wbuf, stream=stream)
+            run_step(c)
         graphs.append(g)
     for i in range(n_lin):
         row = []
@@ -180,15 +190,17 @@ def run_polyq(args):
         lin_graphs.append(row)
     torch.cuda.synchronize()
 
-    for s in range(args.warmup):
-        graphs[s % args.copies].replay()
+    # graph replays launch on the current stream: make it `stream`
+    with torch.cuda.stream(stream):
+        for s in range(args.warmup):
+            graphs[s % args.copies].replay()
     torch.cuda.synchronize()
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
     if ws > 1:
         dist.barrier()
     torch.cuda.synchronize()
-    with ClockSampler(local) as clk:
+    with ClockSampler(local) as clk, torch.cuda.stream(stream):
         t0.record(stream)
         for s in range(args.steps):
             graphs[s % args.copies].replay()
@@ -214,12 +226,13 @@ def run_polyq(args):
     for i in range(n_lin):
         e0 = torch.cuda.Event(enable_timing=True)
         e1 = torch.cuda.Event(enable_timing=True)
-        for r in range(args.copies):
-            lin_graphs[i][r].replay()
-        e0.record(stream)
-        for r in range(reps):
-            lin_graphs[i][r % args.copies].replay()
-        e1.record(stream)
+        with torch.cuda.stream(stream):
+            for r in range(args.copies):
+                lin_graphs[i][r].replay()
+            e0.record(stream)
+            for r in range(reps):
+                lin_graphs[i][r % args.copies].replay()
+            e1.record(stream)
         torch.cuda.synchronize()
         us = 1e3 * e0.elapsed_time(e1) / reps
         per_lin_us[LLAMA[i][0]] = {"us": round(us, 2),
@@ -227,7 +240,7 @@ def run_polyq(args):
     ach = step_bytes / (ms_step * 1e-3) / 1e9
     roof = {"bound": "hbm", "achieved": round(ach, 1), "peak": hbm, "unit": "GB/s",
             "frac": round(ach / hbm, 4), "traffic": None, "peak_kind": peak_kind,
-            "kernel": "gemv_main (+ gemv_prep) of polyq_linear_gemv",
+            "kernel": "gemv_main (+ gemv_prep) of polyq_linear_gemv_group",
             "per_linear": per_lin_us}
 
     # end to end through the public API: pinned host x -> device, GEMVs, y -> host
@@ -236,7 +249,7 @@ def run_polyq(args):
         hx = [torch.from_numpy(np.repeat(x, batch, 0).view(np.int16)).pin_memory() for x in xs_np]
         hy = [torch.empty((batch, N), dtype=torch.float32).pin_memory() for _, N, _ in LLAMA]
         dx = [torch.empty((batch, K), dtype=torch.int16, device=device) for _, _, K in LLAMA]
-        h2d = sum(t.numel() * 2 for t in hx)
+        h2d = sum(hx[grp[0]].numel() * 2 for grp in GROUPS)
         d2h = sum(t.numel() * 4 for t in hy)
         e_steps = max(3, min(args.steps, 50))
         with torch.cuda.stream(stream):
@@ -245,11 +258,14 @@ def run_polyq(args):
                     stream.synchronize()
                     ta = time.perf_counter()
                 c = s % args.copies
-                for i in range(n_lin):
-                    dx[i].copy_(hx[i], non_blocking=True)
-                    polyq.linear_gemv(layers[i][c], dx[i].view(torch.bfloat16), y=ys[i],
-                                      workspace=wbuf, stream=stream)
-                    hy[i].copy_(ys[i], non_blocking=True)
+                for grp in GROUPS:
+                    dx[grp[0]].copy_(hx[grp[0]], non_blocking=True)
+                    polyq.linear_gemv_group([layers[i][c] for i in grp],
+                                            [dx[grp[0]].view(torch.bfloat16)] * len(grp),
+                                            ys=[ys[i] for i in grp], workspace=wbuf,
+                                            stream=stream)
+                    for i in grp:
+                        hy[i].copy_(ys[i], non_blocking=True)
                 stream.synchronize()
             tb = time.perf_counter()
         e2e = {"value": round(step_bytes * e_steps / (tb - ta) / 1e12, 4), "unit": "TB/s",
@@ -275,12 +291,13 @@ def run_polyq(args):
                              f"{L2 / 2**20:.0f} MiB)",
                        "bytes_per_step": step_bytes,
                        "b_real": {n: round(inf["b_real"], 5) for n, inf in infos},
+                       "launch_groups": "q+k+v, o, gate+up, down (4 launches of 2 kernels)",
                        "graph": "one CUDA graph per layer copy"},
             "pct_of_peak": round(100 * value_tbs * 1e3 / (hbm * ws), 2),
             "roofline": roof,
             "cpu_baseline": cpu,
             "e2e": e2e,
-            "gpu_launches": args.steps * n_lin * kernels_per_gemv,
+            "gpu_launches": args.steps * len(GROUPS) * kernels_per_call,
             "clocks": clk.summary(),
             "prefill_gemm": gemm,
         }
@@ -399,7 +416,7 @@ def run_reference(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--steps", type=int, default=20000)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", default="polyq", choices=["polyq", "reference"])
     ap.add_argument("--budget", type=float, default=3.0)

@@ -60,6 +60,7 @@ extern "C" {
 
 #define POLYQ_MAX_BLOCKS 5
 #define POLYQ_GROUP 64
+#define POLYQ_MAX_GROUP 4 /* layers per polyq_linear_gemv_group call */
 
 #define POLYQ_ALLOC_WATERFILL 0 /* Section 3.2 max-heap waterfilling (default) */
 #define POLYQ_ALLOC_LADDER 1    /* descending saliency, each channel climbs */
@@ -185,6 +186,22 @@ int polyq_gemv_workspace_bytes(const polyq_dev_layer* layer, int batch,
 int polyq_linear_gemv(const polyq_dev_layer* layer, const void* x, int batch,
                       float* y, const float* residual, void* workspace,
                       size_t workspace_bytes, void* stream);
+
+/* Device scratch bytes polyq_linear_gemv_group needs for these layers. */
+int polyq_gemv_group_workspace_bytes(const polyq_dev_layer* const* layers,
+                                     int n, int batch, size_t* bytes);
+
+/* Several independent decode GEMVs (the Section 4.1 product of each layer)
+ * in one pair of launches, e.g. q/k/v or gate/up of a decoder layer, which
+ * read the same activation.  layers[i], xs[i], ys[i], residuals[i] (the
+ * array itself and each entry may be NULL) have the meaning they have in
+ * polyq_linear_gemv; 1 <= n <= POLYQ_MAX_GROUP; all layers share `batch`
+ * and one workspace of polyq_gemv_group_workspace_bytes().  Outputs must not
+ * overlap each other or any input. */
+int polyq_linear_gemv_group(const polyq_dev_layer* const* layers, int n,
+                            const void* const* xs, int batch, float* const* ys,
+                            const float* const* residuals, void* workspace,
+                            size_t workspace_bytes, void* stream);
 
 /* Device scratch bytes polyq_linear_gemm needs for this layer and M. */
 int polyq_gemm_workspace_bytes(const polyq_dev_layer* layer, int64_t M,

@@ -21,10 +21,10 @@ namespace gv {
 
 constexpr int kRows = 64;          // rows per work tile (4 consumer warps x 16)
 constexpr int kWarps = 4;          // consumer warps per CTA
-constexpr int kStages = 4;         // TMA pipeline depth
+constexpr int kStages = 3;         // TMA pipeline depth per CTA (3 CTAs per SM)
 constexpr int kPitchSplit = 144;   // row pitch of 128-byte half boxes (16 extra bytes)
 constexpr int kMetaBox = 16;       // meta entries per row loaded per step
-constexpr int kCodesBytes = 2 * kRows * kPitchSplit;  // largest codes area per stage
+constexpr int kCodesBytes = 2 * kRows * kPitchSplit;  // largest codes area per stage (2 boxes)
 constexpr int kMetaBytes = kRows * kMetaBox * 4;
 constexpr int kRecMax = 1344;
 constexpr int kStageBytes = ((kCodesBytes + kMetaBytes + kRecMax) + 127) / 128 * 128;
@@ -38,17 +38,21 @@ __host__ __device__ constexpr int ubits(int bits) { return bits == 8 ? 4 : bits;
 __host__ __device__ constexpr int step_bytes(int bits, int nb) {
   return bits == 16 ? 2 * kU16 : units_of(nb) * ubits(bits) / 8;
 }
-// Steps whose byte size is a multiple of 128 are loaded as 128-byte halves
-// with a 144-byte row pitch (conflict-free 32-byte lane reads); others as one
-// box whose pitch is the step size.
-__host__ __device__ constexpr int halves(int bits, int nb) {
-  return step_bytes(bits, nb) % 128 == 0 ? step_bytes(bits, nb) / 128 : 0;
+// A step is loaded as nbox boxes of equal byte width, box h covering bytes
+// [h*SB/nbox, (h+1)*SB/nbox) of every row.  Lane t reads bytes
+// [t*LB, (t+1)*LB) of each box.  A box that is 128 bytes wide gets a 144-byte
+// row pitch (16 bytes of the next box ride along) so that rows g and g+1 land
+// in different shared-memory banks; all other widths are conflict-free as is.
+__host__ __device__ constexpr int nbox_of(int bits, int nb) { return (bits == 16 || nb == 1) ? 2 : 1; }
+__host__ __device__ constexpr int box_bytes(int bits, int nb) {
+  return step_bytes(bits, nb) / nbox_of(bits, nb);
 }
-__host__ __device__ constexpr int box_width(int bits, int nb) {
-  return halves(bits, nb) ? kPitchSplit : step_bytes(bits, nb);
+__host__ __device__ constexpr int box_pitch(int bits, int nb) {
+  return box_bytes(bits, nb) == 128 ? kPitchSplit : box_bytes(bits, nb);
 }
+__host__ __device__ constexpr int lane_box_bytes(int bits, int nb) { return box_bytes(bits, nb) / 4; }
 __host__ __device__ constexpr int lane_words(int bits, int nb) {
-  return bits == 16 ? 16 : cpl_of(nb) * ubits(bits) / 32;
+  return nbox_of(bits, nb) * lane_box_bytes(bits, nb) / 4;
 }
 // Words per record row (one lane, one batch): pairs plus 16 bytes of padding.
 __host__ __device__ constexpr int rec_lane_words(int nb) { return cpl_of(nb) / 2 + 4; }
@@ -59,15 +63,15 @@ __host__ __device__ constexpr int rec_bytes(int nb) {
 static_assert(rec_bytes(1) <= kRecMax && rec_bytes(2) <= kRecMax && rec_bytes(4) <= kRecMax, "");
 static_assert(rec_bytes(1) % 16 == 0 && rec_bytes(2) % 16 == 0 && rec_bytes(4) % 16 == 0, "");
 
-// Step-relative unit index of the i-th unit that lane t decodes.
+// Step-relative unit index of the i-th unit that lane t decodes.  With two
+// boxes (batch 1) lane t owns chunks t and t+4, so MMA i of the lane loop
+// covers the same chunk position in every lane and a partly filled step can
+// stop early.
 __host__ __device__ inline int lane_unit(int bits, int nb, int t, int i) {
-  const int ub = ubits(bits);
-  if (halves(bits, nb)) {
-    const int per_box = 256 / ub;  // 32 bytes per lane per half
-    const int h = i / per_box;
-    return (128 * h + 32 * t) * 8 / ub + (i % per_box);
-  }
-  return t * cpl_of(nb) + i;
+  const int nbx = nbox_of(bits, nb);
+  const int per = cpl_of(nb) / nbx;  // units per lane per box
+  const int h = i / per;
+  return h * (units_of(nb) / nbx) + t * per + (i % per);
 }
 
 // 16-bit steps: step-relative weight index of the lane's i-th weight (i < 32).

@@ -21,6 +21,7 @@ POLYQ_ECUDA = -3
 POLYQ_EUNSUPPORTED = -4
 POLYQ_ETIMEOUT = -5
 MAX_BLOCKS = 5
+MAX_GROUP = 4
 GROUP = 64
 ALLOC_WATERFILL = 0
 ALLOC_LADDER = 1
@@ -80,6 +81,12 @@ _SIGS = {
     "polyq_dev_layer_fill": (C.c_int, [_P, _P, _P, _P, C.POINTER(DevLayer)]),
     "polyq_gemv_workspace_bytes": (C.c_int, [C.POINTER(DevLayer), C.c_int, C.POINTER(C.c_size_t)]),
     "polyq_linear_gemv": (C.c_int, [C.POINTER(DevLayer), _P, C.c_int, _P, _P, _P, C.c_size_t, _P]),
+    "polyq_gemv_group_workspace_bytes": (C.c_int, [C.POINTER(C.POINTER(DevLayer)), C.c_int,
+                                                   C.c_int, C.POINTER(C.c_size_t)]),
+    "polyq_linear_gemv_group": (C.c_int, [C.POINTER(C.POINTER(DevLayer)), C.c_int,
+                                          C.POINTER(C.c_void_p), C.c_int,
+                                          C.POINTER(C.c_void_p), C.POINTER(C.c_void_p),
+                                          _P, C.c_size_t, _P]),
     "polyq_gemm_workspace_bytes": (C.c_int, [C.POINTER(DevLayer), C.c_int64,
                                              C.POINTER(C.c_size_t)]),
     "polyq_linear_gemm": (C.c_int, [C.POINTER(DevLayer), _P, C.c_int64, _P, _P, C.c_size_t, _P]),
@@ -264,6 +271,47 @@ def linear_gemv(layer: DeviceLayer, x, y=None, residual=None, workspace=None, st
                                   residual.data_ptr() if residual is not None else None,
                                   ws_ptr, ws_len, _stream_ptr(stream)))
     return y
+
+
+def _layer_array(layers):
+    arr = (C.POINTER(DevLayer) * len(layers))()
+    for i, l in enumerate(layers):
+        arr[i] = C.pointer(l.desc)
+    return arr
+
+
+def gemv_group_workspace_bytes(layers, batch: int) -> int:
+    n = C.c_size_t()
+    _check(_lib.polyq_gemv_group_workspace_bytes(_layer_array(layers), len(layers), int(batch),
+                                                 C.byref(n)))
+    return n.value
+
+
+def linear_gemv_group(layers, xs, ys=None, residuals=None, workspace=None, stream=None):
+    """Independent GEMVs in one launch: ys[i] = residuals[i] + xs[i] W_i'^T."""
+    import torch
+    n = len(layers)
+    if len(xs) != n:
+        raise ValueError("one x per layer")
+    batch = xs[0].shape[0]
+    for l, x in zip(layers, xs):
+        if x.dtype != torch.bfloat16 or not x.is_cuda or x.dim() != 2 or x.shape != (batch, l.K):
+            raise ValueError("each x must be a CUDA bf16 tensor [batch][K]")
+    xs = [x.contiguous() for x in xs]
+    if ys is None:
+        ys = [torch.empty((batch, l.N), dtype=torch.float32, device=xs[0].device) for l in layers]
+    need = gemv_group_workspace_bytes(layers, batch)
+    if workspace is None:
+        workspace = torch.empty(need, dtype=torch.uint8, device=xs[0].device)
+    xa = (C.c_void_p * n)(*[x.data_ptr() for x in xs])
+    ya = (C.c_void_p * n)(*[y.data_ptr() for y in ys])
+    ra = None
+    if residuals is not None:
+        ra = (C.c_void_p * n)(*[r.data_ptr() if r is not None else None for r in residuals])
+    _check(_lib.polyq_linear_gemv_group(_layer_array(layers), n, xa, batch, ya, ra,
+                                        workspace.data_ptr(), workspace.numel(),
+                                        _stream_ptr(stream)))
+    return ys
 
 
 def gemm_workspace_bytes(layer: DeviceLayer, M: int) -> int:

@@ -65,16 +65,19 @@ def test_gemv_residual_and_identity_gather(polyq_lib):
     torch.cuda.synchronize()
     yref = O.linear(ref, x) + res.cpu().numpy().astype(np.float64)
     check_tolerance(y.cpu().numpy(), yref, x, 1500)
-    # in-place residual (y aliases residual)
+    # in-place residual (y aliases residual); split tiles add their pieces
+    # atomically, so agreement is to fp32 rounding
     res2 = res.clone()
     polyq_lib.linear_gemv(dev, _x_dev(np.ascontiguousarray(xs_bits)), y=res2, residual=res2)
     torch.cuda.synchronize()
-    assert torch.equal(res2, y)
+    assert torch.allclose(res2, y, rtol=1e-5, atol=1e-5 * float(y.abs().max()))
 
 
 def test_gemv_merged_rows_match_unmerged(polyq_lib):
     """Section 4.3: producer rows permuted by the consumer's perm emit the
-    consumer's basis; outputs equal the unmerged outputs gathered."""
+    consumer's basis; outputs equal the unmerged outputs gathered.  Rows of a
+    tile whose K range is split over CTAs sum their pieces in a different
+    association, so equality is to fp32 rounding, not bitwise."""
     Wp, ap, _, xb, x = make_case(900, 640, 3.0, 13, False, 1)
     host = polyq_lib.HostLayer.pack(Wp, ap, 3.0)
     dev = polyq_lib.DeviceLayer(host, "cuda")
@@ -83,7 +86,8 @@ def test_gemv_merged_rows_match_unmerged(polyq_lib):
     host.permute_rows(cperm)
     devm = polyq_lib.DeviceLayer(host, "cuda")
     ym = polyq_lib.linear_gemv(devm, _x_dev(xb)).cpu().numpy()
-    assert np.array_equal(ym, y[:, cperm])
+    ref = y[:, cperm]
+    assert np.max(np.abs(ym - ref)) <= 1e-5 * np.max(np.abs(ref))
 
 
 @pytest.mark.parametrize("name,N,K,B,batch", [
@@ -106,3 +110,31 @@ def test_gemv_full_size_sampled_rows(polyq_lib, name, N, K, B, batch):
     ref, bits_full = oracle_rows(W, a, B, rows)
     assert np.array_equal(host.export()["bits"], bits_full.astype(np.uint8))
     check_tolerance(y.cpu().numpy()[:, rows], O.linear(ref, x), x, K)
+
+
+@pytest.mark.parametrize("batch", [1, 4])
+def test_gemv_group_matches_oracle(polyq_lib, batch):
+    """Several layers in one launch (q/k/v-like: shared input, own widths and
+    gathers; plus a layer of another shape and forced widths)."""
+    K = 1536
+    specs = [(640, 3.0, 31, False), (256, 3.5, 32, False), (256, 4.5, 33, True), (130, 3.0, 34, True)]
+    layers, refs, xs = [], [], []
+    _, a0 = synth.layer_weights(8, K, 30)
+    xb, x = synth.activations(a0, batch, 30)
+    for N, B, seed, forced in specs:
+        W, a = synth.layer_weights(N, K, seed)
+        bits = synth.random_codes_layer_bits(K, seed) if forced else None
+        host = polyq_lib.HostLayer.pack(W, a, B, forced_bits=bits)
+        layers.append(polyq_lib.DeviceLayer(host, "cuda"))
+        refs.append(O.pack_layer(W, a, B, bits=bits))
+    xt = _x_dev(xb)
+    res = [None, torch.randn(batch, 256, device="cuda"), None, None]
+    ys = polyq_lib.linear_gemv_group(layers, [xt] * 4, residuals=res)
+    torch.cuda.synchronize()
+    for i, (y, ref) in enumerate(zip(ys, refs)):
+        yref = O.linear(ref, x)
+        if res[i] is not None:
+            yref = yref + res[i].cpu().numpy().astype(np.float64)
+        check_tolerance(y.cpu().numpy(), yref, x, K)
+    with pytest.raises(polyq_lib.PolyqError):
+        polyq_lib.linear_gemv_group(layers + layers[:1], [xt] * 5)
