@@ -1,16 +1,486 @@
-// Prefill GEMM entry points (tensor-core kernel lands here).
+// Prefill GEMM of the PolyQ mixed-bit layer on the 5th-generation tensor
+// cores (tcgen05, tensor memory):
+//
+//   Y[m][n] = sum_p X[m][gather[p]] * W'[n][p]        (Section 4.1 product)
+//
+// The contraction runs over 64-wide K tiles; every tile lies inside one bit
+// block (Section 4.2) and one quantisation group, so each weight row of a tile
+// has one (scale, zero).
+//  1. gemm_prep gathers X through `gather` into a clustered fp16 matrix
+//     Xg[M][KT*64] (workspace), zero-padded at block ends, with the K order
+//     inside each tile permuted the same way the dequantiser emits codes.
+//  2. gemm_main: one persistent CTA per SM, 10 warps.
+//       warp 0      TMA producer: Xg tiles (128-byte swizzle), packed code
+//                   bytes and meta of 256 weight rows, or for 16-bit blocks the
+//                   fp16 weights straight into the operand buffer;
+//       warp 1      allocates 512 TMEM columns and issues tcgen05.mma
+//                   (M=128, N=256, K=16, fp16 in, fp32 accumulate), two
+//                   M tiles per weight tile;
+//       warps 2..9  dequantise one weight row each: (q - z) * s in fp16 via
+//                   magic-number decode, written in the UMMA 128-byte-swizzle
+//                   K-major layout; afterwards they drain the accumulator with
+//                   tcgen05.ld and store fp32 Y.
+//     Two pipeline stages; every wait is bounded and reports through the
+//     workspace status word.
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 
+#include <algorithm>
+
 #include "polyq.h"
+#include "polyq_dev.cuh"
 #include "polyq_internal.h"
+
+namespace {
+
+using namespace polyq;
+
+constexpr int BM = 128;           // rows per MMA
+constexpr int MT = 2;             // M tiles per work unit (share one weight tile)
+constexpr int BN = 256;           // weight rows per work unit
+constexpr int BK = 64;            // K per tile (one quantisation group)
+constexpr int kStagesG = 2;
+constexpr int kCodeBox = 80;      // code bytes per row loaded per tile (>= 8 + 64)
+constexpr int kATile = BM * BK * 2;             // 16 KB, 1024-aligned
+constexpr int kBTile = BN * BK * 2;             // 32 KB
+constexpr int kCodes = BN * kCodeBox;           // 20 KB
+constexpr int kMeta = BN * 16;                  // 4 KB
+constexpr int kStageG = MT * kATile + kBTile + kCodes + kMeta;  // 88 KB
+constexpr int kThreadsG = 320;
+constexpr int kDqWarps = 8;
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kIdesc = umma_idesc_f16(BM, BN);
+
+struct GmBlock {
+  int bits, n_ch, pos0, seg_off, grp_off, n_grp;
+  int kt0, n_kt;  // K-tile range of the block
+};
+
+struct GmParams {
+  CUtensorMap tm_x;      // Xg [M][KT*64] fp16, box {64, 128}, 128B swizzle
+  CUtensorMap tm_codes;  // packed [N][S] u8, box {80, 256}
+  CUtensorMap tm_meta;   // meta [N][meta_stride] u32, box {4, 256}
+  CUtensorMap tm_w16;    // packed [N][S/2] u16, box {64, 256}, 128B swizzle
+  GmBlock blk[POLYQ_MAX_BLOCKS];
+  int n_blocks;
+  int M, N, K, KT;
+  int units_m, units;    // work units: (256-row M pair, 256-row N tile)
+  int has_meta;
+  const __nv_bfloat16* x;
+  const int32_t* gather;
+  __half* xg;
+  float* y;
+  int* status;
+};
+
+__device__ __forceinline__ int find_kblock(const GmBlock* blk, int nblk, int kt) {
+  int b = 0;
+  while (b + 1 < nblk && kt >= blk[b + 1].kt0) ++b;
+  return b;
+}
+
+// Position inside a 64-code group of the code that fills K slot `s` of a
+// tile (the order in which the dequantiser emits its fp16 pairs).
+__host__ __device__ inline int slot_code(int bits, int s) {
+  const int i = (s & 31) >> 1, h = s & 1;
+  switch (bits) {
+    case 2: return 16 * (s >> 4) + ((s & 15) >> 1) + 8 * h;
+    case 3: return 32 * (s >> 5) + i + 16 * h;
+    case 4: return 8 * (s >> 3) + ((s & 7) >> 1) + 4 * h;
+    default: return s;  // 8- and 16-bit: natural order
+  }
+}
+
+// ---------------------------------------------------------------------------
+// pre-pass: Xg[m][kt*64 + s] = fp16(X[m][gather[pos0 + 64 g + slot_code(s)]])
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) gemm_prep(const __grid_constant__ GmParams P) {
+  pdl_trigger();
+  pdl_wait();
+  __shared__ GmBlock sblk[POLYQ_MAX_BLOCKS];
+  if (threadIdx.x < POLYQ_MAX_BLOCKS) {
+    switch (threadIdx.x) {
+      case 0: sblk[0] = P.blk[0]; break;
+      case 1: sblk[1] = P.blk[1]; break;
+      case 2: sblk[2] = P.blk[2]; break;
+      case 3: sblk[3] = P.blk[3]; break;
+      default: sblk[4] = P.blk[4]; break;
+    }
+  }
+  if (blockIdx.x == 0 && threadIdx.x == 0) *P.status = 0;
+  __syncthreads();
+  const int Kp = P.KT * BK;
+  const long long pairs = (long long)P.M * (Kp / 2);
+  for (long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x; e < pairs;
+       e += (long long)gridDim.x * blockDim.x) {
+    const int m = (int)(e / (Kp / 2));
+    const int k = 2 * (int)(e - (long long)m * (Kp / 2));
+    const int kt = k / BK, s = k % BK;
+    const GmBlock& B = sblk[find_kblock(sblk, P.n_blocks, kt)];
+    const int g = kt - B.kt0;
+    __half v[2];
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int w = 64 * g + slot_code(B.bits, s + h);
+      float xv = 0.f;
+      if (w < B.n_ch) {
+        const int p = B.pos0 + w;
+        const int src = P.gather ? P.gather[p] : p;
+        xv = __bfloat162float(P.x[(size_t)m * P.K + src]);
+      }
+      v[h] = __float2half_rn(xv);
+    }
+    reinterpret_cast<__half2*>(P.xg)[e] = __halves2half2(v[0], v[1]);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// dequantisation of one weight row of one tile into the swizzled B operand
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void store_pairs_sw128(uint8_t* btile, int r, int chunk,
+                                                  const uint32_t (&p)[4]) {
+  uint8_t* dst = btile + (r >> 3) * 1024 + (r & 7) * 128 + ((chunk ^ (r & 7)) << 4);
+  *reinterpret_cast<uint4*>(dst) = make_uint4(p[0], p[1], p[2], p[3]);
+}
+
+__device__ __forceinline__ uint32_t dq_pair(uint32_t raw, __half2 zz, __half2 ss) {
+  // raw holds fp16 (1024 + q) in each half: (q - z) is exact, the product
+  // (q - z) * s is rounded once to fp16.
+  const __half2 d = __hsub2(*reinterpret_cast<const __half2*>(&raw), zz);
+  const __half2 w = __hmul2(d, ss);
+  return *reinterpret_cast<const uint32_t*>(&w);
+}
+
+__device__ __forceinline__ void dequant_row(int bits, const uint8_t* row_bytes, uint32_t meta,
+                                            uint8_t* btile, int r) {
+  const uint32_t magic = 0x64006400u;
+  const __half s = __ushort_as_half((uint16_t)(meta & 0xFFFFu));
+  const __half z = __ushort_as_half((uint16_t)(meta >> 16));
+  const __half2 ss = __halves2half2(s, s);
+  const __half zz1 = __hadd(z, __float2half(1024.f));
+  const __half2 zz = __halves2half2(zz1, zz1);
+  const uint2* src = reinterpret_cast<const uint2*>(row_bytes);  // 8-byte aligned
+  if (bits == 2) {
+#pragma unroll
+    for (int wp = 0; wp < 2; ++wp) {
+      const uint2 ww = src[wp];
+      const uint32_t w2[2] = {ww.x, ww.y};
+#pragma unroll
+      for (int q = 0; q < 2; ++q) {
+        const uint32_t w = w2[q];
+        const int wd = 2 * wp + q;
+#pragma unroll
+        for (int c2 = 0; c2 < 2; ++c2) {
+          uint32_t p[4];
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const int ii = 4 * c2 + i;
+            p[i] = dq_pair(((w >> (2 * ii)) & 0x00030003u) | magic, zz, ss);
+          }
+          store_pairs_sw128(btile, r, 2 * wd + c2, p);
+        }
+      }
+    }
+  } else if (bits == 3) {
+    uint32_t w[6];
+#pragma unroll
+    for (int k = 0; k < 3; ++k) {
+      const uint2 ww = src[k];
+      w[2 * k] = ww.x;
+      w[2 * k + 1] = ww.y;
+    }
+#pragma unroll
+    for (int u = 0; u < 2; ++u) {
+      const uint32_t a = w[3 * u], b = w[3 * u + 1], c = w[3 * u + 2];
+#pragma unroll
+      for (int c4 = 0; c4 < 4; ++c4) {
+        uint32_t p[4];
+#pragma unroll
+        for (int i4 = 0; i4 < 4; ++i4) {
+          const int i = 4 * c4 + i4;  // codes i and i + 16 of this 32-code unit
+          const int o = 3 * i;
+          const uint32_t lo = o < 32 ? __funnelshift_r(a, b, o) : __funnelshift_r(b, c, o - 32);
+          const uint32_t hi = o < 32 ? __funnelshift_r(b, c, o) : (c >> (o - 32));
+          const uint32_t m2 = __byte_perm(lo, hi, 0x7610);
+          p[i4] = dq_pair((m2 & 0x00070007u) | magic, zz, ss);
+        }
+        store_pairs_sw128(btile, r, 4 * u + c4, p);
+      }
+    }
+  } else if (bits == 4) {
+#pragma unroll
+    for (int wp = 0; wp < 4; ++wp) {
+      const uint2 ww = src[wp];
+      const uint32_t w2[2] = {ww.x, ww.y};
+#pragma unroll
+      for (int q = 0; q < 2; ++q) {
+        const uint32_t w = w2[q];
+        uint32_t p[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) p[i] = dq_pair(((w >> (4 * i)) & 0x000F000Fu) | magic, zz, ss);
+        store_pairs_sw128(btile, r, 2 * wp + q, p);
+      }
+    }
+  } else {  // 8-bit
+#pragma unroll
+    for (int wp = 0; wp < 8; ++wp) {
+      const uint2 ww = src[wp];
+      uint32_t p[4];
+      p[0] = dq_pair(__byte_perm(ww.x, 0x64646464u, 0x4140), zz, ss);
+      p[1] = dq_pair(__byte_perm(ww.x, 0x64646464u, 0x4342), zz, ss);
+      p[2] = dq_pair(__byte_perm(ww.y, 0x64646464u, 0x4140), zz, ss);
+      p[3] = dq_pair(__byte_perm(ww.y, 0x64646464u, 0x4342), zz, ss);
+      store_pairs_sw128(btile, r, wp, p);
+    }
+  }
+}
+
+__global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant__ GmParams P) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  // 1024-byte alignment of the operand tiles (128-byte swizzle atoms)
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+  __shared__ uint64_t bar_full[kStagesG], bar_bready[kStagesG], bar_sfree[kStagesG];
+  __shared__ uint64_t bar_accf, bar_acce;
+  __shared__ uint32_t tmem_base_slot;
+  __shared__ GmBlock sblk[POLYQ_MAX_BLOCKS];
+  __shared__ volatile int s_abort;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  if (threadIdx.x < POLYQ_MAX_BLOCKS) {
+    switch (threadIdx.x) {
+      case 0: sblk[0] = P.blk[0]; break;
+      case 1: sblk[1] = P.blk[1]; break;
+      case 2: sblk[2] = P.blk[2]; break;
+      case 3: sblk[3] = P.blk[3]; break;
+      default: sblk[4] = P.blk[4]; break;
+    }
+  }
+  if (threadIdx.x == 0) {
+    s_abort = 0;
+    for (int s = 0; s < kStagesG; ++s) {
+      mbar_init(smem_u32(&bar_full[s]), 1);
+      mbar_init(smem_u32(&bar_bready[s]), kDqWarps);
+      mbar_init(smem_u32(&bar_sfree[s]), 1);
+    }
+    mbar_init(smem_u32(&bar_accf), 1);
+    mbar_init(smem_u32(&bar_acce), kDqWarps);
+    mbar_fence_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(&tmem_base_slot), kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tmem_base_slot;
+  pdl_trigger();
+
+  const int KT = P.KT;
+  const int nblk = P.n_blocks;
+  auto stage_ptr = [&](int s) { return smem + s * kStageG; };
+  auto fail = [&](int code) {
+    s_abort = 1;
+    atomicExch(P.status, code);
+  };
+
+  if (warp == 0) {
+    // ---------------- TMA producer ----------------
+    if (lane == 0) {
+      prefetch_tmap(&P.tm_x);
+      prefetch_tmap(&P.tm_codes);
+      if (P.has_meta) prefetch_tmap(&P.tm_meta);
+      prefetch_tmap(&P.tm_w16);
+      pdl_wait();  // Xg comes from the pre-pass
+      int kg = 0;
+      for (int u = blockIdx.x; u < P.units && !s_abort; u += gridDim.x) {
+        const int um = u % P.units_m, un = u / P.units_m;
+        for (int kt = 0; kt < KT && !s_abort; ++kt, ++kg) {
+          const int s = kg % kStagesG, use = kg / kStagesG;
+          if (use > 0 && !mbar_wait(smem_u32(&bar_sfree[s]), (use - 1) & 1)) {
+            fail(kStatusTimeoutEmpty);
+            break;
+          }
+          const GmBlock& B = sblk[find_kblock(sblk, nblk, kt)];
+          const int g = kt - B.kt0;
+          uint8_t* st = stage_ptr(s);
+          const uint32_t bar = smem_u32(&bar_full[s]);
+          const bool w16 = B.bits == 16;
+          mbar_expect_tx(bar, MT * kATile + (w16 ? kBTile : kCodes + kMeta));
+#pragma unroll
+          for (int t = 0; t < MT; ++t)
+            tma_load_2d(smem_u32(st + t * kATile), &P.tm_x, kt * BK, um * (MT * BM) + t * BM, bar);
+          if (w16) {
+            tma_load_2d(smem_u32(st + MT * kATile), &P.tm_w16, (B.seg_off + 128 * g) / 2, un * BN,
+                        bar);
+          } else {
+            const int start = B.seg_off + 8 * B.bits * g;
+            tma_load_2d(smem_u32(st + MT * kATile + kBTile), &P.tm_codes, start & ~15, un * BN,
+                        bar);
+            tma_load_2d(smem_u32(st + MT * kATile + kBTile + kCodes), &P.tm_meta,
+                        (B.grp_off + g) & ~3, un * BN, bar);
+          }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ---------------- MMA issuer ----------------
+    if (lane == 0) {
+      int kg = 0, uc = 0;
+      for (int u = blockIdx.x; u < P.units && !s_abort; u += gridDim.x, ++uc) {
+        if (uc > 0 && !mbar_wait(smem_u32(&bar_acce), (uc - 1) & 1)) {
+          fail(kStatusTimeoutEmpty);
+          break;
+        }
+        tc_fence_after();
+        for (int kt = 0; kt < KT && !s_abort; ++kt, ++kg) {
+          const int s = kg % kStagesG, use = kg / kStagesG;
+          if (!mbar_wait(smem_u32(&bar_full[s]), use & 1) ||
+              !mbar_wait(smem_u32(&bar_bready[s]), use & 1)) {
+            fail(kStatusTimeoutFull);
+            break;
+          }
+          tc_fence_after();
+          uint8_t* st = stage_ptr(s);
+          const uint32_t b0 = smem_u32(st + MT * kATile);
+#pragma unroll
+          for (int t = 0; t < MT; ++t) {
+            const uint32_t a0 = smem_u32(st + t * kATile);
+#pragma unroll
+            for (int kk = 0; kk < BK / 16; ++kk)
+              tc_mma_f16(tmem + t * BN, umma_desc_sw128(a0 + 32 * kk), umma_desc_sw128(b0 + 32 * kk),
+                         kIdesc, (kt > 0 || kk > 0) ? 1u : 0u);
+          }
+          tc_commit(smem_u32(&bar_sfree[s]));
+        }
+        tc_commit(smem_u32(&bar_accf));
+      }
+    }
+  } else {
+    // ---------------- dequantisation + epilogue (8 warps) ----------------
+    const int r = threadIdx.x - 64;  // weight row of the tile, 0..255
+    const int q = warp & 3;          // TMEM lane quarter this warp may access
+    const int half = (warp - 2) >> 2;
+    int kg = 0, uc = 0;
+    for (int u = blockIdx.x; u < P.units && !s_abort; u += gridDim.x, ++uc) {
+      const int um = u % P.units_m, un = u / P.units_m;
+      for (int kt = 0; kt < KT && !s_abort; ++kt, ++kg) {
+        const int s = kg % kStagesG, use = kg / kStagesG;
+        if (!mbar_wait(smem_u32(&bar_full[s]), use & 1) ||
+            (use > 0 && !mbar_wait(smem_u32(&bar_sfree[s]), (use - 1) & 1))) {
+          fail(kStatusTimeoutFull);
+          break;
+        }
+        const GmBlock& B = sblk[find_kblock(sblk, nblk, kt)];
+        if (B.bits != 16) {
+          const int g = kt - B.kt0;
+          uint8_t* st = stage_ptr(s);
+          const int start = B.seg_off + 8 * B.bits * g;
+          const uint8_t* row_bytes = st + MT * kATile + kBTile + r * kCodeBox + (start & 15);
+          const uint32_t meta = reinterpret_cast<const uint32_t*>(
+              st + MT * kATile + kBTile + kCodes)[r * 4 + ((B.grp_off + g) & 3)];
+          dequant_row(B.bits, row_bytes, meta, st + MT * kATile, r);
+          fence_proxy_async_smem();
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&bar_bready[s]));
+      }
+      if (s_abort) break;
+      // epilogue: rows 32q + lane of each M tile, columns [128 half, +128)
+      if (!mbar_wait(smem_u32(&bar_accf), uc & 1)) {
+        fail(kStatusTimeoutFull);
+        break;
+      }
+      tc_fence_after();
+#pragma unroll
+      for (int t = 0; t < MT; ++t) {
+        const int m = um * (MT * BM) + t * BM + 32 * q + lane;
+#pragma unroll
+        for (int c4 = 0; c4 < 4; ++c4) {
+          const int col = 128 * half + 32 * c4;
+          uint32_t v[32];
+          tc_ld_32x32b_x32(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(t * BN + col), v);
+          tc_wait_ld();
+          const int n0 = un * BN + col;
+          if (m < P.M) {
+            float* dst = P.y + (size_t)m * P.N + n0;
+            if (n0 + 32 <= P.N && (P.N % 4) == 0) {
+#pragma unroll
+              for (int j = 0; j < 8; ++j)
+                reinterpret_cast<float4*>(dst)[j] =
+                    make_float4(__uint_as_float(v[4 * j]), __uint_as_float(v[4 * j + 1]),
+                                __uint_as_float(v[4 * j + 2]), __uint_as_float(v[4 * j + 3]));
+            } else {
+#pragma unroll
+              for (int j = 0; j < 32; ++j)
+                if (n0 + j < P.N) dst[j] = __uint_as_float(v[j]);
+            }
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&bar_acce));
+    }
+  }
+
+  // all roles done (or aborted): wait for the last tensor-core work, free TMEM
+  __syncthreads();
+  if (warp == 1) {
+    if (lane == 0) {
+      // the last commit of this CTA went to bar_accf; its completion means all
+      // MMAs have finished reading shared memory and writing TMEM
+      int uc = 0;
+      for (int u = blockIdx.x; u < P.units; u += gridDim.x) ++uc;
+      if (uc > 0) mbar_wait(smem_u32(&bar_accf), (uc - 1) & 1);
+    }
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// host side
+// ---------------------------------------------------------------------------
+int k_tiles(const polyq_dev_layer* L, GmBlock* blk) {
+  int kt = 0;
+  for (int i = 0; i < L->n_blocks; ++i) {
+    const polyq_block& b = L->blocks[i];
+    GmBlock g;
+    g.bits = b.bits;
+    g.n_ch = b.n_ch;
+    g.pos0 = b.pos0;
+    g.seg_off = b.seg_off;
+    g.grp_off = b.grp_off;
+    g.n_grp = b.n_grp;
+    g.kt0 = kt;
+    g.n_kt = (b.n_ch + BK - 1) / BK;
+    kt += g.n_kt;
+    if (blk) blk[i] = g;
+  }
+  return kt;
+}
+
+size_t gemm_workspace(const polyq_dev_layer* L, int64_t M) {
+  const size_t xg = (size_t)M * k_tiles(L, nullptr) * BK * 2;
+  return (xg + 255) / 256 * 256 + 256;
+}
+
+}  // namespace
 
 extern "C" int polyq_gemm_workspace_bytes(const polyq_dev_layer* L, int64_t M, size_t* bytes) {
   polyq_clear_error();
   int rc = polyq_check_dev_layer(L, "polyq_gemm_workspace_bytes");
   if (rc) return rc;
-  (void)M;
-  (void)bytes;
-  return polyq_set_error(POLYQ_EUNSUPPORTED, "polyq_gemm_workspace_bytes: GEMM not built yet");
+  if (!bytes) return polyq_set_error(POLYQ_EINVAL, "polyq_gemm_workspace_bytes: bytes is NULL");
+  if (M < 1 || M > (1 << 24))
+    return polyq_set_error(POLYQ_EINVAL, "polyq_gemm_workspace_bytes: M=%lld", (long long)M);
+  *bytes = gemm_workspace(L, M);
+  return POLYQ_OK;
 }
 
 extern "C" int polyq_linear_gemm(const polyq_dev_layer* L, const void* X, int64_t M, float* Y,
@@ -18,6 +488,85 @@ extern "C" int polyq_linear_gemm(const polyq_dev_layer* L, const void* X, int64_
   polyq_clear_error();
   int rc = polyq_check_dev_layer(L, "polyq_linear_gemm");
   if (rc) return rc;
-  (void)X; (void)M; (void)Y; (void)workspace; (void)ws_bytes; (void)stream;
-  return polyq_set_error(POLYQ_EUNSUPPORTED, "polyq_linear_gemm: GEMM not built yet");
+  if (!X || !Y) return polyq_set_error(POLYQ_EINVAL, "polyq_linear_gemm: X or Y is NULL");
+  if (M < 1 || M > (1 << 24))
+    return polyq_set_error(POLYQ_EINVAL, "polyq_linear_gemm: M=%lld", (long long)M);
+  const size_t need = gemm_workspace(L, M);
+  if (!workspace || ws_bytes < need)
+    return polyq_set_error(POLYQ_ENOMEM, "polyq_linear_gemm: workspace needs %zu bytes, got %zu",
+                           need, ws_bytes);
+  if ((uintptr_t)workspace % 256)
+    return polyq_set_error(POLYQ_EINVAL, "polyq_linear_gemm: workspace must be 256-byte aligned");
+  if (L->row_stride % 16)
+    return polyq_set_error(POLYQ_EINVAL, "polyq_linear_gemm: row_stride must be a multiple of 16");
+
+  GmParams P;
+  memset(&P, 0, sizeof P);
+  const int KT = k_tiles(L, P.blk);
+  P.n_blocks = L->n_blocks;
+  P.M = (int)M;
+  P.N = (int)L->N;
+  P.K = (int)L->K;
+  P.KT = KT;
+  P.units_m = (int)((M + MT * BM - 1) / (MT * BM));
+  P.units = P.units_m * (int)((L->N + BN - 1) / BN);
+  P.x = (const __nv_bfloat16*)X;
+  P.gather = L->gather;
+  P.xg = (__half*)workspace;
+  P.y = Y;
+  P.status = (int*)((uint8_t*)workspace + need - 256);
+  rc = polyq_tensor_map_2d(&P.tm_x, P.xg, 2, (uint64_t)KT * BK, (uint64_t)M, (uint64_t)KT * BK * 2,
+                           BK, BM, 1);
+  if (rc) return rc;
+  rc = polyq_tensor_map_2d(&P.tm_codes, L->packed, 1, (uint64_t)L->row_stride, (uint64_t)L->N,
+                           (uint64_t)L->row_stride, kCodeBox, BN);
+  if (rc) return rc;
+  rc = polyq_tensor_map_2d(&P.tm_w16, L->packed, 2, (uint64_t)L->row_stride / 2, (uint64_t)L->N,
+                           (uint64_t)L->row_stride, BK, BN, 1);
+  if (rc) return rc;
+  if (L->n_groups > 0) {
+    rc = polyq_tensor_map_2d(&P.tm_meta, L->meta, 4, (uint64_t)L->meta_stride, (uint64_t)L->N,
+                             (uint64_t)L->meta_stride * 4, 4, BN);
+    if (rc) return rc;
+    P.has_meta = 1;
+  }
+
+  cudaStream_t st = (cudaStream_t)stream;
+  int sms = 0;
+  rc = polyq_sm_count(&sms);
+  if (rc) return rc;
+  static bool attr_done[8] = {false};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  const size_t smem = (size_t)kStagesG * kStageG + 1024;
+  if (!attr_done[dev & 7]) {
+    cudaError_t e = cudaFuncSetAttribute(gemm_main, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e != cudaSuccess)
+      return polyq_set_error(POLYQ_ECUDA, "polyq_linear_gemm: smem attribute: %s",
+                             cudaGetErrorString(e));
+    attr_done[dev & 7] = true;
+  }
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.stream = st;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  const long long pairs = M * (long long)(KT * BK / 2);
+  cfg.gridDim = dim3((unsigned)std::min<long long>((pairs + 255) / 256, (long long)sms * 16));
+  cfg.blockDim = dim3(256);
+  cudaError_t e = cudaLaunchKernelEx(&cfg, gemm_prep, P);
+  if (e != cudaSuccess)
+    return polyq_set_error(POLYQ_ECUDA, "polyq_linear_gemm: prep launch: %s", cudaGetErrorString(e));
+  // no programmatic overlap for the main kernel: it owns all of TMEM on an SM
+  cfg.numAttrs = 0;
+  cfg.gridDim = dim3((unsigned)std::min(P.units, sms));
+  cfg.blockDim = dim3(kThreadsG);
+  cfg.dynamicSmemBytes = smem;
+  e = cudaLaunchKernelEx(&cfg, gemm_main, P);
+  if (e != cudaSuccess)
+    return polyq_set_error(POLYQ_ECUDA, "polyq_linear_gemm: launch: %s", cudaGetErrorString(e));
+  return POLYQ_OK;
 }

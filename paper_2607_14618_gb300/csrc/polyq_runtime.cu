@@ -20,7 +20,7 @@ using EncodeFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, voi
 std::mutex g_mu;
 EncodeFn g_encode = nullptr;
 std::map<int, int> g_sms;
-using Key = std::tuple<uintptr_t, int, uint64_t, uint64_t, uint64_t, uint32_t, uint32_t>;
+using Key = std::tuple<uintptr_t, int, uint64_t, uint64_t, uint64_t, uint32_t, uint32_t, int>;
 std::map<Key, CUtensorMap> g_maps;
 
 int get_encode(EncodeFn* fn) {
@@ -59,8 +59,8 @@ int polyq_sm_count(int* out) {
 
 int polyq_tensor_map_2d(CUtensorMap* out, const void* base, int elem_bytes, uint64_t cols,
                         uint64_t rows, uint64_t row_stride_bytes, uint32_t box_cols,
-                        uint32_t box_rows) {
-  Key k{(uintptr_t)base, elem_bytes, cols, rows, row_stride_bytes, box_cols, box_rows};
+                        uint32_t box_rows, int swizzle128) {
+  Key k{(uintptr_t)base, elem_bytes, cols, rows, row_stride_bytes, box_cols, box_rows, swizzle128};
   std::lock_guard<std::mutex> lk(g_mu);
   auto it = g_maps.find(k);
   if (it != g_maps.end()) {
@@ -80,7 +80,8 @@ int polyq_tensor_map_2d(CUtensorMap* out, const void* base, int elem_bytes, uint
   CUtensorMap m;
   std::memset(&m, 0, sizeof m);
   CUresult r = enc(&m, dt, 2, const_cast<void*>(base), dims, strides, box, es,
-                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE,
+                   swizzle128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS)
     return polyq_set_error(POLYQ_ECUDA, "cuTensorMapEncodeTiled failed (%d)", (int)r);

@@ -1,0 +1,71 @@
+"""GPU parity of the tcgen05 prefill GEMM against the oracle (through the C ABI)."""
+import numpy as np
+import pytest
+
+from oracle import polyq_oracle as O
+from paper_2607_14618_gb300 import synth
+from tests.gpu_util import check_tolerance, oracle_rows
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+
+def _x_dev(xb):
+    return torch.from_numpy(np.ascontiguousarray(xb).view(np.int16)).cuda().view(torch.bfloat16)
+
+
+@pytest.mark.parametrize("M,N,K,B,seed,forced", [
+    (256, 256, 1100, 3.0, 51, True),     # all five widths, one work unit
+    (300, 300, 1100, 3.0, 52, True),     # ragged M and N, two units per axis
+    (1, 100, 700, 3.0, 53, True),        # a single token
+    (512, 640, 2048, 3.0, 54, False),    # allocation at B = 3
+    (130, 257, 1536, 6.0, 55, False),    # B = 6: many 8-bit channels
+    (64, 64, 320, 16.0, 56, False),      # all 16-bit
+    (96, 96, 640, 2.0, 57, False),       # all 2-bit
+])
+def test_gemm_matches_oracle(polyq_lib, M, N, K, B, seed, forced):
+    W, a = synth.layer_weights(N, K, seed)
+    bits = synth.random_codes_layer_bits(K, seed) if forced else None
+    Xb, X = synth.activations(a, M, seed)
+    host = polyq_lib.HostLayer.pack(W, a, B, forced_bits=bits)
+    dev = polyq_lib.DeviceLayer(host, "cuda")
+    ref = O.pack_layer(W, a, B, bits=bits)
+    Y = polyq_lib.linear_gemm(dev, _x_dev(Xb))
+    torch.cuda.synchronize()
+    check_tolerance(Y.cpu().numpy(), O.linear(ref, X), X, K)
+
+
+def test_gemm_identity_gather_and_repeat(polyq_lib):
+    W, a = synth.layer_weights(384, 1200, 58)
+    bits = synth.random_codes_layer_bits(1200, 58)
+    Xb, X = synth.activations(a, 200, 58)
+    host = polyq_lib.HostLayer.pack(W, a, 3.0, forced_bits=bits)
+    ref = O.pack_layer(W, a, 3.0, bits=bits)
+    dev = polyq_lib.DeviceLayer(host, "cuda", identity_gather=True)
+    Xs = np.ascontiguousarray(Xb[:, ref["perm"]])
+    ws = torch.zeros(polyq_lib.gemm_workspace_bytes(dev, 200), dtype=torch.uint8, device="cuda")
+    Y1 = polyq_lib.linear_gemm(dev, _x_dev(Xs), workspace=ws)
+    Y2 = polyq_lib.linear_gemm(dev, _x_dev(Xs), workspace=ws)
+    torch.cuda.synchronize()
+    check_tolerance(Y1.cpu().numpy(), O.linear(ref, X), X, 1200)
+    assert torch.equal(Y1, Y2)  # no atomics: deterministic
+
+
+@pytest.mark.parametrize("name,N,K,M", [
+    ("llama-gate", 13824, 5120, 512),
+    ("llama-down", 5120, 13824, 2048),
+])
+def test_gemm_full_size_sampled(polyq_lib, name, N, K, M):
+    seed = 9000 + N + K
+    W, a = synth.layer_weights(N, K, seed)
+    Xb, X = synth.activations(a, M, seed)
+    host = polyq_lib.HostLayer.pack(W, a, 3.0)
+    dev = polyq_lib.DeviceLayer(host, "cuda")
+    Y = polyq_lib.linear_gemm(dev, _x_dev(Xb))
+    torch.cuda.synchronize()
+    rng = np.random.default_rng(2)
+    rows = np.unique(np.concatenate([[0, N - 1], rng.integers(0, N, 40)]))
+    ms = np.unique(np.concatenate([[0, M - 1], rng.integers(0, M, 6)]))
+    ref, _ = oracle_rows(W, a, 3.0, rows)
+    yref = O.linear(ref, X[ms])
+    check_tolerance(Y.cpu().numpy()[np.ix_(ms, rows)], yref, X[ms], K)
