@@ -171,6 +171,16 @@ __device__ __forceinline__ uint64_t umma_desc_sw128(uint32_t smem_addr) {
   d |= (uint64_t)2u << 61;                              // 128-byte swizzle
   return d;
 }
+// Same for 64-byte rows with the 64-byte swizzle (8-row atoms 512 bytes apart).
+__device__ __forceinline__ uint64_t umma_desc_sw64(uint32_t smem_addr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((smem_addr >> 4) & 0x3FFFu);        // start address
+  d |= (uint64_t)1u << 16;                              // leading byte offset (unused)
+  d |= (uint64_t)(512u >> 4) << 32;                     // stride byte offset: 8-row atoms
+  d |= (uint64_t)1u << 46;                              // descriptor version (sm_100)
+  d |= (uint64_t)4u << 61;                              // 64-byte swizzle
+  return d;
+}
 // Instruction descriptor for kind::f16 with fp16 A/B, fp32 D, K-major A and B.
 __host__ __device__ constexpr uint32_t umma_idesc_f16(int M, int N) {
   return (1u << 4)                       // D format: f32
@@ -189,8 +199,8 @@ __device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v 
 // ---------------------------------------------------------------------------
 int polyq_sm_count(int* out);
 // 2-D tensor map over a row-major [rows][cols] array of `elem_bytes` elements
-// with a box of {box_cols, box_rows} (optionally 128-byte swizzled); cached
-// per (address, shape, box, swizzle).
+// with a box of {box_cols, box_rows}; swizzle_bytes is 0 (none), 64 or 128.
+// Cached per (address, shape, box, swizzle).
 int polyq_tensor_map_2d(CUtensorMap* out, const void* base, int elem_bytes, uint64_t cols,
                         uint64_t rows, uint64_t row_stride_bytes, uint32_t box_cols,
-                        uint32_t box_rows, int swizzle128 = 0);
+                        uint32_t box_rows, int swizzle_bytes = 0);

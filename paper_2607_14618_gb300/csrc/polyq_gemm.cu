@@ -3,25 +3,27 @@
 //
 //   Y[m][n] = sum_p X[m][gather[p]] * W'[n][p]        (Section 4.1 product)
 //
-// The contraction runs over 64-wide K tiles; every tile lies inside one bit
-// block (Section 4.2) and one quantisation group, so each weight row of a tile
-// has one (scale, zero).
+// The contraction runs over 32-wide K tiles (half a quantisation group); every
+// tile lies inside one bit block (Section 4.2) and one group, so each weight
+// row of a tile has one (scale, zero).
 //  1. gemm_prep gathers X through `gather` into a clustered fp16 matrix
-//     Xg[M][KT*64] (workspace), zero-padded at block ends, with the K order
+//     Xg[M][KT*32] (workspace), zero-padded at block ends, with the K order
 //     inside each tile permuted the same way the dequantiser emits codes.
 //  2. gemm_main: one persistent CTA per SM, 10 warps.
-//       warp 0      TMA producer: Xg tiles (128-byte swizzle), packed code
+//       warp 0      TMA producer: Xg tiles (64-byte swizzle), packed code
 //                   bytes and meta of 256 weight rows, or for 16-bit blocks the
 //                   fp16 weights straight into the operand buffer;
 //       warp 1      allocates 512 TMEM columns and issues tcgen05.mma
 //                   (M=128, N=256, K=16, fp16 in, fp32 accumulate), two
 //                   M tiles per weight tile;
 //       warps 2..9  dequantise one weight row each: (q - z) * s in fp16 via
-//                   magic-number decode, written in the UMMA 128-byte-swizzle
+//                   magic-number decode, written in the UMMA 64-byte-swizzle
 //                   K-major layout; afterwards they drain the accumulator with
 //                   tcgen05.ld and store fp32 Y.
-//     Two pipeline stages; every wait is bounded and reports through the
-//     workspace status word.
+//     Four pipeline stages.  When the (M, N) tiles cannot fill the GPU the K
+//     range is split and the pieces are added into a zeroed Y (so the order of
+//     those additions varies); otherwise Y is stored directly.  Every wait is
+//     bounded and reports through the workspace status word.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
@@ -40,14 +42,16 @@ using namespace polyq;
 constexpr int BM = 128;           // rows per MMA
 constexpr int MT = 2;             // M tiles per work unit (share one weight tile)
 constexpr int BN = 256;           // weight rows per work unit
-constexpr int BK = 64;            // K per tile (one quantisation group)
-constexpr int kStagesG = 2;
-constexpr int kCodeBox = 80;      // code bytes per row loaded per tile (>= 8 + 64)
-constexpr int kATile = BM * BK * 2;             // 16 KB, 1024-aligned
-constexpr int kBTile = BN * BK * 2;             // 32 KB
-constexpr int kCodes = BN * kCodeBox;           // 20 KB
+constexpr int BK = 32;            // K per tile: half a quantisation group
+constexpr int kStagesG = 4;
+constexpr int kCodeBox = 48;      // code bytes per row loaded per tile: an odd
+                                  // number of 16-byte chunks keeps row reads
+                                  // conflict-free; covers offset (<= 12) + 32
+constexpr int kATile = BM * BK * 2;             // 8 KB (64-byte rows)
+constexpr int kBTile = BN * BK * 2;             // 16 KB
+constexpr int kCodes = BN * kCodeBox;           // 12 KB
 constexpr int kMeta = BN * 16;                  // 4 KB
-constexpr int kStageG = MT * kATile + kBTile + kCodes + kMeta;  // 88 KB
+constexpr int kStageG = MT * kATile + kBTile + kCodes + kMeta;  // 48 KB
 constexpr int kThreadsG = 320;
 constexpr int kDqWarps = 8;
 constexpr uint32_t kTmemCols = 512;
@@ -59,14 +63,14 @@ struct GmBlock {
 };
 
 struct GmParams {
-  CUtensorMap tm_x;      // Xg [M][KT*64] fp16, box {64, 128}, 128B swizzle
-  CUtensorMap tm_codes;  // packed [N][S] u8, box {80, 256}
+  CUtensorMap tm_x;      // Xg [M][KT*32] fp16, box {32, 128}, 64B swizzle
+  CUtensorMap tm_codes;  // packed [N][S] u8, box {48, 256}
   CUtensorMap tm_meta;   // meta [N][meta_stride] u32, box {4, 256}
-  CUtensorMap tm_w16;    // packed [N][S/2] u16, box {64, 256}, 128B swizzle
+  CUtensorMap tm_w16;    // packed [N][S/2] u16, box {32, 256}, 64B swizzle
   GmBlock blk[POLYQ_MAX_BLOCKS];
   int n_blocks;
   int M, N, K, KT;
-  int units_m, units;    // work units: (256-row M pair, 256-row N tile)
+  int units_m, units_n, ksplit, units;  // work units: (M pair, N tile, K split)
   int has_meta;
   const __nv_bfloat16* x;
   const int32_t* gather;
@@ -81,20 +85,22 @@ __device__ __forceinline__ int find_kblock(const GmBlock* blk, int nblk, int kt)
   return b;
 }
 
-// Position inside a 64-code group of the code that fills K slot `s` of a
-// tile (the order in which the dequantiser emits its fp16 pairs).
+// Position inside a 32-code half group of the code that fills K slot `s`
+// (0..31) of a tile (the order in which the dequantiser emits its fp16 pairs).
 __host__ __device__ inline int slot_code(int bits, int s) {
-  const int i = (s & 31) >> 1, h = s & 1;
+  const int h = s & 1;
   switch (bits) {
     case 2: return 16 * (s >> 4) + ((s & 15) >> 1) + 8 * h;
-    case 3: return 32 * (s >> 5) + i + 16 * h;
+    case 3: return (s >> 1) + 16 * h;
     case 4: return 8 * (s >> 3) + ((s & 7) >> 1) + 4 * h;
     default: return s;  // 8- and 16-bit: natural order
   }
 }
 
 // ---------------------------------------------------------------------------
-// pre-pass: Xg[m][kt*64 + s] = fp16(X[m][gather[pos0 + 64 g + slot_code(s)]])
+// pre-pass: Xg[m][kt*32 + s] = fp16(X[m][gather[pos0 + 32 h + slot_code(s)]])
+// for the h-th 32-code half group of the block (tile kt); Y is zeroed when the
+// K range is split over CTAs
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(256) gemm_prep(const __grid_constant__ GmParams P) {
   pdl_trigger();
@@ -111,6 +117,12 @@ __global__ void __launch_bounds__(256) gemm_prep(const __grid_constant__ GmParam
   }
   if (blockIdx.x == 0 && threadIdx.x == 0) *P.status = 0;
   __syncthreads();
+  if (P.ksplit > 1) {
+    const long long total4 = (long long)P.M * P.N / 4;
+    for (long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x; e < total4;
+         e += (long long)gridDim.x * blockDim.x)
+      reinterpret_cast<float4*>(P.y)[e] = make_float4(0.f, 0.f, 0.f, 0.f);
+  }
   const int Kp = P.KT * BK;
   const long long pairs = (long long)P.M * (Kp / 2);
   for (long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x; e < pairs;
@@ -119,11 +131,11 @@ __global__ void __launch_bounds__(256) gemm_prep(const __grid_constant__ GmParam
     const int k = 2 * (int)(e - (long long)m * (Kp / 2));
     const int kt = k / BK, s = k % BK;
     const GmBlock& B = sblk[find_kblock(sblk, P.n_blocks, kt)];
-    const int g = kt - B.kt0;
+    const int hg = kt - B.kt0;  // half group index inside the block
     __half v[2];
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
-      const int w = 64 * g + slot_code(B.bits, s + h);
+      const int w = 32 * hg + slot_code(B.bits, s + h);
       float xv = 0.f;
       if (w < B.n_ch) {
         const int p = B.pos0 + w;
@@ -139,10 +151,18 @@ __global__ void __launch_bounds__(256) gemm_prep(const __grid_constant__ GmParam
 // ---------------------------------------------------------------------------
 // dequantisation of one weight row of one tile into the swizzled B operand
 // ---------------------------------------------------------------------------
-__device__ __forceinline__ void store_pairs_sw128(uint8_t* btile, int r, int chunk,
-                                                  const uint32_t (&p)[4]) {
-  uint8_t* dst = btile + (r >> 3) * 1024 + (r & 7) * 128 + ((chunk ^ (r & 7)) << 4);
+// Row r, 16-byte chunk c (0..3) of a K-major tile with 64-byte rows and the
+// 64-byte swizzle (chunk index XOR bits 7..8 of the address).
+__device__ __forceinline__ void store_pairs_sw64(uint8_t* btile, int r, int chunk,
+                                                 const uint32_t (&p)[4]) {
+  uint8_t* dst = btile + r * 64 + ((chunk ^ ((r >> 1) & 3)) << 4);
   *reinterpret_cast<uint4*>(dst) = make_uint4(p[0], p[1], p[2], p[3]);
+}
+
+__device__ __forceinline__ void red_add_v4(float* p, float a, float b, float c, float d) {
+  asm volatile("red.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(p), "f"(a), "f"(b), "f"(c),
+               "f"(d)
+               : "memory");
 }
 
 __device__ __forceinline__ uint32_t dq_pair(uint32_t raw, __half2 zz, __half2 ss) {
@@ -153,7 +173,9 @@ __device__ __forceinline__ uint32_t dq_pair(uint32_t raw, __half2 zz, __half2 ss
   return *reinterpret_cast<const uint32_t*>(&w);
 }
 
-__device__ __forceinline__ void dequant_row(int bits, const uint8_t* row_bytes, uint32_t meta,
+// Dequantise 32 codes of weight row r.  `w` holds the row's code words
+// starting at the first code (2-bit: 2 words, 3-bit: 3, 4-bit: 4, 8-bit: 8).
+__device__ __forceinline__ void dequant_row(int bits, const uint32_t (&w)[8], uint32_t meta,
                                             uint8_t* btile, int r) {
   const uint32_t magic = 0x64006400u;
   const __half s = __ushort_as_half((uint16_t)(meta & 0xFFFFu));
@@ -161,78 +183,52 @@ __device__ __forceinline__ void dequant_row(int bits, const uint8_t* row_bytes, 
   const __half2 ss = __halves2half2(s, s);
   const __half zz1 = __hadd(z, __float2half(1024.f));
   const __half2 zz = __halves2half2(zz1, zz1);
-  const uint2* src = reinterpret_cast<const uint2*>(row_bytes);  // 8-byte aligned
   if (bits == 2) {
 #pragma unroll
-    for (int wp = 0; wp < 2; ++wp) {
-      const uint2 ww = src[wp];
-      const uint32_t w2[2] = {ww.x, ww.y};
+    for (int wd = 0; wd < 2; ++wd) {
 #pragma unroll
-      for (int q = 0; q < 2; ++q) {
-        const uint32_t w = w2[q];
-        const int wd = 2 * wp + q;
+      for (int c2 = 0; c2 < 2; ++c2) {
+        uint32_t p[4];
 #pragma unroll
-        for (int c2 = 0; c2 < 2; ++c2) {
-          uint32_t p[4];
-#pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            const int ii = 4 * c2 + i;
-            p[i] = dq_pair(((w >> (2 * ii)) & 0x00030003u) | magic, zz, ss);
-          }
-          store_pairs_sw128(btile, r, 2 * wd + c2, p);
+        for (int i = 0; i < 4; ++i) {
+          const int ii = 4 * c2 + i;
+          p[i] = dq_pair(((w[wd] >> (2 * ii)) & 0x00030003u) | magic, zz, ss);
         }
+        store_pairs_sw64(btile, r, 2 * wd + c2, p);
       }
     }
   } else if (bits == 3) {
-    uint32_t w[6];
+    const uint32_t a = w[0], b = w[1], c = w[2];
 #pragma unroll
-    for (int k = 0; k < 3; ++k) {
-      const uint2 ww = src[k];
-      w[2 * k] = ww.x;
-      w[2 * k + 1] = ww.y;
-    }
+    for (int c4 = 0; c4 < 4; ++c4) {
+      uint32_t p[4];
 #pragma unroll
-    for (int u = 0; u < 2; ++u) {
-      const uint32_t a = w[3 * u], b = w[3 * u + 1], c = w[3 * u + 2];
-#pragma unroll
-      for (int c4 = 0; c4 < 4; ++c4) {
-        uint32_t p[4];
-#pragma unroll
-        for (int i4 = 0; i4 < 4; ++i4) {
-          const int i = 4 * c4 + i4;  // codes i and i + 16 of this 32-code unit
-          const int o = 3 * i;
-          const uint32_t lo = o < 32 ? __funnelshift_r(a, b, o) : __funnelshift_r(b, c, o - 32);
-          const uint32_t hi = o < 32 ? __funnelshift_r(b, c, o) : (c >> (o - 32));
-          const uint32_t m2 = __byte_perm(lo, hi, 0x7610);
-          p[i4] = dq_pair((m2 & 0x00070007u) | magic, zz, ss);
-        }
-        store_pairs_sw128(btile, r, 4 * u + c4, p);
+      for (int i4 = 0; i4 < 4; ++i4) {
+        const int i = 4 * c4 + i4;  // codes i and i + 16
+        const int o = 3 * i;
+        const uint32_t lo = o < 32 ? __funnelshift_r(a, b, o) : __funnelshift_r(b, c, o - 32);
+        const uint32_t hi = o < 32 ? __funnelshift_r(b, c, o) : (c >> (o - 32));
+        p[i4] = dq_pair((__byte_perm(lo, hi, 0x7610) & 0x00070007u) | magic, zz, ss);
       }
+      store_pairs_sw64(btile, r, c4, p);
     }
   } else if (bits == 4) {
 #pragma unroll
-    for (int wp = 0; wp < 4; ++wp) {
-      const uint2 ww = src[wp];
-      const uint32_t w2[2] = {ww.x, ww.y};
+    for (int wd = 0; wd < 4; ++wd) {
+      uint32_t p[4];
 #pragma unroll
-      for (int q = 0; q < 2; ++q) {
-        const uint32_t w = w2[q];
-        uint32_t p[4];
-#pragma unroll
-        for (int i = 0; i < 4; ++i) p[i] = dq_pair(((w >> (4 * i)) & 0x000F000Fu) | magic, zz, ss);
-        store_pairs_sw128(btile, r, 2 * wp + q, p);
-      }
+      for (int i = 0; i < 4; ++i) p[i] = dq_pair(((w[wd] >> (4 * i)) & 0x000F000Fu) | magic, zz, ss);
+      store_pairs_sw64(btile, r, wd, p);
     }
   } else {  // 8-bit
 #pragma unroll
-    for (int wp = 0; wp < 8; ++wp) {
-      const uint2 ww = src[wp];
+    for (int c = 0; c < 4; ++c) {
       uint32_t p[4];
-      p[0] = dq_pair(__byte_perm(ww.x, 0x64646464u, 0x4140), zz, ss);
-      p[1] = dq_pair(__byte_perm(ww.x, 0x64646464u, 0x4342), zz, ss);
-      p[2] = dq_pair(__byte_perm(ww.y, 0x64646464u, 0x4140), zz, ss);
-      p[3] = dq_pair(__byte_perm(ww.y, 0x64646464u, 0x4342), zz, ss);
-      store_pairs_sw128(btile, r, wp, p);
+      p[0] = dq_pair(__byte_perm(w[2 * c], 0x64646464u, 0x4140), zz, ss);
+      p[1] = dq_pair(__byte_perm(w[2 * c], 0x64646464u, 0x4342), zz, ss);
+      p[2] = dq_pair(__byte_perm(w[2 * c + 1], 0x64646464u, 0x4140), zz, ss);
+      p[3] = dq_pair(__byte_perm(w[2 * c + 1], 0x64646464u, 0x4342), zz, ss);
+      store_pairs_sw64(btile, r, c, p);
     }
   }
 }
@@ -297,15 +293,18 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
       pdl_wait();  // Xg comes from the pre-pass
       int kg = 0;
       for (int u = blockIdx.x; u < P.units && !s_abort; u += gridDim.x) {
-        const int um = u % P.units_m, un = u / P.units_m;
-        for (int kt = 0; kt < KT && !s_abort; ++kt, ++kg) {
+        const int um = u % P.units_m, un = (u / P.units_m) % P.units_n;
+        const int ks = u / (P.units_m * P.units_n);
+        const int kt_lo = (int)((long long)ks * KT / P.ksplit);
+        const int kt_hi = (int)((long long)(ks + 1) * KT / P.ksplit);
+        for (int kt = kt_lo; kt < kt_hi && !s_abort; ++kt, ++kg) {
           const int s = kg % kStagesG, use = kg / kStagesG;
           if (use > 0 && !mbar_wait(smem_u32(&bar_sfree[s]), (use - 1) & 1)) {
             fail(kStatusTimeoutEmpty);
             break;
           }
           const GmBlock& B = sblk[find_kblock(sblk, nblk, kt)];
-          const int g = kt - B.kt0;
+          const int hg = kt - B.kt0;  // half group
           uint8_t* st = stage_ptr(s);
           const uint32_t bar = smem_u32(&bar_full[s]);
           const bool w16 = B.bits == 16;
@@ -314,14 +313,14 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
           for (int t = 0; t < MT; ++t)
             tma_load_2d(smem_u32(st + t * kATile), &P.tm_x, kt * BK, um * (MT * BM) + t * BM, bar);
           if (w16) {
-            tma_load_2d(smem_u32(st + MT * kATile), &P.tm_w16, (B.seg_off + 128 * g) / 2, un * BN,
+            tma_load_2d(smem_u32(st + MT * kATile), &P.tm_w16, (B.seg_off + 64 * hg) / 2, un * BN,
                         bar);
           } else {
-            const int start = B.seg_off + 8 * B.bits * g;
+            const int start = B.seg_off + 4 * B.bits * hg;
             tma_load_2d(smem_u32(st + MT * kATile + kBTile), &P.tm_codes, start & ~15, un * BN,
                         bar);
             tma_load_2d(smem_u32(st + MT * kATile + kBTile + kCodes), &P.tm_meta,
-                        (B.grp_off + g) & ~3, un * BN, bar);
+                        (B.grp_off + hg / 2) & ~3, un * BN, bar);
           }
         }
       }
@@ -331,12 +330,15 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
     if (lane == 0) {
       int kg = 0, uc = 0;
       for (int u = blockIdx.x; u < P.units && !s_abort; u += gridDim.x, ++uc) {
+        const int ks = u / (P.units_m * P.units_n);
+        const int kt_lo = (int)((long long)ks * KT / P.ksplit);
+        const int kt_hi = (int)((long long)(ks + 1) * KT / P.ksplit);
         if (uc > 0 && !mbar_wait(smem_u32(&bar_acce), (uc - 1) & 1)) {
           fail(kStatusTimeoutEmpty);
           break;
         }
         tc_fence_after();
-        for (int kt = 0; kt < KT && !s_abort; ++kt, ++kg) {
+        for (int kt = kt_lo; kt < kt_hi && !s_abort; ++kt, ++kg) {
           const int s = kg % kStagesG, use = kg / kStagesG;
           if (!mbar_wait(smem_u32(&bar_full[s]), use & 1) ||
               !mbar_wait(smem_u32(&bar_bready[s]), use & 1)) {
@@ -351,8 +353,8 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
             const uint32_t a0 = smem_u32(st + t * kATile);
 #pragma unroll
             for (int kk = 0; kk < BK / 16; ++kk)
-              tc_mma_f16(tmem + t * BN, umma_desc_sw128(a0 + 32 * kk), umma_desc_sw128(b0 + 32 * kk),
-                         kIdesc, (kt > 0 || kk > 0) ? 1u : 0u);
+              tc_mma_f16(tmem + t * BN, umma_desc_sw64(a0 + 32 * kk), umma_desc_sw64(b0 + 32 * kk),
+                         kIdesc, (kt > kt_lo || kk > 0) ? 1u : 0u);
           }
           tc_commit(smem_u32(&bar_sfree[s]));
         }
@@ -366,8 +368,11 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
     const int half = (warp - 2) >> 2;
     int kg = 0, uc = 0;
     for (int u = blockIdx.x; u < P.units && !s_abort; u += gridDim.x, ++uc) {
-      const int um = u % P.units_m, un = u / P.units_m;
-      for (int kt = 0; kt < KT && !s_abort; ++kt, ++kg) {
+      const int um = u % P.units_m, un = (u / P.units_m) % P.units_n;
+      const int ks = u / (P.units_m * P.units_n);
+      const int kt_lo = (int)((long long)ks * KT / P.ksplit);
+      const int kt_hi = (int)((long long)(ks + 1) * KT / P.ksplit);
+      for (int kt = kt_lo; kt < kt_hi && !s_abort; ++kt, ++kg) {
         const int s = kg % kStagesG, use = kg / kStagesG;
         if (!mbar_wait(smem_u32(&bar_full[s]), use & 1) ||
             (use > 0 && !mbar_wait(smem_u32(&bar_sfree[s]), (use - 1) & 1))) {
@@ -376,13 +381,39 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
         }
         const GmBlock& B = sblk[find_kblock(sblk, nblk, kt)];
         if (B.bits != 16) {
-          const int g = kt - B.kt0;
+          const int hg = kt - B.kt0;
           uint8_t* st = stage_ptr(s);
-          const int start = B.seg_off + 8 * B.bits * g;
-          const uint8_t* row_bytes = st + MT * kATile + kBTile + r * kCodeBox + (start & 15);
+          const int start = B.seg_off + 4 * B.bits * hg;
+          // the row's code bytes start at offset (start & 15) of a 16-byte
+          // aligned window; two conflict-free 16-byte reads cover them
+          const uint4* rp = reinterpret_cast<const uint4*>(st + MT * kATile + kBTile + r * kCodeBox);
+          const uint4 c0 = rp[0], c1 = rp[1];
+          const uint32_t cw[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
+          uint32_t w[8];
+          switch ((start & 15) >> 2) {  // uniform over the CTA
+            case 0:
+#pragma unroll
+              for (int k = 0; k < 8; ++k) w[k] = cw[k];
+              break;
+            case 1:
+#pragma unroll
+              for (int k = 0; k < 7; ++k) w[k] = cw[k + 1];
+              w[7] = 0;
+              break;
+            case 2:
+#pragma unroll
+              for (int k = 0; k < 6; ++k) w[k] = cw[k + 2];
+              w[6] = w[7] = 0;
+              break;
+            default:
+#pragma unroll
+              for (int k = 0; k < 5; ++k) w[k] = cw[k + 3];
+              w[5] = w[6] = w[7] = 0;
+              break;
+          }
           const uint32_t meta = reinterpret_cast<const uint32_t*>(
-              st + MT * kATile + kBTile + kCodes)[r * 4 + ((B.grp_off + g) & 3)];
-          dequant_row(B.bits, row_bytes, meta, st + MT * kATile, r);
+              st + MT * kATile + kBTile + kCodes)[r * 4 + ((B.grp_off + hg / 2) & 3)];
+          dequant_row(B.bits, w, meta, st + MT * kATile, r);
           fence_proxy_async_smem();
         }
         __syncwarp();
@@ -407,7 +438,19 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
           const int n0 = un * BN + col;
           if (m < P.M) {
             float* dst = P.y + (size_t)m * P.N + n0;
-            if (n0 + 32 <= P.N && (P.N % 4) == 0) {
+            const bool vec = n0 + 32 <= P.N && (P.N % 4) == 0;
+            if (P.ksplit > 1) {  // Y was zeroed by the pre-pass: add this K range
+              if (vec) {
+#pragma unroll
+                for (int j = 0; j < 8; ++j)
+                  red_add_v4(dst + 4 * j, __uint_as_float(v[4 * j]), __uint_as_float(v[4 * j + 1]),
+                             __uint_as_float(v[4 * j + 2]), __uint_as_float(v[4 * j + 3]));
+              } else {
+#pragma unroll
+                for (int j = 0; j < 32; ++j)
+                  if (n0 + j < P.N) atomicAdd(dst + j, __uint_as_float(v[j]));
+              }
+            } else if (vec) {
 #pragma unroll
               for (int j = 0; j < 8; ++j)
                 reinterpret_cast<float4*>(dst)[j] =
@@ -458,7 +501,7 @@ int k_tiles(const polyq_dev_layer* L, GmBlock* blk) {
     g.grp_off = b.grp_off;
     g.n_grp = b.n_grp;
     g.kt0 = kt;
-    g.n_kt = (b.n_ch + BK - 1) / BK;
+    g.n_kt = (b.n_ch + BK - 1) / BK;  // half groups
     kt += g.n_kt;
     if (blk) blk[i] = g;
   }
@@ -509,20 +552,20 @@ extern "C" int polyq_linear_gemm(const polyq_dev_layer* L, const void* X, int64_
   P.K = (int)L->K;
   P.KT = KT;
   P.units_m = (int)((M + MT * BM - 1) / (MT * BM));
-  P.units = P.units_m * (int)((L->N + BN - 1) / BN);
+  P.units_n = (int)((L->N + BN - 1) / BN);
   P.x = (const __nv_bfloat16*)X;
   P.gather = L->gather;
   P.xg = (__half*)workspace;
   P.y = Y;
   P.status = (int*)((uint8_t*)workspace + need - 256);
   rc = polyq_tensor_map_2d(&P.tm_x, P.xg, 2, (uint64_t)KT * BK, (uint64_t)M, (uint64_t)KT * BK * 2,
-                           BK, BM, 1);
+                           BK, BM, 64);
   if (rc) return rc;
   rc = polyq_tensor_map_2d(&P.tm_codes, L->packed, 1, (uint64_t)L->row_stride, (uint64_t)L->N,
                            (uint64_t)L->row_stride, kCodeBox, BN);
   if (rc) return rc;
   rc = polyq_tensor_map_2d(&P.tm_w16, L->packed, 2, (uint64_t)L->row_stride / 2, (uint64_t)L->N,
-                           (uint64_t)L->row_stride, BK, BN, 1);
+                           (uint64_t)L->row_stride, BK, BN, 64);
   if (rc) return rc;
   if (L->n_groups > 0) {
     rc = polyq_tensor_map_2d(&P.tm_meta, L->meta, 4, (uint64_t)L->meta_stride, (uint64_t)L->N,
@@ -535,6 +578,16 @@ extern "C" int polyq_linear_gemm(const polyq_dev_layer* L, const void* X, int64_
   int sms = 0;
   rc = polyq_sm_count(&sms);
   if (rc) return rc;
+  // Split K when there are too few (M, N) tiles to keep two waves of SMs busy;
+  // each split keeps at least 16 K tiles.
+  {
+    const int mn = P.units_m * P.units_n;
+    int ks = 1;
+    if (mn < 2 * sms) ks = std::min((2 * sms + mn - 1) / mn, std::max(1, KT / 16));
+    if (ks > 1 && (P.N % 4) != 0) ks = 1;  // the zeroing pass writes float4
+    P.ksplit = ks;
+    P.units = mn * ks;
+  }
   static bool attr_done[8] = {false};
   int dev = 0;
   cudaGetDevice(&dev);

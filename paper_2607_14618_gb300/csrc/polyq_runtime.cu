@@ -59,8 +59,8 @@ int polyq_sm_count(int* out) {
 
 int polyq_tensor_map_2d(CUtensorMap* out, const void* base, int elem_bytes, uint64_t cols,
                         uint64_t rows, uint64_t row_stride_bytes, uint32_t box_cols,
-                        uint32_t box_rows, int swizzle128) {
-  Key k{(uintptr_t)base, elem_bytes, cols, rows, row_stride_bytes, box_cols, box_rows, swizzle128};
+                        uint32_t box_rows, int swizzle_bytes) {
+  Key k{(uintptr_t)base, elem_bytes, cols, rows, row_stride_bytes, box_cols, box_rows, swizzle_bytes};
   std::lock_guard<std::mutex> lk(g_mu);
   auto it = g_maps.find(k);
   if (it != g_maps.end()) {
@@ -81,7 +81,9 @@ int polyq_tensor_map_2d(CUtensorMap* out, const void* base, int elem_bytes, uint
   std::memset(&m, 0, sizeof m);
   CUresult r = enc(&m, dt, 2, const_cast<void*>(base), dims, strides, box, es,
                    CU_TENSOR_MAP_INTERLEAVE_NONE,
-                   swizzle128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
+                   swizzle_bytes == 128  ? CU_TENSOR_MAP_SWIZZLE_128B
+                   : swizzle_bytes == 64 ? CU_TENSOR_MAP_SWIZZLE_64B
+                                         : CU_TENSOR_MAP_SWIZZLE_NONE,
                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS)
     return polyq_set_error(POLYQ_ECUDA, "cuTensorMapEncodeTiled failed (%d)", (int)r);

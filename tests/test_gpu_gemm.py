@@ -48,7 +48,8 @@ def test_gemm_identity_gather_and_repeat(polyq_lib):
     Y2 = polyq_lib.linear_gemm(dev, _x_dev(Xs), workspace=ws)
     torch.cuda.synchronize()
     check_tolerance(Y1.cpu().numpy(), O.linear(ref, X), X, 1200)
-    assert torch.equal(Y1, Y2)  # no atomics: deterministic
+    # a small problem splits K over CTAs: repeated runs agree to fp32 rounding
+    assert torch.allclose(Y1, Y2, rtol=1e-5, atol=1e-5 * float(Y1.abs().max()))
 
 
 @pytest.mark.parametrize("name,N,K,M", [
