@@ -187,6 +187,36 @@ int polyq_linear_gemv(const polyq_dev_layer* layer, const void* x, int batch,
                       float* y, const float* residual, void* workspace,
                       size_t workspace_bytes, void* stream);
 
+/* Scratch, in bytes, compiled into the library for polyq_linear_gemv_noalloc
+ * (1 MiB).  A layer needs 256 bytes plus, per input channel, from about 2.3
+ * bytes (batch 1, widths 2-4) up to 21 bytes (batch 4, width 8), rounded up
+ * to whole steps; so every layer with K <= 49152 fits at any batch and any
+ * mix of widths. */
+#define POLYQ_NOALLOC_SCRATCH_BYTES (1u << 20)
+
+/* polyq_linear_gemv without a workspace argument: it allocates no device
+ * memory and takes none from the caller.  The paper has no counterpart; this
+ * is for callers that cannot allocate, such as a plugin living inside a host
+ * program that owns all device memory through its own pool and hands out no
+ * allocation hook, or a latency-bound loop that may not take the device-wide
+ * synchronisation that cudaMalloc and cudaFree can cause.
+ *
+ * The scratch is one fixed array of POLYQ_NOALLOC_SCRATCH_BYTES compiled into
+ * this library; each device that loads the library keeps its copy until the
+ * process exits.  The first call on a device, with that device current, looks
+ * up the array's device address once (cudaGetSymbolAddress); make that first
+ * call before any stream capture on that device.  Every call on a device uses
+ * the same array, so calls whose kernels may overlap on the GPU (different
+ * streams, or different host threads without ordering) race and corrupt each
+ * other's results; serialise them, e.g. on one stream.  The kernels rewrite
+ * every byte of scratch they read on each call and zero the status word
+ * themselves, so nothing left by an earlier call leaks into a later one.
+ * Arguments and results are those of polyq_linear_gemv.  Returns
+ * POLYQ_ENOMEM, touching nothing, when the layer and batch need more than
+ * POLYQ_NOALLOC_SCRATCH_BYTES (see polyq_gemv_workspace_bytes). */
+int polyq_linear_gemv_noalloc(const polyq_dev_layer* layer, const void* x, int batch,
+                              float* y, const float* residual, void* stream);
+
 /* Device scratch bytes polyq_linear_gemv_group needs for these layers. */
 int polyq_gemv_group_workspace_bytes(const polyq_dev_layer* const* layers,
                                      int n, int batch, size_t* bytes);

@@ -29,6 +29,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <mutex>
 
 #include "polyq.h"
 #include "polyq_dev.cuh"
@@ -792,4 +793,74 @@ extern "C" int polyq_linear_gemv_group(const polyq_dev_layer* const* layers, int
   polyq_clear_error();
   return gemv_group("polyq_linear_gemv_group", layers, n, xs, batch, ys, residuals, workspace,
                     ws_bytes, (cudaStream_t)stream);
+}
+
+// ---------------------------------------------------------------------------
+// the same GEMV with library-owned scratch instead of a caller workspace
+// ---------------------------------------------------------------------------
+// Some callers cannot allocate device memory: a plugin inside a host program
+// whose own pool owns the device, or a latency-bound loop that cannot take the
+// device-wide synchronisation cudaMalloc/cudaFree may cause.  For them the
+// records and the status word live in this fixed array, one copy per device
+// that loads the library, kept until the process exits.  In host code the name
+// below stands for a host-side shadow, never the device address: the address
+// is looked up with cudaGetSymbolAddress, once per device.
+static __device__ __align__(256) uint8_t polyq_noalloc_scratch[POLYQ_NOALLOC_SCRATCH_BYTES];
+
+namespace {
+
+constexpr int kMaxDevices = 64;
+std::mutex g_noalloc_mu;
+void* g_noalloc_ptr[kMaxDevices] = {};
+
+// Device address of the scratch array on the current device; the first call
+// per device does the lookup (so it must precede any stream capture there).
+int noalloc_scratch(void** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess)
+    return polyq_set_error(POLYQ_ECUDA, "polyq_linear_gemv_noalloc: cudaGetDevice: %s",
+                           cudaGetErrorString(e));
+  if (dev < 0 || dev >= kMaxDevices)
+    return polyq_set_error(POLYQ_EUNSUPPORTED, "polyq_linear_gemv_noalloc: device %d >= %d",
+                           dev, kMaxDevices);
+  std::lock_guard<std::mutex> lk(g_noalloc_mu);
+  if (!g_noalloc_ptr[dev]) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, polyq_noalloc_scratch);
+    if (e != cudaSuccess || !p)
+      return polyq_set_error(POLYQ_ECUDA,
+                             "polyq_linear_gemv_noalloc: scratch address on device %d: %s", dev,
+                             cudaGetErrorString(e));
+    g_noalloc_ptr[dev] = p;
+  }
+  *out = g_noalloc_ptr[dev];
+  return POLYQ_OK;
+}
+
+}  // namespace
+
+extern "C" int polyq_linear_gemv_noalloc(const polyq_dev_layer* L, const void* x, int batch,
+                                         float* y, const float* residual, void* stream) {
+  polyq_clear_error();
+  const char* who = "polyq_linear_gemv_noalloc";
+  const polyq_dev_layer* one[1] = {L};
+  int rc = check_group(who, one, 1, batch);
+  if (rc) return rc;
+  const size_t need = workspace_for(one, 1, batch);
+  if (need > POLYQ_NOALLOC_SCRATCH_BYTES)
+    return polyq_set_error(POLYQ_ENOMEM,
+                           "%s: this layer at batch %d needs %zu bytes of scratch, above the "
+                           "fixed maximum of %u; call polyq_linear_gemv with a workspace",
+                           who, batch, need, (unsigned)POLYQ_NOALLOC_SCRATCH_BYTES);
+  void* scratch = nullptr;
+  rc = noalloc_scratch(&scratch);
+  if (rc) return rc;
+  // gemv_prep writes every record the main kernel reads and zeroes the status
+  // word before anything reads it, so stale contents need no clearing here.
+  const void* xs[1] = {x};
+  float* ys[1] = {y};
+  const float* rs[1] = {residual};
+  return gemv_group(who, one, 1, xs, batch, ys, rs, scratch, POLYQ_NOALLOC_SCRATCH_BYTES,
+                    (cudaStream_t)stream);
 }

@@ -23,6 +23,7 @@ POLYQ_ETIMEOUT = -5
 MAX_BLOCKS = 5
 MAX_GROUP = 4
 GROUP = 64
+NOALLOC_SCRATCH_BYTES = 1 << 20  # scratch compiled in for linear_gemv_noalloc
 ALLOC_WATERFILL = 0
 ALLOC_LADDER = 1
 
@@ -81,6 +82,7 @@ _SIGS = {
     "polyq_dev_layer_fill": (C.c_int, [_P, _P, _P, _P, C.POINTER(DevLayer)]),
     "polyq_gemv_workspace_bytes": (C.c_int, [C.POINTER(DevLayer), C.c_int, C.POINTER(C.c_size_t)]),
     "polyq_linear_gemv": (C.c_int, [C.POINTER(DevLayer), _P, C.c_int, _P, _P, _P, C.c_size_t, _P]),
+    "polyq_linear_gemv_noalloc": (C.c_int, [C.POINTER(DevLayer), _P, C.c_int, _P, _P, _P]),
     "polyq_gemv_group_workspace_bytes": (C.c_int, [C.POINTER(C.POINTER(DevLayer)), C.c_int,
                                                    C.c_int, C.POINTER(C.c_size_t)]),
     "polyq_linear_gemv_group": (C.c_int, [C.POINTER(C.POINTER(DevLayer)), C.c_int,
@@ -270,6 +272,30 @@ def linear_gemv(layer: DeviceLayer, x, y=None, residual=None, workspace=None, st
     _check(_lib.polyq_linear_gemv(C.byref(layer.desc), x.data_ptr(), batch, y.data_ptr(),
                                   residual.data_ptr() if residual is not None else None,
                                   ws_ptr, ws_len, _stream_ptr(stream)))
+    return y
+
+
+def linear_gemv_noalloc(layer: DeviceLayer, x, y, residual=None, stream=None):
+    """linear_gemv on the library's fixed scratch array, for callers that cannot
+    allocate device memory (a plugin whose host program owns the device through
+    its own pool, or a loop that cannot take cudaMalloc's device-wide sync).
+
+    `y` must be passed: nothing is allocated here.  Calls that may overlap on
+    the GPU share the scratch and race; the first call on a device looks up the
+    scratch address and should come before any stream capture there.
+    """
+    import torch
+    if x.dtype != torch.bfloat16 or not x.is_cuda or x.dim() != 2 or x.shape[1] != layer.K:
+        raise ValueError("x must be a CUDA bf16 tensor [batch][K]")
+    if not x.is_contiguous():
+        raise ValueError("x must be contiguous (no copy is made here)")
+    batch = x.shape[0]
+    if (y is None or y.dtype != torch.float32 or not y.is_contiguous()
+            or tuple(y.shape) != (batch, layer.N)):
+        raise ValueError("y must be a contiguous CUDA fp32 tensor [batch][N]")
+    _check(_lib.polyq_linear_gemv_noalloc(C.byref(layer.desc), x.data_ptr(), batch, y.data_ptr(),
+                                          residual.data_ptr() if residual is not None else None,
+                                          _stream_ptr(stream)))
     return y
 
 

@@ -1,0 +1,87 @@
+"""polyq_linear_gemv_noalloc: the decode GEMV on the library's own fixed scratch.
+
+Some callers cannot allocate device memory (a plugin inside a host program
+whose memory pool owns the device, or a loop that cannot take the device-wide
+synchronisation cudaMalloc/cudaFree may cause), so this entry point takes no
+workspace.  Its results must match polyq_linear_gemv's on the same inputs,
+call after call, although every call reuses the same scratch array.  The file
+name makes pytest collect it last.
+"""
+import numpy as np
+import pytest
+
+from paper_2607_14618_gb300 import synth
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+
+def _x_dev(xb):
+    return torch.from_numpy(np.ascontiguousarray(xb).view(np.int16)).cuda().view(torch.bfloat16)
+
+
+def _same(got, ref):
+    # two runs of the GEMV kernels differ only in the order of the fp32 atomic
+    # additions of split tiles: the run-to-run tolerance of the GEMV tests
+    assert torch.allclose(got, ref, rtol=1e-5, atol=1e-5 * float(ref.abs().max()))
+
+
+def test_noalloc_matches_workspace_entry_on_two_calls(polyq_lib):
+    # call 1: a layer with all five widths at batch 4, no residual
+    W1, a1 = synth.layer_weights(1000, 3000, 71)
+    bits1 = synth.random_codes_layer_bits(3000, 71)
+    dev1 = polyq_lib.DeviceLayer(polyq_lib.HostLayer.pack(W1, a1, 3.0, forced_bits=bits1), "cuda")
+    xb1, _ = synth.activations(a1, 4, 71)
+    x1 = _x_dev(xb1)
+    # call 2: another layer at batch 1 with a residual, so that records left by
+    # call 1 (other shape, other batch) would show if they leaked through
+    W2, a2 = synth.layer_weights(2048, 2048, 72)
+    dev2 = polyq_lib.DeviceLayer(polyq_lib.HostLayer.pack(W2, a2, 3.0), "cuda")
+    xb2, _ = synth.activations(a2, 1, 72)
+    x2 = _x_dev(xb2)
+    res2 = torch.randn(1, 2048, device="cuda", dtype=torch.float32)
+
+    ref1 = polyq_lib.linear_gemv(dev1, x1)
+    ref2 = polyq_lib.linear_gemv(dev2, x2, residual=res2)
+    torch.cuda.synchronize()
+
+    y1 = torch.full((4, 1000), float("nan"), device="cuda")
+    y2 = torch.full((1, 2048), float("nan"), device="cuda")
+    polyq_lib.linear_gemv_noalloc(dev1, x1, y1)
+    polyq_lib.linear_gemv_noalloc(dev2, x2, y2, residual=res2)
+    torch.cuda.synchronize()
+    _same(y1, ref1)
+    _same(y2, ref2)
+
+    # the same two calls again, in the other order, on the now-used scratch
+    y2b = torch.full_like(y2, float("nan"))
+    y1b = torch.full_like(y1, float("nan"))
+    polyq_lib.linear_gemv_noalloc(dev2, x2, y2b, residual=res2)
+    polyq_lib.linear_gemv_noalloc(dev1, x1, y1b)
+    torch.cuda.synchronize()
+    _same(y1b, ref1)
+    _same(y2b, ref2)
+
+
+def test_noalloc_rejects_layers_beyond_the_scratch(polyq_lib):
+    # all 8-bit at batch 4 needs 21 bytes per input channel: K = 65536 needs
+    # about 1.3 MiB, above the fixed 1 MiB
+    N, K = 16, 65536
+    W, a = synth.layer_weights(N, K, 73)
+    bits = np.full(K, 8, dtype=np.uint8)
+    dev = polyq_lib.DeviceLayer(polyq_lib.HostLayer.pack(W, a, 8.0, forced_bits=bits), "cuda")
+    assert polyq_lib.gemv_workspace_bytes(dev, 4) > polyq_lib.NOALLOC_SCRATCH_BYTES
+    xb, _ = synth.activations(a, 4, 73)
+    y = torch.zeros(4, N, device="cuda")
+    with pytest.raises(polyq_lib.PolyqError) as e:
+        polyq_lib.linear_gemv_noalloc(dev, _x_dev(xb), y)
+    assert e.value.code == polyq_lib.POLYQ_ENOMEM
+    assert "scratch" in str(e.value)
+    torch.cuda.synchronize()
+    assert not bool(y.any())  # rejected before anything was launched
+    # the same layer at batch 1 fits (4.5 bytes per channel) and is served
+    ref = polyq_lib.linear_gemv(dev, _x_dev(xb[:1]))
+    y1 = torch.empty(1, N, device="cuda")
+    polyq_lib.linear_gemv_noalloc(dev, _x_dev(xb[:1]), y1)
+    torch.cuda.synchronize()
+    _same(y1, ref)
