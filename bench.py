@@ -36,6 +36,23 @@ WORKLOAD = ("llama2-13b decode linears q,k,v,o 5120x5120, gate,up 13824x5120, "
             "down 5120x13824; batch 1; B=3.0")
 # launches of one decoder layer: q/k/v and gate/up read the same input
 GROUPS = [(0, 1, 2), (3,), (4, 5), (6,)]
+# DRAM bytes (read + write) of one step's eight GEMV launches, summed from the
+# ncu launch list in profiles/gemv_decode_llama13b_b3_launches.md, with the
+# SHA-1 of the kernel sources it was taken on; reported as null once those
+# sources change.
+TRAFFIC = {"bytes_per_step": 143049000,
+           "sources_sha1": "5d2d6e2be369f248d55c0686925fb1beb0336c3f",
+           "profile": "profiles/gemv_decode_llama13b_b3_launches.md"}
+GEMV_SOURCES = ("polyq_gemv.cu", "polyq_gemv_layout.cuh", "polyq_dev.cuh")
+
+
+def _gemv_sources_sha1():
+    import hashlib
+    h = hashlib.sha1()
+    for f in GEMV_SOURCES:
+        with open(os.path.join(ROOT, "paper_2607_14618_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()
 
 
 def _peaks():
@@ -238,9 +255,14 @@ def run_polyq(args):
         per_lin_us[LLAMA[i][0]] = {"us": round(us, 2),
                                    "GB/s": round(per_lin_bytes[i] / (us * 1e-6) / 1e9, 1)}
     ach = step_bytes / (ms_step * 1e-3) / 1e9
+    traffic = (TRAFFIC["bytes_per_step"] if batch == 1 and args.budget == 3.0
+               and _gemv_sources_sha1() == TRAFFIC["sources_sha1"] else None)
     roof = {"bound": "hbm", "achieved": round(ach, 1), "peak": hbm, "unit": "GB/s",
-            "frac": round(ach / hbm, 4), "traffic": None, "peak_kind": peak_kind,
+            "frac": round(ach / hbm, 4), "traffic": traffic, "peak_kind": peak_kind,
             "kernel": "gemv_main (+ gemv_prep) of polyq_linear_gemv_group",
+            "launch_unit": "one step: 4 grouped GEMV calls (8 launches), "
+                           f"{step_bytes} algorithmic bytes",
+            "traffic_source": TRAFFIC["profile"] if traffic else None,
             "per_linear": per_lin_us}
 
     # end to end through the public API: pinned host x -> device, GEMVs, y -> host
