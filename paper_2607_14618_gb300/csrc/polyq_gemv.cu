@@ -1,34 +1,43 @@
 // Decode GEMV of the PolyQ mixed-bit layer (Section 4.1 factorisation with
-// the Section 4.2 bit blocks), one pass over all blocks of one or several
+// the Section 4.2 bit blocks), one launch over all blocks of one or several
 // independent layers:
 //
 //   y[b][n] = residual[b][n] + sum_p x[b][gather[p]] * W'[n][p]
 //
-// Two kernels per call:
-//  1. gemv_prep: for every step of every block, gathers the activations
-//     through `gather`, lays them out in the order the main kernel decodes the
-//     codes (scaled by the powers of two the decoder leaves on each code), sums
-//     them per chunk for the zero-point and magic-number corrections, and sets
-//     y to the residual (or zero).
-//  2. gemv_main: persistent CTAs; one producer warp streams 64-row tiles of
-//     packed codes and scale/zero metadata with TMA into a 3-stage
-//     shared-memory ring; four consumer warps turn each code pair into two
-//     exact bf16 values 128 + q*2^p with a single LOP3 and multiply them with
-//     the activations on the tensor cores (mma.sync m16n8k16, fp32
-//     accumulation).  Each MMA column holds one 64-code chunk, so a chunk's
-//     dot product is exact and its scale/zero are applied once:
-//        y += s * (D - 128*sum(x') - z*sum(x)).
-//     The (layer, tile, step) items of all layers of a call form one list;
-//     each CTA takes a contiguous range and keeps row sums in registers across
-//     a tile's steps.  A tile split between CTAs gets one fp32 atomic addition
-//     per piece into y, so the order of those few additions is not fixed from
-//     run to run.
+// Two kernels per call, chained with programmatic dependent launch:
+//  * gemv_prep, one CTA per (layer, step): gathers x through `gather`, scales
+//    each value by the power of two that the decoder leaves on its code,
+//    rounds it to fp16 and stores the step's activation record together with
+//    per-chunk sums for the magic-number and zero-point corrections.  The
+//    gather indices are loaded before the wait for the previous kernel.
+//  * gemv_main, persistent, 160 threads per CTA, 3 CTAs per SM.  The (layer,
+//    64-row tile, step) work items of all layers of the call form one list;
+//    each CTA takes a contiguous range of it.  Warp 4 (one thread) streams
+//    each item's packed codes and scale/zero metadata with TMA through a
+//    3-stage shared-memory ring, the first stages before the grid-dependency
+//    wait (weights do not depend on earlier kernels), and adds the item's
+//    record once the pre-pass is done.  Warps 0-3 each own 16 rows: a code
+//    pair becomes two exact fp16 values 1024 + q*2^p with one LOP3 against the
+//    register-held constant 0x64006400, and mma.sync m16n8k16 multiplies them
+//    with the record.  Each MMA column holds one 64-code chunk (one
+//    quantisation group), so a chunk's dot product D is exact up to fp32
+//    accumulation and its scale/zero apply once:
+//        y += s * (D - 1024*sum(x') - z*sum(x)).
+//    16-bit blocks feed their fp16 weights to the same MMA directly.
+//  * Row sums stay in registers across a tile's steps.  A tile whose steps
+//    are split over CTAs is finished by the CTA holding its first step (its
+//    "owner"): the other pieces, which are the first items of later CTAs,
+//    leave their sums in the workspace and count up a per-tile counter; the
+//    owner waits for the count, adds the pieces in CTA order and the
+//    residual, and stores y once.  Results are therefore reproducible bit for
+//    bit, and y is never read before it is written.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <cstring>
 #include <mutex>
 
 #include "polyq.h"
@@ -43,10 +52,16 @@ using namespace polyq::gv;
 
 constexpr int kCtasPerSm = 3;
 constexpr int kMaxGrid = 1024;  // persistent CTAs at most
+constexpr int kThreads = 32 * (kWarps + 1);
+constexpr int kConsumers = 32 * kWarps;
+constexpr int kStatusFixupTimeout = 3;
+// Upper bound on the time an owner waits for the other pieces of its tile.
+constexpr unsigned long long kFixupWaitNs = 2000000000ull;
 
 struct GvBlock {
-  int bits, n_ch, pos0, seg_off, grp_off, n_grp;
+  int bits, n_ch, pos0, seg_off, grp_off;
   int step0, n_steps;  // step range of this block inside its layer
+  int units;           // units per step
 };
 
 // One layer of a call.  Tensor maps first (64-byte aligned).
@@ -56,10 +71,11 @@ struct GvLayer {
   GvBlock blk[POLYQ_MAX_BLOCKS];
   int n_blocks;
   int N, K;
-  int steps;      // steps per row
-  int items;      // tiles * steps
-  int item0;      // first item of this layer in the call's list
-  int rec0;       // first record of this layer
+  int steps;  // steps per row
+  int items;  // tiles * steps
+  int item0;  // first item of this layer in the call's list
+  int tile0;  // first tile of this layer in the call's tile counters
+  int rec0;   // first activation record of this layer (one per step)
   const __nv_bfloat16* x;
   const int32_t* gather;
   float* y;
@@ -70,11 +86,14 @@ struct GvParams {
   GvLayer L[POLYQ_MAX_GROUP];
   int n_layers;
   int items;       // all layers
-  int recs;        // all layers' steps
+  int recs;        // activation records of all layers
   int batch;
-  uint32_t magic;  // 0x43004300 (two bf16 128.0), kept in a register
-  uint8_t* rec;    // recs * rec_bytes(NB)
-  int* status;
+  uint32_t magic;  // 0x64006400 (two fp16 1024.0), kept in a register
+  // workspace
+  int* status;     // sticky error word
+  uint32_t* cnt;   // [tiles][kWarps] piece counters, zero between calls
+  uint8_t* rec;    // [recs][rec_bytes(NB)] activation records
+  float* part;     // [grid][kRows][NB] piece sums
 };
 
 // Per-CTA shared copy of the scalars and block tables (runtime-indexed reads
@@ -85,7 +104,8 @@ struct GvShared {
   int N[POLYQ_MAX_GROUP];
   int steps[POLYQ_MAX_GROUP];
   int item0[POLYQ_MAX_GROUP + 1];
-  int rec0[POLYQ_MAX_GROUP];
+  int tile0[POLYQ_MAX_GROUP];
+  int rec0[POLYQ_MAX_GROUP + 1];
 };
 
 __device__ __forceinline__ void load_shared(const GvParams& P, GvShared* S) {
@@ -103,170 +123,256 @@ __device__ __forceinline__ void load_shared(const GvParams& P, GvShared* S) {
       S->N[l] = P.L[l].N;
       S->steps[l] = P.L[l].steps;
       S->item0[l] = P.L[l].item0;
+      S->tile0[l] = P.L[l].tile0;
       S->rec0[l] = P.L[l].rec0;
     }
   }
-  if (threadIdx.x == 0) S->item0[P.n_layers] = P.items;
-}
-
-__device__ __forceinline__ int find_block(const GvBlock* blk, int nblk, int s) {
-  int b = 0;
-  while (b + 1 < nblk && s >= blk[b + 1].step0) ++b;
-  return b;
-}
-
-__device__ __forceinline__ int find_layer(const int* starts, int nl, int v) {
-  int l = 0;
-  while (l + 1 < nl && v >= starts[l + 1]) ++l;
-  return l;
-}
-
-__device__ __forceinline__ uint32_t float_to_bf16_bits(float f) {
-  // values here are bf16 values scaled by powers of two: exact
-  return (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(f));
-}
-
-// ---------------------------------------------------------------------------
-// pre-pass: one CTA per step of every layer
-// ---------------------------------------------------------------------------
-template <int NB>
-__global__ void __launch_bounds__(256) gemv_prep(const __grid_constant__ GvParams P) {
-  pdl_trigger();
-  pdl_wait();  // x comes from the previous kernel; y and the workspace may still be in use
-  constexpr int CPL = cpl_of(NB);
-  constexpr int NG = ng_of(NB);
-  constexpr int U = units_of(NB);
-  constexpr int LW = rec_lane_words(NB);
-  __shared__ float xs_scaled[NB][U];
-  __shared__ float xs_plain[NB][U];
-  __shared__ GvShared S;
-  load_shared(P, &S);
-  __syncthreads();
-  const int nl = P.n_layers;
-  const int batch = P.batch;
-
-  // y starts as the residual (or zero); the main kernel adds its pieces
-#pragma unroll
-  for (int l = 0; l < POLYQ_MAX_GROUP; ++l) {
-    if (l >= nl) break;
-    float* y = P.L[l].y;
-    const float* res = P.L[l].residual;
-    if (y == res) continue;
-    const int total = batch * P.L[l].N;
-    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < total; i += gridDim.x * blockDim.x)
-      y[i] = res ? res[i] : 0.f;
+  if (threadIdx.x == 0) {
+    S->item0[P.n_layers] = P.items;
+    S->rec0[P.n_layers] = P.recs;
   }
-  if (blockIdx.x == 0 && threadIdx.x == 0) *P.status = 0;
+}
 
-  const int r = blockIdx.x;  // record index
-  if (r >= P.recs) return;
-  const int l = find_layer(S.rec0, nl, r);
-  const int s = r - S.rec0[l];
-  const int bi = find_block(S.blk[l], S.n_blocks[l], s);
-  const GvBlock B = S.blk[l][bi];
-  const int j = s - B.step0;
-  uint32_t* rec = reinterpret_cast<uint32_t*>(P.rec + (size_t)r * rec_bytes(NB));
-  const __nv_bfloat16* x = nullptr;
-  const int32_t* gather = nullptr;
-  int K = 0;
-#pragma unroll
-  for (int q = 0; q < POLYQ_MAX_GROUP; ++q)
-    if (q == l) {
-      x = P.L[q].x;
-      gather = P.L[q].gather;
-      K = P.L[q].K;
-    }
+// Position of a work item: layer, tile, step of the layer, block, step of the
+// block.  Items of a CTA are consecutive, so the position advances in place.
+struct ItemPos {
+  int l, tile, s, bi, j;
 
-  auto xval = [&](int b, int w) -> float {  // activation of block weight w
-    if (b >= batch || w >= B.n_ch) return 0.f;
-    const int p = B.pos0 + w;
-    const int src = gather ? gather[p] : p;
-    return __bfloat162float(x[(size_t)b * K + src]);
-  };
-
-  if (B.bits == 16) {
-    for (int e = threadIdx.x; e < NB * 4 * 16; e += blockDim.x) {
-      const int b = e / 64, t = (e / 16) % 4, k = e % 16;
-      const int w0 = j * kU16 + lane_weight16(t, 2 * k);
-      const int w1 = j * kU16 + lane_weight16(t, 2 * k + 1);
-      const uint32_t lo = float_to_bf16_bits(xval(b, w0));
-      const uint32_t hi = float_to_bf16_bits(xval(b, w1));
-      rec[(b * 4 + t) * LW + k] = lo | (hi << 16);
-    }
-    return;
+  __device__ __forceinline__ void init(const GvShared& S, int nl, int item) {
+    l = 0;
+    while (l + 1 < nl && item >= S.item0[l + 1]) ++l;
+    const int li = item - S.item0[l];
+    tile = li / S.steps[l];
+    s = li - tile * S.steps[l];
+    bi = 0;
+    while (bi + 1 < S.n_blocks[l] && s >= S.blk[l][bi + 1].step0) ++bi;
+    j = s - S.blk[l][bi].step0;
   }
-  const bool nib = B.bits == 8;
-  const int ub = ubits(B.bits);
-  // one thread per (lane t, pair j) of the step
-  for (int e = threadIdx.x; e < 4 * (CPL / 2); e += blockDim.x) {
-    const int t = e / (CPL / 2), jp = e % (CPL / 2);
-    int ulo, plo, uhi, phi;
-    pair_units(ub, jp, &ulo, &plo, &uhi, &phi);
-    const int su[2] = {lane_unit(B.bits, NB, t, ulo), lane_unit(B.bits, NB, t, uhi)};
-    const int pp[2] = {plo, phi};
-#pragma unroll
-    for (int b = 0; b < NB; ++b) {
-      float v[2];
-#pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        const int gu = j * U + su[h];  // unit index inside the block
-        float xv, scale = ldexpf(1.f, -pp[h]);
-        if (nib) {
-          xv = xval(b, gu >> 1);
-          if (gu & 1) scale *= 16.f;
-          xs_plain[b][su[h]] = (gu & 1) ? 0.f : xv;
-        } else {
-          xv = xval(b, gu);
-          xs_plain[b][su[h]] = xv;
-        }
-        v[h] = xv * scale;
-        xs_scaled[b][su[h]] = v[h];
+  __device__ __forceinline__ bool tile_end(const GvShared& S) const {
+    return s == S.steps[l] - 1;
+  }
+  __device__ __forceinline__ void next(const GvShared& S, int nl) {
+    ++s;
+    ++j;
+    if (s == S.steps[l]) {
+      s = 0;
+      j = 0;
+      bi = 0;
+      ++tile;
+      if (l + 1 < nl && S.item0[l] + tile * S.steps[l] >= S.item0[l + 1]) {
+        ++l;
+        tile = 0;
       }
-      rec[(b * 4 + t) * LW + jp] = float_to_bf16_bits(v[0]) | (float_to_bf16_bits(v[1]) << 16);
+    } else if (j == S.blk[l][bi].n_steps) {
+      ++bi;
+      j = 0;
     }
   }
-  __syncthreads();
-  // per-chunk sums in a fixed order: C1 = 128 * sum x', X = sum x
-  const int pw = rec_pair_words(NB);
-  float* recf = reinterpret_cast<float*>(rec);
-  for (int e = threadIdx.x; e < NB * NG; e += blockDim.x) {
-    const int b = e / NG, c = e % NG;
-    float c1 = 0.f, xx = 0.f;
-    for (int u = 64 * c; u < 64 * c + 64; ++u) {
-      c1 += xs_scaled[b][u];
-      xx += xs_plain[b][u];
-    }
-    recf[pw + b * NG + c] = 128.f * c1;
-    recf[pw + NB * NG + b * NG + c] = xx;
-  }
+};
+
+__device__ __forceinline__ const __nv_bfloat16* layer_x(const GvParams& P, int l) {
+  const __nv_bfloat16* x = P.L[0].x;
+#pragma unroll
+  for (int q = 1; q < POLYQ_MAX_GROUP; ++q)
+    if (q == l) x = P.L[q].x;
+  return x;
+}
+__device__ __forceinline__ const int32_t* layer_gather(const GvParams& P, int l) {
+  const int32_t* g = P.L[0].gather;
+#pragma unroll
+  for (int q = 1; q < POLYQ_MAX_GROUP; ++q)
+    if (q == l) g = P.L[q].gather;
+  return g;
+}
+__device__ __forceinline__ int layer_K(const GvParams& P, int l) {
+  int k = P.L[0].K;
+#pragma unroll
+  for (int q = 1; q < POLYQ_MAX_GROUP; ++q)
+    if (q == l) k = P.L[q].K;
+  return k;
+}
+
+
+__device__ __forceinline__ uint32_t pack_half2(__half lo, __half hi) {
+  return (uint32_t)__half_as_ushort(lo) | ((uint32_t)__half_as_ushort(hi) << 16);
 }
 
 // ---------------------------------------------------------------------------
-// main kernel
+// activation records (consumer warps, shared memory)
 // ---------------------------------------------------------------------------
-template <int UB>
+// Which activation values one consumer thread contributes to a record.  A
+// record has at most two slots per thread:
+//  * b < 16: slot s is the (batch, chunk) pair bc = warp + 4s of the step;
+//    lane q of the warp makes the q-th of the chunk's 32 lane pairs.
+//  * 16-bit: slot s is entry e = tid + 128s of the [batch][lane][16] pairs.
+struct SlotGeom {
+  bool valid;
+  int bb, c, t, jp;
+  int ch[2];  // channels (inside the block) of the pair's low and high half
+  int p[2];   // power-of-two scale exponents of the two halves
+};
+
+template <int NB, int BITS>
+__device__ __forceinline__ SlotGeom slot_geom_t(int warp, int lane, int tid, int s, int j,
+                                                const uint32_t* p3) {
+  SlotGeom g;
+  if constexpr (BITS == 16) {
+    const int e = tid + kConsumers * s;
+    g.valid = e < NB * 64;
+    g.bb = e / 64;
+    g.t = (e / 16) % 4;
+    g.jp = e % 16;
+    g.c = 0;
+    g.ch[0] = j * 128 + lane_weight16(g.t, 2 * g.jp);
+    g.ch[1] = j * 128 + lane_weight16(g.t, 2 * g.jp + 1);
+    g.p[0] = g.p[1] = 0;
+  } else {
+    constexpr int U = step_units(BITS, NB), NGS = U / 64;
+    constexpr int GP = group_pairs(BITS), GU = group_units(BITS);
+    const int bc = warp + kWarps * s;
+    g.valid = bc < NB * NGS;
+    g.bb = bc / NGS;
+    g.c = bc - g.bb * NGS;
+    chunk_pair(BITS, NB, g.c, lane, &g.t, &g.jp);
+    const int jj = g.jp % GP, base = (g.jp / GP) * GU;
+    int lo, hi;
+    if constexpr (BITS == 3) {
+      const uint32_t e = p3[jj];  // lo | hi << 8 | (win + 16) << 16
+      lo = (int)(e & 0xFF);
+      hi = (int)((e >> 8) & 0xFF);
+      const int win = (int)(e >> 16) - 16;
+      g.p[0] = 3 * lo - win;
+      g.p[1] = 3 * hi - win - 16;
+    } else {
+      const PairDef d = pair_def(BITS, jj);
+      lo = d.lo;
+      hi = d.hi;
+      g.p[0] = d.plo;
+      g.p[1] = d.phi;
+    }
+    g.ch[0] = j * U + lane_unit(BITS, NB, g.t, base + lo);
+    g.ch[1] = j * U + lane_unit(BITS, NB, g.t, base + hi);
+  }
+  return g;
+}
+
+template <int NB>
+__device__ __forceinline__ SlotGeom slot_geom(int bits, int warp, int lane, int tid, int s,
+                                              int j, const uint32_t* p3) {
+  switch (bits) {
+    case 2: return slot_geom_t<NB, 2>(warp, lane, tid, s, j, p3);
+    case 3: return slot_geom_t<NB, 3>(warp, lane, tid, s, j, p3);
+    case 4: return slot_geom_t<NB, 4>(warp, lane, tid, s, j, p3);
+    case 8: return slot_geom_t<NB, 8>(warp, lane, tid, s, j, p3);
+    default: return slot_geom_t<NB, 16>(warp, lane, tid, s, j, p3);
+  }
+}
+
+// A record is built once per call by the consumer warps of one CTA.
+// Pass 1: the gather indices (static layer data, so this may run before the
+// grid-dependency wait).
+template <int NB>
+__device__ __forceinline__ void rec_sources(const GvParams& P, const GvBlock& B, int l, int j,
+                                            int warp, int lane, const uint32_t* p3,
+                                            int (&src)[2][2]) {
+  const int32_t* gather = layer_gather(P, l);
+#pragma unroll
+  for (int s = 0; s < 2; ++s) {
+    src[s][0] = src[s][1] = -1;
+    const SlotGeom g = slot_geom<NB>(B.bits, warp, lane, threadIdx.x, s, j, p3);
+    if (g.valid && g.bb < P.batch) {
+#pragma unroll
+      for (int h = 0; h < 2; ++h)
+        if (g.ch[h] < B.n_ch) {
+          const int p = B.pos0 + g.ch[h];
+          src[s][h] = gather ? __ldg(gather + p) : p;
+        }
+    }
+  }
+}
+
+// Passes 2 and 3: load the activations, scale, round to fp16, store the
+// pairs and (b < 16) the per-chunk sums C1 = 1024 * sum x' and X = sum x.
+template <int NB>
+__device__ __forceinline__ void rec_build(const GvParams& P, const GvBlock& B, int l, int j,
+                                          int warp, int lane, const uint32_t* p3,
+                                          const int (&src)[2][2], uint32_t* rec) {
+  constexpr int LW = rec_lane_words(NB);
+  constexpr int PW = rec_pair_words(NB);
+  constexpr int NGM = 8 / NB;
+  const __nv_bfloat16* x = layer_x(P, l);
+  const int K = layer_K(P, l);
+  float xv[2][2];
+#pragma unroll
+  for (int s = 0; s < 2; ++s) {
+    const SlotGeom g = slot_geom<NB>(B.bits, warp, lane, threadIdx.x, s, j, p3);
+#pragma unroll
+    for (int h = 0; h < 2; ++h)
+      xv[s][h] = src[s][h] >= 0 ? __bfloat162float(x[(size_t)g.bb * K + src[s][h]]) : 0.f;
+  }
+  float* recf = reinterpret_cast<float*>(rec);
+#pragma unroll
+  for (int s = 0; s < 2; ++s) {
+    const SlotGeom g = slot_geom<NB>(B.bits, warp, lane, threadIdx.x, s, j, p3);
+    if (!g.valid) continue;  // uniform over the warp for b < 16
+    const __half hlo = __float2half_rn(ldexpf(xv[s][0], -g.p[0]));
+    const __half hhi = __float2half_rn(ldexpf(xv[s][1], -g.p[1]));
+    rec[(g.bb * 4 + g.t) * LW + g.jp] = pack_half2(hlo, hhi);
+    if (B.bits != 16) {
+      float s1 = __half2float(hlo) + __half2float(hhi);
+      float s2 = xv[s][0] + xv[s][1];
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        s1 += __shfl_xor_sync(0xffffffffu, s1, o);
+        s2 += __shfl_xor_sync(0xffffffffu, s2, o);
+      }
+      if (lane == 0) {
+        recf[PW + g.bb * NGM + g.c] = kMagicF * s1;
+        recf[PW + NB * NGM + g.bb * NGM + g.c] = s2;
+      }
+    }
+  }
+}
+
+// Layer, block and block step of record r.
+__device__ __forceinline__ void rec_pos(const GvShared& S, int nl, int r, int* l, int* bi,
+                                        int* j) {
+  int q = 0;
+  while (q + 1 < nl && r >= S.rec0[q + 1]) ++q;
+  const int s = r - S.rec0[q];
+  int b = 0;
+  while (b + 1 < S.n_blocks[q] && s >= S.blk[q][b + 1].step0) ++b;
+  *l = q;
+  *bi = b;
+  *j = s - S.blk[q][b].step0;
+}
+
+// ---------------------------------------------------------------------------
+// MMA steps
+// ---------------------------------------------------------------------------
+template <int BITS>
 __device__ __forceinline__ uint32_t window(const uint32_t* w, int off) {
   // bits [off, off+32) of the little-endian stream held in w[]
   if (off < 0) return w[0] << (-off);
   const int k = off >> 5, r = off & 31;
   if (r == 0) return w[k];
-  if (UB == 3 && k == 2) return w[2] >> r;
+  if (k + 1 >= group_words(BITS)) return w[k] >> r;
   return __funnelshift_r(w[k], w[k + 1], r);
 }
 
-// Pair register for lane pair j from the lane's words of one row.  `magic` is
-// 0x43004300 and lives in a register, so each pair costs one LOP3 with the
-// mask as its immediate operand (plus the shift of its window, shared by the
-// pairs that use the same window).
-template <int UB>
+// Pair register for lane pair j of one row's words: one LOP3 with the mask
+// as its immediate and `magic` in a register, plus the window's shift, which
+// the pairs sharing a window share.
+template <int BITS>
 __device__ __forceinline__ uint32_t make_pair(const uint32_t* words, int j, uint32_t magic) {
-  constexpr int GP = group_pairs(UB);
-  constexpr int GW = group_words(UB);
-  const PairDef d = pair_def(UB, j % GP);
+  constexpr int GP = group_pairs(BITS);
+  constexpr int GW = group_words(BITS);
+  constexpr uint32_t QM = (1u << BITS) - 1u;
+  const PairDef d = pair_def(BITS, j % GP);
   const uint32_t* g = words + (j / GP) * GW;
-  const uint32_t win = UB == 3 ? window<3>(g, d.win) : (d.win ? (g[0] >> d.win) : g[0]);
-  const uint32_t m = (((1u << UB) - 1u) << d.plo) | ((((1u << UB) - 1u) << d.phi) << 16);
-  return (win & m) | magic;
+  const uint32_t win = window<BITS>(g, d.win);
+  const uint32_t m = (QM << d.plo) | ((QM << d.phi) << 16);
+  return lop3_and_or(win, m, magic);
 }
 
 // Load the lane's words of tile row r from the stage's codes area (box h at
@@ -300,92 +406,83 @@ __device__ __forceinline__ void load_words(uint32_t* w, const uint8_t* codes, in
   }
 }
 
-// One MMA step of a b<16 block for this warp's 16 rows; adds the chunk
-// results into acc[row][batch].
-//
-// The lane's codes come in groups (one word for 2/4-bit, three words for
-// 3-bit); group q yields GP pairs = GP/2 MMAs.  Groups are visited in
-// increasing unit order, so the first group that starts past the block's last
-// code ends the step for the whole warp.
+// One step of a b<16 block for this warp's 16 rows; adds the chunk results,
+// scaled, into acc[row][batch].
 template <int NB, int BITS>
 __device__ __forceinline__ void step_mma(const GvParams& P, const GvBlock& B, int j,
-                                         const uint8_t* stage, const uint32_t* zero16,
-                                         int warp, int lane, float (&acc)[2][NB]) {
-  constexpr int UB = ubits(BITS);
-  constexpr int NG = ng_of(NB);
+                                         const uint8_t* stage, const uint32_t* rec,
+                                         const uint32_t* zeros, int warp, int lane,
+                                         float (&acc)[2][NB]) {
+  constexpr int U = step_units(BITS, NB);
+  constexpr int NGS = step_chunks(BITS, NB);
+  constexpr int NGM = 8 / NB;
   constexpr int NW = lane_words(BITS, NB);
   constexpr int LW = rec_lane_words(NB);
-  constexpr int GP = group_pairs(UB), GU = group_units(UB), GW = group_words(UB);
-  constexpr int NGRP = NW / GW;
-  constexpr int NACC = 8;
+  constexpr int PW = rec_pair_words(NB);
+  constexpr int GP = group_pairs(BITS), GW = group_words(BITS);
+  constexpr int NBX = nbox_of(BITS, NB);
+  constexpr int GPB = NW / GW / NBX;      // groups per box
+  constexpr int CPB = U / NBX / 64;       // chunks per box
+  static_assert(GP % 4 == 0 && GPB * GW * NBX == NW, "step geometry");
   const int g = lane >> 2, t = lane & 3;
   const int rA = warp * 16 + g, rB = rA + 8;
   const uint32_t* meta_s = reinterpret_cast<const uint32_t*>(stage + kCodesBytes);
-  const uint32_t* rec = reinterpret_cast<const uint32_t*>(stage + kCodesBytes + kMetaBytes);
-
   const uint32_t magic = P.magic;
+
   uint32_t wa[NW], wb[NW];
   load_words<BITS, NB>(wa, stage, rA, t);
   load_words<BITS, NB>(wb, stage, rB, t);
 
-  // This lane holds column n = g of the B fragment for lane t's k-slots; the
-  // column is non-zero only for the chunk (and batch) that the group of lane t
-  // belongs to.  The chunk of group q is the lane's first chunk + a constant.
-  const int my_b = g / NG, my_c = g % NG;
-  const uint32_t* brow = rec + (my_b * 4 + t) * LW;
+  // Column g of the B fragment is (batch my_b, chunk my_c); lane t's codes in
+  // box h belong to chunk c_t + h*CPB, so only a matching lane loads its
+  // activations, the others read zeros.
+  const int my_b = g / NGS, my_c = g % NGS;
   const int dc = my_b < P.batch ? my_c - lane_unit(BITS, NB, t, 0) / 64 : -1000;
+  const uint32_t* brow = rec + (my_b * 4 + t) * LW;
+  const int uvalid = min(U, B.n_ch - j * U);
 
-  const int per_step = units_of(NB);
-  const int u_valid = min(per_step, (B.n_ch - j * (BITS == 8 ? per_step / 2 : per_step)) *
-                                        (BITS == 8 ? 2 : 1));
-  float d[NACC][4];
+  float d[4][4];
 #pragma unroll
-  for (int q = 0; q < NACC; ++q) d[q][0] = d[q][1] = d[q][2] = d[q][3] = 0.f;
-
+  for (int q = 0; q < 4; ++q) d[q][0] = d[q][1] = d[q][2] = d[q][3] = 0.f;
 #pragma unroll
-  for (int q = 0; q < NGRP; ++q) {
-    if (lane_unit(BITS, NB, 0, q * GU) >= u_valid) break;
-    const int coff = lane_unit(BITS, NB, 0, q * GU) / 64 - lane_unit(BITS, NB, 0, 0) / 64;
-    const uint32_t* bsrc = dc == coff ? brow + q * GP : zero16;
-    const int bstep = dc == coff ? 4 : 0;
+  for (int h = 0; h < NBX; ++h) {
+    if (h == 1 && uvalid <= U / 2) break;  // the second half of the step is empty
+    const uint32_t* bsrc = dc == h * CPB ? brow + h * GPB * GP : zeros;
 #pragma unroll
-    for (int m2 = 0; m2 < GP / 4; ++m2) {  // two MMAs per 16-byte activation load
-      const uint4 bv = *reinterpret_cast<const uint4*>(bsrc + m2 * bstep);
+    for (int qq = 0; qq < GPB; ++qq) {
+      const int q = h * GPB + qq;
 #pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        const int jp = q * GP + 4 * m2 + 2 * h;  // lane pair index
-        const uint32_t a0 = make_pair<UB>(wa, jp, magic);
-        const uint32_t a1 = make_pair<UB>(wb, jp, magic);
-        const uint32_t a2 = make_pair<UB>(wa, jp + 1, magic);
-        const uint32_t a3 = make_pair<UB>(wb, jp + 1, magic);
-        mma_bf16_16816(d[(jp / 2) % NACC], a0, a1, a2, a3, h ? bv.z : bv.x, h ? bv.w : bv.y);
+      for (int m2 = 0; m2 < GP / 4; ++m2) {  // two MMAs per 16-byte activation load
+        const uint4 bv = *reinterpret_cast<const uint4*>(bsrc + qq * GP + 4 * m2);
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+          const int jp = q * GP + 4 * m2 + 2 * hh;  // lane pair index
+          const uint32_t a0 = make_pair<BITS>(wa, jp, magic);
+          const uint32_t a1 = make_pair<BITS>(wb, jp, magic);
+          const uint32_t a2 = make_pair<BITS>(wa, jp + 1, magic);
+          const uint32_t a3 = make_pair<BITS>(wb, jp + 1, magic);
+          mma_f16_16816(d[(jp / 2) & 3], a0, a1, a2, a3, hh ? bv.z : bv.x, hh ? bv.w : bv.y);
+        }
       }
     }
   }
   float D[4];
 #pragma unroll
-  for (int v = 0; v < 4; ++v)
-    D[v] = ((d[0][v] + d[1][v]) + (d[2][v] + d[3][v])) +
-           ((d[4][v] + d[5][v]) + (d[6][v] + d[7][v]));
+  for (int v = 0; v < 4; ++v) D[v] = (d[0][v] + d[1][v]) + (d[2][v] + d[3][v]);
 
-  // epilogue: columns 2t, 2t+1 -> batch be, chunks c0, c0+1
-  const int be = (2 * t) / NG;
-  if (be < P.batch) {
-    const int c0 = (2 * t) % NG;
-    constexpr bool nib = BITS == 8;
-    const int gfirst = B.grp_off + (nib ? (j * NG) / 2 : j * NG);
-    const int x0 = gfirst & ~3;
-    const float* recf = reinterpret_cast<const float*>(rec);
-    constexpr int PW = rec_pair_words(NB);
+  // epilogue: columns 2t, 2t+1 -> (batch, chunk) (col / NGS, col % NGS)
+  const int g0 = (B.grp_off + j * NGS) & 3;  // first group of the step in the meta box
+  const float* recf = reinterpret_cast<const float*>(rec);
 #pragma unroll
-    for (int cc = 0; cc < 2; ++cc) {
-      const int c = c0 + cc;
-      const int gi = B.grp_off + (nib ? (j * NG + c) / 2 : j * NG + c);
-      const float C1 = recf[PW + be * NG + c];
-      const float X = recf[PW + NB * NG + be * NG + c];
+  for (int cc = 0; cc < 2; ++cc) {
+    const int col = 2 * t + cc;
+    const int be = col / NGS, c = col % NGS;
+    if (be < P.batch) {
+      const float C1 = recf[PW + be * NGM + c];
+      const float X = recf[PW + NB * NGM + be * NGM + c];
 #pragma unroll
       for (int r = 0; r < 2; ++r) {
-        const uint32_t m = meta_s[(r ? rB : rA) * kMetaBox + (gi - x0)];
+        const uint32_t m = meta_s[(r ? rB : rA) * kMetaBox + g0 + c];
         const float sc = __half2float(__ushort_as_half((uint16_t)(m & 0xFFFFu)));
         const float ze = __half2float(__ushort_as_half((uint16_t)(m >> 16)));
         const float v = sc * fmaf(-ze, X, D[2 * r + cc] - C1);
@@ -397,70 +494,113 @@ __device__ __forceinline__ void step_mma(const GvParams& P, const GvBlock& B, in
   }
 }
 
-// One 16-bit step (fp16 weights, CUDA-core FMAs).  Lane t holds weights
-// [16t, 16t+16) of each 64-weight half; the second half is skipped when the
-// block ends in the first.
+// One 16-bit step: the fp16 weights are the MMA's A operand as stored; column
+// n of B is batch row n.  Lane t holds weights [16t, 16t+16) of each of the
+// two 64-weight boxes.
 template <int NB>
 __device__ __forceinline__ void step_16(const GvParams& P, const GvBlock& B, int j,
-                                        const uint8_t* stage, int warp, int lane,
+                                        const uint8_t* stage, const uint32_t* rec,
+                                        const uint32_t* zeros, int warp, int lane,
                                         float (&acc)[2][NB]) {
   constexpr int LW = rec_lane_words(NB);
-  constexpr int PITCH = box_pitch(16, NB);
+  constexpr int PITCH = kPitchSplit;
+  static_assert(box_pitch(16, NB) == PITCH && nbox_of(16, NB) == 2, "16-bit geometry");
   const int g = lane >> 2, t = lane & 3;
   const int rA = warp * 16 + g, rB = rA + 8;
-  const uint32_t* rec = reinterpret_cast<const uint32_t*>(stage + kCodesBytes + kMetaBytes);
-  const int halves_used = (B.n_ch - j * kU16) > 64 ? 2 : 1;
+  const int uvalid = min(128, B.n_ch - j * 128);
+  const uint32_t* bsrc = g < P.batch ? rec + (g * 4 + t) * LW : zeros;
+  float d[2][4];
+#pragma unroll
+  for (int q = 0; q < 2; ++q) d[q][0] = d[q][1] = d[q][2] = d[q][3] = 0.f;
 #pragma unroll
   for (int h = 0; h < 2; ++h) {
-    if (h >= halves_used) break;
-    uint32_t wa[8], wb[8];
-    {
-      const uint4* pa = reinterpret_cast<const uint4*>(stage + h * kRows * PITCH + rA * PITCH + 32 * t);
-      const uint4* pb = reinterpret_cast<const uint4*>(stage + h * kRows * PITCH + rB * PITCH + 32 * t);
-      const uint4 a0 = pa[0], a1 = pa[1], b0 = pb[0], b1 = pb[1];
-      wa[0] = a0.x; wa[1] = a0.y; wa[2] = a0.z; wa[3] = a0.w;
-      wa[4] = a1.x; wa[5] = a1.y; wa[6] = a1.z; wa[7] = a1.w;
-      wb[0] = b0.x; wb[1] = b0.y; wb[2] = b0.z; wb[3] = b0.w;
-      wb[4] = b1.x; wb[5] = b1.y; wb[6] = b1.z; wb[7] = b1.w;
-    }
+    if (h == 1 && uvalid <= 64) break;
+    const uint4* pa = reinterpret_cast<const uint4*>(stage + h * kRows * PITCH + rA * PITCH + 32 * t);
+    const uint4* pb = reinterpret_cast<const uint4*>(stage + h * kRows * PITCH + rB * PITCH + 32 * t);
+    const uint4 a0 = pa[0], a1 = pa[1], b0 = pb[0], b1 = pb[1];
+    const uint32_t wa[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+    const uint32_t wb[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
 #pragma unroll
-    for (int b = 0; b < NB; ++b) {
-      if (b >= P.batch) break;
-      const uint32_t* xr = rec + (b * 4 + t) * LW + 8 * h;
-      float sa = 0.f, sb = 0.f;
+    for (int m2 = 0; m2 < 2; ++m2) {
+      const uint4 bv = *reinterpret_cast<const uint4*>(bsrc + 8 * h + 4 * m2);
 #pragma unroll
-      for (int k2 = 0; k2 < 2; ++k2) {
-        const uint4 xv = reinterpret_cast<const uint4*>(xr)[k2];
-        const uint32_t xw[4] = {xv.x, xv.y, xv.z, xv.w};
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          const int k = 4 * k2 + q;
-          const float x0 = bf16_lo(xw[q]), x1 = bf16_hi(xw[q]);
-          const float2 fa = __half22float2(*reinterpret_cast<const __half2*>(&wa[k]));
-          const float2 fb = __half22float2(*reinterpret_cast<const __half2*>(&wb[k]));
-          sa = fmaf(fa.x, x0, sa);
-          sa = fmaf(fa.y, x1, sa);
-          sb = fmaf(fb.x, x0, sb);
-          sb = fmaf(fb.y, x1, sb);
-        }
+      for (int hh = 0; hh < 2; ++hh) {
+        const int k = 4 * m2 + 2 * hh;
+        mma_f16_16816(d[hh], wa[k], wb[k], wa[k + 1], wb[k + 1], hh ? bv.z : bv.x,
+                      hh ? bv.w : bv.y);
       }
-      acc[0][b] += sa;
-      acc[1][b] += sb;
+    }
+  }
+#pragma unroll
+  for (int cc = 0; cc < 2; ++cc) {
+    const int be = 2 * t + cc;
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+      const float v = d[0][2 * r + cc] + d[1][2 * r + cc];
+#pragma unroll
+      for (int b = 0; b < NB; ++b)
+        if (b == be) acc[r][b] += v;
     }
   }
 }
 
+__device__ __forceinline__ uint32_t ld_acquire_u32(const uint32_t* p) {
+  uint32_t v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ unsigned long long global_ns() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+__device__ __forceinline__ void fence_proxy_async_global() {
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+
+// ---------------------------------------------------------------------------
+// pre-pass: one CTA of 128 threads per activation record (layer, step)
+// ---------------------------------------------------------------------------
 template <int NB>
-__global__ void __launch_bounds__(160, 3) gemv_main(const __grid_constant__ GvParams P) {
-  extern __shared__ __align__(128) uint8_t smem[];
-  uint8_t* stages = smem;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kStages * kStageBytes);
-  uint32_t* zero16 = reinterpret_cast<uint32_t*>(bars + 2 * kStages);
+__global__ void __launch_bounds__(kConsumers) gemv_prep(const __grid_constant__ GvParams P) {
+  pdl_trigger();  // the main kernel may start streaming weights right away
   __shared__ GvShared S;
+  __shared__ uint32_t s_p3[16];  // 3-bit pair schedule
+  load_shared(P, &S);
+  if (threadIdx.x < 16) {
+    const PairDef d = pair3(threadIdx.x);
+    s_p3[threadIdx.x] = (uint32_t)d.lo | ((uint32_t)d.hi << 8) | ((uint32_t)(d.win + 16) << 16);
+  }
+  __syncthreads();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int r = blockIdx.x;
+  int l, bi, j;
+  rec_pos(S, P.n_layers, r, &l, &bi, &j);
+  int src[2][2];
+  rec_sources<NB>(P, S.blk[l][bi], l, j, warp, lane, s_p3, src);  // static layer data
+  pdl_wait();  // x comes from the previous kernel; the records may still be in use
+  rec_build<NB>(P, S.blk[l][bi], l, j, warp, lane, s_p3, src,
+                reinterpret_cast<uint32_t*>(P.rec + (size_t)r * rec_bytes(NB)));
+}
+
+template <int NB>
+__global__ void __launch_bounds__(kThreads, kCtasPerSm) gemv_main(const __grid_constant__ GvParams P) {
+  extern __shared__ __align__(128) uint8_t smem[];
+  constexpr int RB = rec_bytes(NB);
+  uint8_t* stages = smem;
+  uint32_t* zeros = reinterpret_cast<uint32_t*>(smem + kStages * kStageBytes);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(zeros + 64);
+  __shared__ GvShared S;
+  // Set once any wait of this CTA gives up: later waits are skipped so that
+  // every warp still reaches the consumer barriers and the kernel ends.
+  __shared__ volatile int s_abort;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t full0 = smem_u32(bars), empty0 = smem_u32(bars + kStages);
 
   load_shared(P, &S);
+  if (threadIdx.x == 0) s_abort = 0;
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(full0 + 8 * s, 1);
@@ -468,7 +608,7 @@ __global__ void __launch_bounds__(160, 3) gemv_main(const __grid_constant__ GvPa
     }
     mbar_fence_init();
   }
-  if (threadIdx.x < 4) zero16[threadIdx.x] = 0u;
+  if (threadIdx.x < 64) zeros[threadIdx.x] = 0u;
   __syncthreads();
   pdl_trigger();
   const int nl = P.n_layers;
@@ -478,26 +618,17 @@ __global__ void __launch_bounds__(160, 3) gemv_main(const __grid_constant__ GvPa
   const int lo = (int)((long long)blockIdx.x * I / C);
   const int hi = (int)((long long)(blockIdx.x + 1) * I / C);
   const int n_mine = hi - lo;
-  constexpr int RB = rec_bytes(NB);
 
   if (warp == kWarps) {
     // ---------------- producer ----------------
-    if (lane != 0) return;
-    for (int l = 0; l < nl; ++l) {
-      for (int b = 0; b < S.n_blocks[l]; ++b) prefetch_tmap(&P.L[l].tm_codes[b]);
-      prefetch_tmap(&P.L[l].tm_meta);
-    }
-    auto issue_weights = [&](int k, int slot) {
-      const int item = lo + k;
-      const int l = find_layer(S.item0, nl, item);
-      const int li = item - S.item0[l];
-      const int steps = S.steps[l];
-      const int tile = li / steps, s = li - tile * steps;
-      const int bi = find_block(S.blk[l], S.n_blocks[l], s);
-      const GvBlock& B = S.blk[l][bi];
-      const int j = s - B.step0;
-      const uint32_t dst = smem_u32(stages + slot * kStageBytes);
-      const uint32_t bar = full0 + 8 * slot;
+    // The packed weights do not depend on earlier kernels: request the first
+    // stages before the grid-dependency wait.  The activation records come
+    // from this call's builders and are loaded once they are flagged ready.
+    ItemPos it;
+    it.init(S, nl, lo);
+    auto issue_weights = [&](int k, const ItemPos& q) {
+      const int slot = k % kStages;
+      const GvBlock& B = S.blk[q.l][q.bi];
       int sb, nbx, pitch;
       switch (B.bits) {
         case 2: sb = step_bytes(2, NB); nbx = nbox_of(2, NB); pitch = box_pitch(2, NB); break;
@@ -506,104 +637,177 @@ __global__ void __launch_bounds__(160, 3) gemv_main(const __grid_constant__ GvPa
         case 8: sb = step_bytes(8, NB); nbx = nbox_of(8, NB); pitch = box_pitch(8, NB); break;
         default: sb = step_bytes(16, NB); nbx = nbox_of(16, NB); pitch = box_pitch(16, NB); break;
       }
+      const uint32_t dst = smem_u32(stages + slot * kStageBytes);
+      const uint32_t bar = full0 + 8 * slot;
       uint32_t bytes = nbx * pitch * kRows + RB;
       if (B.bits < 16) bytes += kMetaBytes;
       mbar_expect_tx(bar, bytes);
-      const CUtensorMap* tm = &P.L[l].tm_codes[bi];
-      for (int q = 0; q < nbx; ++q)
-        tma_load_2d(dst + q * kRows * pitch, tm, B.seg_off + j * sb + q * (sb / nbx), tile * kRows,
-                    bar);
+      const CUtensorMap* tm = &P.L[q.l].tm_codes[q.bi];
+      for (int h = 0; h < nbx; ++h)
+        tma_load_2d(dst + h * kRows * pitch, tm, B.seg_off + q.j * sb + h * (sb / nbx),
+                    q.tile * kRows, bar);
       if (B.bits < 16) {
-        const int ngs = B.bits == 8 ? ng_of(NB) / 2 : ng_of(NB);
-        const int x0 = (B.grp_off + j * ngs) & ~3;
-        tma_load_2d(dst + kCodesBytes, &P.L[l].tm_meta, x0, tile * kRows, bar);
+        const int x0 = (B.grp_off + q.j * (B.units / 64)) & ~3;
+        tma_load_2d(dst + kCodesBytes, &P.L[q.l].tm_meta, x0, q.tile * kRows, bar);
       }
-    };
-    auto issue_rec = [&](int k, int slot) {
-      const int item = lo + k;
-      const int l = find_layer(S.item0, nl, item);
-      const int s = (item - S.item0[l]) % S.steps[l];
-      const uint32_t dst = smem_u32(stages + slot * kStageBytes + kCodesBytes + kMetaBytes);
-      bulk_load(dst, P.rec + (size_t)(S.rec0[l] + s) * RB, RB, full0 + 8 * slot);
     };
     const int pre = min(n_mine, kStages);
-    for (int k = 0; k < pre; ++k) issue_weights(k, k);
-    pdl_wait();  // activation records come from the pre-pass
-    for (int k = 0; k < pre; ++k) issue_rec(k, k);
-    for (int k = kStages; k < n_mine; ++k) {
-      const int slot = k % kStages;
-      const uint32_t par = ((k / kStages) - 1) & 1;
-      if (!mbar_wait(empty0 + 8 * slot, par)) {
-        atomicExch(P.status, kStatusTimeoutEmpty);
-        break;
+    if (lane == 0) {
+      for (int l = 0; l < nl; ++l) {
+        for (int b = 0; b < S.n_blocks[l]; ++b) prefetch_tmap(&P.L[l].tm_codes[b]);
+        prefetch_tmap(&P.L[l].tm_meta);
       }
-      issue_weights(k, slot);
-      issue_rec(k, slot);
+      ItemPos q = it;
+      for (int k = 0; k < pre; ++k) {
+        issue_weights(k, q);
+        q.next(S, nl);
+      }
+    }
+    pdl_wait();  // the records come from the pre-pass of this call
+    fence_proxy_async_global();  // it wrote them through the generic proxy
+    if (lane != 0) return;
+    for (int k = 0; k < n_mine; ++k) {
+      const int slot = k % kStages;
+      if (s_abort) break;
+      if (k >= kStages) {
+        if (!mbar_wait(empty0 + 8 * slot, ((k / kStages) - 1) & 1)) {
+          atomicExch(P.status, kStatusTimeoutEmpty);
+          s_abort = 1;
+          break;
+        }
+        issue_weights(k, it);
+      }
+      const int r = S.rec0[it.l] + it.s;
+      bulk_load(smem_u32(stages + slot * kStageBytes + kCodesBytes + kMetaBytes),
+                P.rec + (size_t)r * RB, RB, full0 + 8 * slot);
+      it.next(S, nl);
     }
     return;
   }
 
   // ---------------- consumers ----------------
-  pdl_wait();
   const int g = lane >> 2, t = lane & 3;
+  const int tid = threadIdx.x;
+  pdl_wait();  // y, the workspace and the records are this call's from here on
   float acc[2][NB];
 #pragma unroll
   for (int r = 0; r < 2; ++r)
 #pragma unroll
     for (int b = 0; b < NB; ++b) acc[r][b] = 0.f;
+  ItemPos it;
+  it.init(S, nl, lo);
   for (int k = 0; k < n_mine; ++k) {
     const int slot = k % kStages;
-    const uint32_t par = (k / kStages) & 1;
-    if (!mbar_wait(full0 + 8 * slot, par)) {
-      if (lane == 0) atomicExch(P.status, kStatusTimeoutFull);
-      return;
+    if (s_abort || !mbar_wait(full0 + 8 * slot, (k / kStages) & 1)) {
+      if (lane == 0 && !s_abort) atomicExch(P.status, kStatusTimeoutFull);
+      s_abort = 1;
+      it.next(S, nl);
+      continue;
     }
-    const int item = lo + k;
-    const int l = find_layer(S.item0, nl, item);
-    const int li = item - S.item0[l];
-    const int steps = S.steps[l];
-    const int tile = li / steps, s = li - tile * steps;
-    const int bi = find_block(S.blk[l], S.n_blocks[l], s);
-    const GvBlock B = S.blk[l][bi];
-    const int j = s - B.step0;
+    const GvBlock B = S.blk[it.l][it.bi];
     const uint8_t* stage = stages + slot * kStageBytes;
+    const uint32_t* rec = reinterpret_cast<const uint32_t*>(stage + kCodesBytes + kMetaBytes);
     switch (B.bits) {
-      case 2: step_mma<NB, 2>(P, B, j, stage, zero16, warp, lane, acc); break;
-      case 3: step_mma<NB, 3>(P, B, j, stage, zero16, warp, lane, acc); break;
-      case 4: step_mma<NB, 4>(P, B, j, stage, zero16, warp, lane, acc); break;
-      case 8: step_mma<NB, 8>(P, B, j, stage, zero16, warp, lane, acc); break;
-      default: step_16<NB>(P, B, j, stage, warp, lane, acc); break;
+      case 2: step_mma<NB, 2>(P, B, it.j, stage, rec, zeros, warp, lane, acc); break;
+      case 3: step_mma<NB, 3>(P, B, it.j, stage, rec, zeros, warp, lane, acc); break;
+      case 4: step_mma<NB, 4>(P, B, it.j, stage, rec, zeros, warp, lane, acc); break;
+      case 8: step_mma<NB, 8>(P, B, it.j, stage, rec, zeros, warp, lane, acc); break;
+      default: step_16<NB>(P, B, it.j, stage, rec, zeros, warp, lane, acc); break;
     }
     __syncwarp();
     if (lane == 0) mbar_arrive(empty0 + 8 * slot);
-    if (s != steps - 1 && k != n_mine - 1) continue;
 
-    // ---- flush this warp's 16 rows of `tile` of layer l ----
-    // Sum the four lanes of each row, then add the piece into y.  A tile whose
-    // steps are split over CTAs receives one addition per piece.
+    if (it.tile_end(S) || k == n_mine - 1) {
+      // ---- finish this warp's 16 rows of the tile piece ----
 #pragma unroll
-    for (int r = 0; r < 2; ++r)
+      for (int r = 0; r < 2; ++r)
 #pragma unroll
-      for (int b = 0; b < NB; ++b) {
-        float v = acc[r][b];
-        v += __shfl_xor_sync(0xffffffffu, v, 1);
-        v += __shfl_xor_sync(0xffffffffu, v, 2);
-        acc[r][b] = v;
+        for (int b = 0; b < NB; ++b) {
+          float v = acc[r][b];
+          v += __shfl_xor_sync(0xffffffffu, v, 1);
+          v += __shfl_xor_sync(0xffffffffu, v, 2);
+          acc[r][b] = v;
+        }
+      const int l = it.l;
+      const int steps = S.steps[l];
+      const int T0 = S.item0[l] + it.tile * steps;  // first item of the tile
+      const int T1 = T0 + steps - 1;
+      const int N = S.N[l];
+      uint32_t* cnt = P.cnt + (size_t)(S.tile0[l] + it.tile) * kWarps + warp;
+      // lane t finishes batch row t of rows g and g+8
+      float mine[2];
+#pragma unroll
+      for (int r = 0; r < 2; ++r) {
+        mine[r] = 0.f;
+#pragma unroll
+        for (int b = 0; b < NB; ++b)
+          if (b == t) mine[r] = acc[r][b];
       }
-    float* y = nullptr;
+      const bool active = t < P.batch;
+      if (T0 < lo) {
+        // not the owner: leave this piece for the CTA holding the tile's
+        // first step
+        if (active) {
 #pragma unroll
-    for (int q = 0; q < POLYQ_MAX_GROUP; ++q)
-      if (q == l) y = P.L[q].y;
-    const int N = S.N[l];
+          for (int r = 0; r < 2; ++r)
+            P.part[((size_t)blockIdx.x * kRows + warp * 16 + g + 8 * r) * NB + t] = mine[r];
+        }
+        __threadfence();
+        __syncwarp();
+        if (lane == 0) atomicAdd(cnt, 1u);
+      } else {
+        int c_last = blockIdx.x;
+        if (T1 >= hi) {
+          // the other pieces sit at the start of CTAs blockIdx.x+1 .. c_last
+          c_last = (int)(((long long)(T1 + 1) * C - 1) / I);
+          const uint32_t need = (uint32_t)(c_last - (int)blockIdx.x);
+          if (lane == 0 && !s_abort) {
+            const unsigned long long t_start = global_ns();
+            while (ld_acquire_u32(cnt) < need) {
+              __nanosleep(64);
+              if (global_ns() - t_start > kFixupWaitNs) {
+                atomicExch(P.status, kStatusFixupTimeout);
+                break;
+              }
+            }
+          }
+          __syncwarp();
+          __threadfence();
+        }
+        float* y = P.L[0].y;
+        const float* res = P.L[0].residual;
 #pragma unroll
-    for (int r = 0; r < 2; ++r)
+        for (int q = 1; q < POLYQ_MAX_GROUP; ++q)
+          if (q == l) {
+            y = P.L[q].y;
+            res = P.L[q].residual;
+          }
 #pragma unroll
-      for (int b = 0; b < NB; ++b) {
-        const int n = tile * kRows + warp * 16 + g + 8 * r;
-        if (b == t && b < P.batch && n < N) atomicAdd(y + (size_t)b * N + n, acc[r][b]);
-        acc[r][b] = 0.f;
+        for (int r = 0; r < 2; ++r) {
+          const int row = warp * 16 + g + 8 * r;
+          const int n = it.tile * kRows + row;
+          float v = mine[r];
+          if (active)
+            for (int c = (int)blockIdx.x + 1; c <= c_last; ++c)
+              v += __ldcg(P.part + ((size_t)c * kRows + row) * NB + t);
+          if (active && n < N) {
+            const size_t o = (size_t)t * N + n;
+            y[o] = (res ? res[o] : 0.f) + v;
+          }
+        }
+        if (c_last != (int)blockIdx.x) {
+          __syncwarp();
+          if (lane == 0) *cnt = 0u;
+        }
       }
+#pragma unroll
+      for (int r = 0; r < 2; ++r)
+#pragma unroll
+        for (int b = 0; b < NB; ++b) acc[r][b] = 0.f;
+    }
+    it.next(S, nl);
   }
+
 }
 
 // ---------------------------------------------------------------------------
@@ -621,21 +825,64 @@ int steps_of(const polyq_dev_layer* L, int nb, GvBlock* blk) {
     g.pos0 = b.pos0;
     g.seg_off = b.seg_off;
     g.grp_off = b.grp_off;
-    g.n_grp = b.n_grp;
+    g.units = step_units(b.bits, nb);
     g.step0 = s;
-    const int per = b.bits == 16 ? kU16 : (b.bits == 8 ? units_of(nb) / 2 : units_of(nb));
-    g.n_steps = (b.n_ch + per - 1) / per;
+    g.n_steps = (b.n_ch + g.units - 1) / g.units;
     s += g.n_steps;
     if (blk) blk[i] = g;
   }
   return s;
 }
 
-size_t workspace_for(const polyq_dev_layer* const* L, int n, int batch) {
+// CTAs of one launch: all of them must be resident at once (an owner waits
+// for pieces of later CTAs), so never more than the device holds.
+int grid_for(int items, int* grid) {
+  int sms = 0;
+  int rc = polyq_sm_count(&sms);
+  if (rc) return rc;
+  *grid = std::max(1, std::min(std::min(items, kCtasPerSm * sms), kMaxGrid));
+  return POLYQ_OK;
+}
+
+// Workspace.  The tile counters sit at a fixed offset with a fixed capacity,
+// so that calls of different shapes can share one workspace without one
+// call's data landing on another's counters:
+//   [0, 256)               status word
+//   [256, +16*kMaxTiles)   tile piece counters (zero between calls)
+// then this call's activation records and piece sums.
+constexpr int kMaxRecs = 4096;
+constexpr int kMaxTiles = 8192;
+struct WsLayout {
+  size_t cnt_off, rec_off, part_off, bytes;
+  int grid, tiles, items, recs;
+};
+
+int workspace_layout(const polyq_dev_layer* const* L, int n, int batch, WsLayout* w) {
   const int nb = nb_of(batch);
-  size_t recs = 0;
-  for (int i = 0; i < n; ++i) recs += (size_t)steps_of(L[i], nb, nullptr);
-  return (recs * rec_bytes(nb) + 255) / 256 * 256 + 256;  // records + status word
+  long long items = 0, tiles = 0, recs = 0;
+  for (int i = 0; i < n; ++i) {
+    const long long t = (L[i]->N + kRows - 1) / kRows;
+    const long long st = steps_of(L[i], nb, nullptr);
+    tiles += t;
+    items += t * st;
+    recs += st;
+  }
+  if (items > (1ll << 30) || tiles > kMaxTiles || recs > kMaxRecs)
+    return polyq_set_error(POLYQ_EUNSUPPORTED,
+                           "polyq gemv: a call covers at most %d row tiles of 64 and %d steps "
+                           "(got %lld and %lld)",
+                           kMaxTiles, kMaxRecs, tiles, recs);
+  w->items = (int)items;
+  w->tiles = (int)tiles;
+  w->recs = (int)recs;
+  int rc = grid_for(w->items, &w->grid);
+  if (rc) return rc;
+  auto up = [](size_t v) { return (v + 255) / 256 * 256; };
+  w->cnt_off = 256;
+  w->rec_off = w->cnt_off + (size_t)kMaxTiles * kWarps * 4;
+  w->part_off = w->rec_off + up((size_t)recs * rec_bytes(nb));
+  w->bytes = w->part_off + (size_t)w->grid * kRows * nb * 4;
+  return POLYQ_OK;
 }
 
 int check_group(const char* who, const polyq_dev_layer* const* L, int n, int batch) {
@@ -650,40 +897,41 @@ int check_group(const char* who, const polyq_dev_layer* const* L, int n, int bat
   return POLYQ_OK;
 }
 
+constexpr size_t kSmemBytes = (size_t)kStages * kStageBytes + 64 * 4 + 2 * kStages * 8;
+
 template <int NB>
-int launch(const GvParams& P, int recs, cudaStream_t st) {
-  static bool attr_done[8] = {false};
+int launch(const GvParams& P, int grid, cudaStream_t st) {
+  static bool attr_done[64] = {false};
   int dev = 0;
   cudaGetDevice(&dev);
-  const size_t smem = (size_t)kStages * kStageBytes + 2 * kStages * 8 + 16;
-  if (!attr_done[dev & 7]) {
+  if (!attr_done[dev & 63]) {
     cudaError_t e = cudaFuncSetAttribute(gemv_main<NB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)smem);
+                                         (int)kSmemBytes);
     if (e != cudaSuccess)
       return polyq_set_error(POLYQ_ECUDA, "polyq gemv: smem attribute: %s", cudaGetErrorString(e));
-    attr_done[dev & 7] = true;
+    int per_sm = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, gemv_main<NB>, kThreads, kSmemBytes);
+    if (e != cudaSuccess || per_sm < kCtasPerSm)
+      return polyq_set_error(POLYQ_ECUDA, "polyq gemv: %d CTAs per SM fit, %d needed (%s)", per_sm,
+                             kCtasPerSm, cudaGetErrorString(e));
+    attr_done[dev & 63] = true;
   }
-  int sms = 0;
-  int rc = polyq_sm_count(&sms);
-  if (rc) return rc;
   cudaLaunchAttribute at[1];
   at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   at[0].val.programmaticStreamSerializationAllowed = 1;
-
   cudaLaunchConfig_t cfg = {};
   cfg.stream = st;
   cfg.attrs = at;
   cfg.numAttrs = 1;
-  cfg.gridDim = dim3((unsigned)std::max(recs, 1));
-  cfg.blockDim = dim3(256);
+  cfg.gridDim = dim3((unsigned)P.recs);
+  cfg.blockDim = dim3(kConsumers);
   cfg.dynamicSmemBytes = 0;
   cudaError_t e = cudaLaunchKernelEx(&cfg, gemv_prep<NB>, P);
   if (e != cudaSuccess)
-    return polyq_set_error(POLYQ_ECUDA, "polyq gemv: prep launch: %s", cudaGetErrorString(e));
-
-  cfg.gridDim = dim3((unsigned)std::min(std::min(P.items, kCtasPerSm * sms), kMaxGrid));
-  cfg.blockDim = dim3(32 * (kWarps + 1));
-  cfg.dynamicSmemBytes = smem;
+    return polyq_set_error(POLYQ_ECUDA, "polyq gemv: pre-pass launch: %s", cudaGetErrorString(e));
+  cfg.gridDim = dim3((unsigned)grid);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = kSmemBytes;
   e = cudaLaunchKernelEx(&cfg, gemv_main<NB>, P);
   if (e != cudaSuccess)
     return polyq_set_error(POLYQ_ECUDA, "polyq gemv: launch: %s", cudaGetErrorString(e));
@@ -698,16 +946,18 @@ int gemv_group(const char* who, const polyq_dev_layer* const* L, int n, const vo
   if (!xs || !ys) return polyq_set_error(POLYQ_EINVAL, "%s: x or y is NULL", who);
   for (int i = 0; i < n; ++i)
     if (!xs[i] || !ys[i]) return polyq_set_error(POLYQ_EINVAL, "%s: x or y %d is NULL", who, i);
-  const size_t need = workspace_for(L, n, batch);
-  if (!workspace || ws_bytes < need)
-    return polyq_set_error(POLYQ_ENOMEM, "%s: workspace needs %zu bytes, got %zu", who, need,
+  WsLayout w;
+  rc = workspace_layout(L, n, batch, &w);
+  if (rc) return rc;
+  if (!workspace || ws_bytes < w.bytes)
+    return polyq_set_error(POLYQ_ENOMEM, "%s: workspace needs %zu bytes, got %zu", who, w.bytes,
                            ws_bytes);
   if ((uintptr_t)workspace % 256)
     return polyq_set_error(POLYQ_EINVAL, "%s: workspace must be 256-byte aligned", who);
   const int nb = nb_of(batch);
   GvParams P;
   memset(&P, 0, sizeof P);
-  int items = 0, recs = 0;
+  int items = 0, tiles = 0, recs = 0;
   for (int i = 0; i < n; ++i) {
     GvLayer& G = P.L[i];
     const polyq_dev_layer* D = L[i];
@@ -727,27 +977,33 @@ int gemv_group(const char* who, const polyq_dev_layer* const* L, int n, const vo
     G.N = (int)D->N;
     G.K = (int)D->K;
     G.steps = steps;
-    G.items = (int)((D->N + kRows - 1) / kRows) * steps;
+    const int t = (int)((D->N + kRows - 1) / kRows);
+    G.items = t * steps;
     G.item0 = items;
+    G.tile0 = tiles;
     G.rec0 = recs;
     G.x = (const __nv_bfloat16*)xs[i];
     G.gather = D->gather;
     G.y = ys[i];
     G.residual = res ? res[i] : nullptr;
     items += G.items;
+    tiles += t;
     recs += steps;
   }
   P.n_layers = n;
   P.items = items;
   P.recs = recs;
   P.batch = batch;
-  P.magic = 0x43004300u;
-  P.rec = (uint8_t*)workspace;
-  P.status = (int*)((uint8_t*)workspace + need - 256);
+  P.magic = kMagic;
+  uint8_t* ws = (uint8_t*)workspace;
+  P.status = (int*)ws;
+  P.cnt = (uint32_t*)(ws + w.cnt_off);
+  P.rec = ws + w.rec_off;
+  P.part = (float*)(ws + w.part_off);
   switch (nb) {
-    case 1: return launch<1>(P, recs, st);
-    case 2: return launch<2>(P, recs, st);
-    default: return launch<4>(P, recs, st);
+    case 1: return launch<1>(P, w.grid, st);
+    case 2: return launch<2>(P, w.grid, st);
+    default: return launch<4>(P, w.grid, st);
   }
 }
 
@@ -759,7 +1015,10 @@ extern "C" int polyq_gemv_workspace_bytes(const polyq_dev_layer* L, int batch, s
   int rc = check_group("polyq_gemv_workspace_bytes", one, 1, batch);
   if (rc) return rc;
   if (!bytes) return polyq_set_error(POLYQ_EINVAL, "polyq_gemv_workspace_bytes: bytes is NULL");
-  *bytes = workspace_for(one, 1, batch);
+  WsLayout w;
+  rc = workspace_layout(one, 1, batch, &w);
+  if (rc) return rc;
+  *bytes = w.bytes;
   return POLYQ_OK;
 }
 
@@ -770,7 +1029,10 @@ extern "C" int polyq_gemv_group_workspace_bytes(const polyq_dev_layer* const* la
   if (rc) return rc;
   if (!bytes)
     return polyq_set_error(POLYQ_EINVAL, "polyq_gemv_group_workspace_bytes: bytes is NULL");
-  *bytes = workspace_for(layers, n, batch);
+  WsLayout w;
+  rc = workspace_layout(layers, n, batch, &w);
+  if (rc) return rc;
+  *bytes = w.bytes;
   return POLYQ_OK;
 }
 
@@ -801,10 +1063,10 @@ extern "C" int polyq_linear_gemv_group(const polyq_dev_layer* const* layers, int
 // Some callers cannot allocate device memory: a plugin inside a host program
 // whose own pool owns the device, or a latency-bound loop that cannot take the
 // device-wide synchronisation cudaMalloc/cudaFree may cause.  For them the
-// records and the status word live in this fixed array, one copy per device
-// that loads the library, kept until the process exits.  In host code the name
-// below stands for a host-side shadow, never the device address: the address
-// is looked up with cudaGetSymbolAddress, once per device.
+// status word, tile counters and piece sums live in this fixed array, one copy
+// per device that loads the library, kept until the process exits.  In host
+// code the name below stands for a host-side shadow, never the device address:
+// the address is looked up with cudaGetSymbolAddress, once per device.
 static __device__ __align__(256) uint8_t polyq_noalloc_scratch[POLYQ_NOALLOC_SCRATCH_BYTES];
 
 namespace {
@@ -847,17 +1109,24 @@ extern "C" int polyq_linear_gemv_noalloc(const polyq_dev_layer* L, const void* x
   const polyq_dev_layer* one[1] = {L};
   int rc = check_group(who, one, 1, batch);
   if (rc) return rc;
-  const size_t need = workspace_for(one, 1, batch);
-  if (need > POLYQ_NOALLOC_SCRATCH_BYTES)
+  WsLayout w;
+  rc = workspace_layout(one, 1, batch, &w);
+  if (rc) return rc;
+  if (w.bytes > POLYQ_NOALLOC_SCRATCH_BYTES)
     return polyq_set_error(POLYQ_ENOMEM,
                            "%s: this layer at batch %d needs %zu bytes of scratch, above the "
                            "fixed maximum of %u; call polyq_linear_gemv with a workspace",
-                           who, batch, need, (unsigned)POLYQ_NOALLOC_SCRATCH_BYTES);
+                           who, batch, w.bytes, (unsigned)POLYQ_NOALLOC_SCRATCH_BYTES);
   void* scratch = nullptr;
   rc = noalloc_scratch(&scratch);
   if (rc) return rc;
-  // gemv_prep writes every record the main kernel reads and zeroes the status
-  // word before anything reads it, so stale contents need no clearing here.
+  // The status word and the tile counters must start at zero.  Finished
+  // calls leave them so, but one that gave up on a wait may not, and this
+  // caller cannot reset the library's array itself: clear them on every call.
+  cudaError_t e = cudaMemsetAsync(scratch, 0, w.rec_off, (cudaStream_t)stream);
+  if (e != cudaSuccess)
+    return polyq_set_error(POLYQ_ECUDA, "%s: clearing the scratch counters: %s", who,
+                           cudaGetErrorString(e));
   const void* xs[1] = {x};
   float* ys[1] = {y};
   const float* rs[1] = {residual};

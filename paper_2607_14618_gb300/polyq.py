@@ -266,7 +266,8 @@ def linear_gemv(layer: DeviceLayer, x, y=None, residual=None, workspace=None, st
         y = torch.empty((batch, layer.N), dtype=torch.float32, device=x.device)
     ws_need = gemv_workspace_bytes(layer, batch)
     if workspace is None and ws_need:
-        workspace = torch.empty(ws_need, dtype=torch.uint8, device=x.device)
+        # the tile counters in the workspace start at zero; calls keep them so
+        workspace = torch.zeros(ws_need, dtype=torch.uint8, device=x.device)
     ws_ptr = workspace.data_ptr() if workspace is not None else None
     ws_len = workspace.numel() if workspace is not None else 0
     _check(_lib.polyq_linear_gemv(C.byref(layer.desc), x.data_ptr(), batch, y.data_ptr(),
@@ -328,7 +329,7 @@ def linear_gemv_group(layers, xs, ys=None, residuals=None, workspace=None, strea
         ys = [torch.empty((batch, l.N), dtype=torch.float32, device=xs[0].device) for l in layers]
     need = gemv_group_workspace_bytes(layers, batch)
     if workspace is None:
-        workspace = torch.empty(need, dtype=torch.uint8, device=xs[0].device)
+        workspace = torch.zeros(need, dtype=torch.uint8, device=xs[0].device)
     xa = (C.c_void_p * n)(*[x.data_ptr() for x in xs])
     ya = (C.c_void_p * n)(*[y.data_ptr() for y in ys])
     ra = None
@@ -375,6 +376,6 @@ def unpack_codes(layer: DeviceLayer, stream=None):
 
 
 def gemv_launches_per_call(layer: DeviceLayer, batch: int) -> int:
-    """Kernels one polyq_linear_gemv call enqueues (activation pre-pass and
-    the streaming kernel)."""
+    """Kernels one polyq_linear_gemv (or _group) call enqueues: the activation
+    record pre-pass and the streaming kernel."""
     return 2

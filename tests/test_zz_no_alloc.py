@@ -63,25 +63,41 @@ def test_noalloc_matches_workspace_entry_on_two_calls(polyq_lib):
     _same(y2b, ref2)
 
 
-def test_noalloc_rejects_layers_beyond_the_scratch(polyq_lib):
-    # all 8-bit at batch 4 needs 21 bytes per input channel: K = 65536 needs
-    # about 1.3 MiB, above the fixed 1 MiB
+def _wide_layer(polyq_lib):
+    # one 64-row tile (16 rows) of K = 65536 all-8-bit channels
     N, K = 16, 65536
-    W, a = synth.layer_weights(N, K, 73)
+    W, a = synth.layer_weights(N, K, 74)
     bits = np.full(K, 8, dtype=np.uint8)
     dev = polyq_lib.DeviceLayer(polyq_lib.HostLayer.pack(W, a, 8.0, forced_bits=bits), "cuda")
+    return dev, a
+
+
+def test_noalloc_rejects_layers_beyond_the_scratch(polyq_lib):
+    # At batch 4 a step covers 128 channels, so this layer has 512 steps whose
+    # activation records (1344 bytes each) do not fit the fixed 1 MiB.
+    dev, a = _wide_layer(polyq_lib)
     assert polyq_lib.gemv_workspace_bytes(dev, 4) > polyq_lib.NOALLOC_SCRATCH_BYTES
-    xb, _ = synth.activations(a, 4, 73)
-    y = torch.zeros(4, N, device="cuda")
+    xb, _ = synth.activations(a, 4, 74)
+    y = torch.full((4, dev.N), 7.0, device="cuda")
     with pytest.raises(polyq_lib.PolyqError) as e:
         polyq_lib.linear_gemv_noalloc(dev, _x_dev(xb), y)
     assert e.value.code == polyq_lib.POLYQ_ENOMEM
     assert "scratch" in str(e.value)
     torch.cuda.synchronize()
-    assert not bool(y.any())  # rejected before anything was launched
-    # the same layer at batch 1 fits (4.5 bytes per channel) and is served
-    ref = polyq_lib.linear_gemv(dev, _x_dev(xb[:1]))
-    y1 = torch.empty(1, N, device="cuda")
-    polyq_lib.linear_gemv_noalloc(dev, _x_dev(xb[:1]), y1)
-    torch.cuda.synchronize()
-    _same(y1, ref)
+    assert bool((y == 7.0).all())  # rejected before anything was launched
+
+
+def test_noalloc_wide_layer_many_pieces(polyq_lib):
+    # The same layer at batch 1 fits (256 steps of 256 channels).  Its one
+    # tile is split over every CTA, so one owner adds hundreds of pieces.
+    dev, a = _wide_layer(polyq_lib)
+    assert polyq_lib.gemv_workspace_bytes(dev, 1) <= polyq_lib.NOALLOC_SCRATCH_BYTES
+    xb, _ = synth.activations(a, 1, 74)
+    x = _x_dev(xb)
+    ref = polyq_lib.linear_gemv(dev, x)
+    y = torch.empty(1, dev.N, device="cuda")
+    for _ in range(2):
+        y.fill_(float("nan"))
+        polyq_lib.linear_gemv_noalloc(dev, x, y)
+        torch.cuda.synchronize()
+        _same(y, ref)
