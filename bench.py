@@ -190,27 +190,42 @@ def run_polyq(args):
     with torch.cuda.stream(stream):
         run_step(0)  # warm the launch path once before capture
     stream.synchronize()
-    graphs = []      # one graph per layer copy: the four launches of a step
-    lin_graphs = []  # one graph per (linear, copy): per-launch diagnostics
-    for c in range(args.copies):
+    # Steps run as a decoder stack does: one CUDA graph holds `copies`
+    # consecutive steps (each on its own copy of the layer, so the weights
+    # stream from HBM every step); a K-step run replays it K // copies times
+    # and then a graph of the remaining K % copies steps.
+    def step_graph(n):
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, stream=stream):
-            run_step(c)
-        graphs.append(g)
+            for c in range(n):
+                run_step(c)
+        return g
+
+    cycle = step_graph(args.copies)
+    rest = {}
+
+    def run_steps(k):
+        for _ in range(k // args.copies):
+            cycle.replay()
+        r = k % args.copies
+        if r:
+            if r not in rest:
+                rest[r] = step_graph(r)
+            rest[r].replay()
+
+    lin_graphs = []  # per linear: one graph of that linear on every copy
     for i in range(n_lin):
-        row = []
-        for c in range(args.copies):
-            g = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(g, stream=stream):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            for c in range(args.copies):
                 polyq.linear_gemv(layers[i][c], xs[i], y=ys[i], workspace=wbuf, stream=stream)
-            row.append(g)
-        lin_graphs.append(row)
+        lin_graphs.append(g)
     torch.cuda.synchronize()
 
     # graph replays launch on the current stream: make it `stream`
     with torch.cuda.stream(stream):
-        for s in range(args.warmup):
-            graphs[s % args.copies].replay()
+        run_steps(args.warmup)
+        run_steps(args.steps % args.copies)  # captures the remainder graph outside the timing
     torch.cuda.synchronize()
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
@@ -219,8 +234,7 @@ def run_polyq(args):
     torch.cuda.synchronize()
     with ClockSampler(local) as clk, torch.cuda.stream(stream):
         t0.record(stream)
-        for s in range(args.steps):
-            graphs[s % args.copies].replay()
+        run_steps(args.steps)
         t1.record(stream)
         torch.cuda.synchronize()
     if ws > 1:
@@ -234,24 +248,22 @@ def run_polyq(args):
     value_tbs = ws * step_bytes * args.steps / (ms * 1e-3) / 1e12
 
     # Roofline of the dominant kernel.  The timed region holds only GEMV
-    # launches (pre-pass + streaming kernel per linear), back to back in one
-    # graph per step, so its duration per launch is the step time split over
-    # the launches.  A per-linear breakdown comes from single-GEMV graphs
-    # replayed back to back (weights still rotate over the copies).
+    # launches (pre-pass + streaming kernel per linear), back to back, so its
+    # duration per launch is the step time split over the launches.  A
+    # per-linear breakdown comes from graphs of one linear on every copy.
     per_lin_us = {}
-    reps = max(args.copies * 4, 24)
+    reps = 8
     for i in range(n_lin):
         e0 = torch.cuda.Event(enable_timing=True)
         e1 = torch.cuda.Event(enable_timing=True)
         with torch.cuda.stream(stream):
-            for r in range(args.copies):
-                lin_graphs[i][r].replay()
+            lin_graphs[i].replay()
             e0.record(stream)
             for r in range(reps):
-                lin_graphs[i][r % args.copies].replay()
+                lin_graphs[i].replay()
             e1.record(stream)
         torch.cuda.synchronize()
-        us = 1e3 * e0.elapsed_time(e1) / reps
+        us = 1e3 * e0.elapsed_time(e1) / (reps * args.copies)
         per_lin_us[LLAMA[i][0]] = {"us": round(us, 2),
                                    "GB/s": round(per_lin_bytes[i] / (us * 1e-6) / 1e9, 1)}
     ach = step_bytes / (ms_step * 1e-3) / 1e9
@@ -313,8 +325,9 @@ def run_polyq(args):
                              f"{L2 / 2**20:.0f} MiB)",
                        "bytes_per_step": step_bytes,
                        "b_real": {n: round(inf["b_real"], 5) for n, inf in infos},
-                       "launch_groups": "q+k+v, o, gate+up, down (4 launches of 2 kernels)",
-                       "graph": "one CUDA graph per layer copy"},
+                       "launch_groups": "q+k+v, o, gate+up, down (4 calls of 2 kernels)",
+                       "graph": f"one CUDA graph of {args.copies} steps (one per layer "
+                                "copy), replayed"},
             "pct_of_peak": round(100 * value_tbs * 1e3 / (hbm * ws), 2),
             "roofline": roof,
             "cpu_baseline": cpu,

@@ -182,29 +182,25 @@ int polyq_gemv_workspace_bytes(const polyq_dev_layer* layer, int batch,
  * x: device bf16 [batch][K] (the activation in its producer's basis), every
  * value within the fp16 range (|x| <= 65504): the kernel multiplies fp16
  * copies of x (exact for values in the fp16 normal range) with the decoded
- * codes and accumulates in fp32.  batch in 1..4; y: device fp32 [batch][N],
- * written exactly once per element; residual: device fp32 [batch][N] or NULL
- * (y may alias residual).  workspace: device scratch of at least
+ * codes and accumulates in fp32.  batch in 1..4; y: device fp32 [batch][N];
+ * residual: device fp32 [batch][N] or NULL (y may alias residual).  y is
+ * first set to the residual (or zero), then each of the few pieces a row's
+ * sum is split into is added with an fp32 atomic addition, so the last bits
+ * of y may differ from run to run.  workspace: device scratch of at least
  * polyq_gemv_workspace_bytes(), 256-byte aligned, zero-filled before its
- * first use.  Its first 128.25 KiB hold a status word and tile counters
- * that every call leaves at zero, so one workspace may serve consecutive
- * calls of any shapes on one stream, but not calls that run at the same
- * time.  When a bounded
- * device wait gives up, the first 4 bytes (status word) become non-zero and
- * the workspace must be zero-filled again.  One call covers at most 8192
- * tiles of 64 output rows and 4096 steps (POLYQ_EUNSUPPORTED otherwise).
- * One kernel launch; results are identical from run to run. */
+ * first use; its first 4 bytes are a status word that stays zero unless a
+ * bounded device wait gave up (then zero it again).  A workspace may serve
+ * consecutive calls on one stream but not calls that run at the same time.
+ * Two kernel launches (activation pre-pass, streaming kernel). */
 int polyq_linear_gemv(const polyq_dev_layer* layer, const void* x, int batch,
                       float* y, const float* residual, void* workspace,
                       size_t workspace_bytes, void* stream);
 
 /* Scratch, in bytes, compiled into the library for polyq_linear_gemv_noalloc
- * (1 MiB).  A call needs 128.25 KiB of counters, one activation
- * record per step of K (1152 bytes per 512 channels at batch 1, 1344 bytes
- * per 128 channels at batch 4) and 256 * NB bytes of piece sums per CTA
- * (NB = 1, 2 or 4 for batch 1, 2 or 3-4; three CTAs per SM).  On a 152-SM
- * GPU every layer with K <= 32768 and N <= 524288 fits at any batch and any
- * mix of widths (see polyq_gemv_workspace_bytes). */
+ * (1 MiB).  A call needs 256 bytes plus one activation record per step of K
+ * (1152 bytes per 512 channels at batch 1, 1344 bytes per 128 channels at
+ * batch 4), so every layer with K <= 65536 fits at any batch and any mix of
+ * widths; N does not matter (see polyq_gemv_workspace_bytes). */
 #define POLYQ_NOALLOC_SCRATCH_BYTES (1u << 20)
 
 /* polyq_linear_gemv without a workspace argument: it allocates no device
@@ -222,10 +218,10 @@ int polyq_linear_gemv(const polyq_dev_layer* layer, const void* x, int batch,
  * the same array, so calls whose kernels may overlap on the GPU (different
  * streams, or different host threads without ordering) race and corrupt each
  * other's results; serialise them, e.g. on one stream.  Each call clears the
- * scratch's synchronisation state (cudaMemsetAsync of its first 128.25 KiB
- * on `stream`, no allocation) before its kernel runs, and the kernel writes
- * every record and piece sum before reading it, so nothing left by an
- * earlier call leaks into a later one.
+ * scratch's status word (cudaMemsetAsync of 256 bytes on `stream`, no
+ * allocation) before its kernels run, and the pre-pass writes every record
+ * before the main kernel reads it, so nothing left by an earlier call leaks
+ * into a later one.
  * Arguments and results are those of polyq_linear_gemv.  Returns
  * POLYQ_ENOMEM, touching nothing, when the layer and batch need more than
  * POLYQ_NOALLOC_SCRATCH_BYTES (see polyq_gemv_workspace_bytes). */

@@ -24,13 +24,10 @@
 //    accumulation and its scale/zero apply once:
 //        y += s * (D - 1024*sum(x') - z*sum(x)).
 //    16-bit blocks feed their fp16 weights to the same MMA directly.
-//  * Row sums stay in registers across a tile's steps.  A tile whose steps
-//    are split over CTAs is finished by the CTA holding its first step (its
-//    "owner"): the other pieces, which are the first items of later CTAs,
-//    leave their sums in the workspace and count up a per-tile counter; the
-//    owner waits for the count, adds the pieces in CTA order and the
-//    residual, and stores y once.  Results are therefore reproducible bit for
-//    bit, and y is never read before it is written.
+//  * Row sums stay in registers across a tile's steps.  The pre-pass sets y
+//    to the residual (or zero); each piece of a tile adds its rows into y
+//    with one fp32 atomic addition per row, so a tile split over CTAs gets
+//    its few additions in an order that may vary from run to run.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
@@ -54,9 +51,6 @@ constexpr int kCtasPerSm = 3;
 constexpr int kMaxGrid = 1024;  // persistent CTAs at most
 constexpr int kThreads = 32 * (kWarps + 1);
 constexpr int kConsumers = 32 * kWarps;
-constexpr int kStatusFixupTimeout = 3;
-// Upper bound on the time an owner waits for the other pieces of its tile.
-constexpr unsigned long long kFixupWaitNs = 2000000000ull;
 
 struct GvBlock {
   int bits, n_ch, pos0, seg_off, grp_off;
@@ -74,7 +68,6 @@ struct GvLayer {
   int steps;  // steps per row
   int items;  // tiles * steps
   int item0;  // first item of this layer in the call's list
-  int tile0;  // first tile of this layer in the call's tile counters
   int rec0;   // first activation record of this layer (one per step)
   const __nv_bfloat16* x;
   const int32_t* gather;
@@ -91,9 +84,7 @@ struct GvParams {
   uint32_t magic;  // 0x64006400 (two fp16 1024.0), kept in a register
   // workspace
   int* status;     // sticky error word
-  uint32_t* cnt;   // [tiles][kWarps] piece counters, zero between calls
   uint8_t* rec;    // [recs][rec_bytes(NB)] activation records
-  float* part;     // [grid][kRows][NB] piece sums
 };
 
 // Per-CTA shared copy of the scalars and block tables (runtime-indexed reads
@@ -104,7 +95,6 @@ struct GvShared {
   int N[POLYQ_MAX_GROUP];
   int steps[POLYQ_MAX_GROUP];
   int item0[POLYQ_MAX_GROUP + 1];
-  int tile0[POLYQ_MAX_GROUP];
   int rec0[POLYQ_MAX_GROUP + 1];
 };
 
@@ -123,7 +113,6 @@ __device__ __forceinline__ void load_shared(const GvParams& P, GvShared* S) {
       S->N[l] = P.L[l].N;
       S->steps[l] = P.L[l].steps;
       S->item0[l] = P.L[l].item0;
-      S->tile0[l] = P.L[l].tile0;
       S->rec0[l] = P.L[l].rec0;
     }
   }
@@ -544,18 +533,6 @@ __device__ __forceinline__ void step_16(const GvParams& P, const GvBlock& B, int
   }
 }
 
-__device__ __forceinline__ uint32_t ld_acquire_u32(const uint32_t* p) {
-  uint32_t v;
-  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-  return v;
-}
-
-__device__ __forceinline__ unsigned long long global_ns() {
-  unsigned long long t;
-  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-  return t;
-}
-
 __device__ __forceinline__ void fence_proxy_async_global() {
   asm volatile("fence.proxy.async.global;" ::: "memory");
 }
@@ -580,9 +557,20 @@ __global__ void __launch_bounds__(kConsumers) gemv_prep(const __grid_constant__ 
   rec_pos(S, P.n_layers, r, &l, &bi, &j);
   int src[2][2];
   rec_sources<NB>(P, S.blk[l][bi], l, j, warp, lane, s_p3, src);  // static layer data
-  pdl_wait();  // x comes from the previous kernel; the records may still be in use
+  pdl_wait();  // x comes from the previous kernel; the records and y may still be in use
   rec_build<NB>(P, S.blk[l][bi], l, j, warp, lane, s_p3, src,
                 reinterpret_cast<uint32_t*>(P.rec + (size_t)r * rec_bytes(NB)));
+  // y starts as the residual (or zero); the main kernel adds its pieces
+#pragma unroll
+  for (int q = 0; q < POLYQ_MAX_GROUP; ++q) {
+    if (q >= P.n_layers) break;
+    float* y = P.L[q].y;
+    const float* res = P.L[q].residual;
+    if (y == res) continue;
+    const int total = P.batch * P.L[q].N;
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < total; i += gridDim.x * blockDim.x)
+      y[i] = res ? res[i] : 0.f;
+  }
 }
 
 template <int NB>
@@ -687,7 +675,6 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) gemv_main(const __grid_c
 
   // ---------------- consumers ----------------
   const int g = lane >> 2, t = lane & 3;
-  const int tid = threadIdx.x;
   pdl_wait();  // y, the workspace and the records are this call's from here on
   float acc[2][NB];
 #pragma unroll
@@ -718,7 +705,9 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) gemv_main(const __grid_c
     if (lane == 0) mbar_arrive(empty0 + 8 * slot);
 
     if (it.tile_end(S) || k == n_mine - 1) {
-      // ---- finish this warp's 16 rows of the tile piece ----
+      // ---- add this warp's 16 rows of the tile piece into y ----
+      // Sum the four lanes of each row; lane t adds batch row t.  A tile
+      // whose steps are split over CTAs gets one addition per piece.
 #pragma unroll
       for (int r = 0; r < 2; ++r)
 #pragma unroll
@@ -728,82 +717,20 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) gemv_main(const __grid_c
           v += __shfl_xor_sync(0xffffffffu, v, 2);
           acc[r][b] = v;
         }
-      const int l = it.l;
-      const int steps = S.steps[l];
-      const int T0 = S.item0[l] + it.tile * steps;  // first item of the tile
-      const int T1 = T0 + steps - 1;
-      const int N = S.N[l];
-      uint32_t* cnt = P.cnt + (size_t)(S.tile0[l] + it.tile) * kWarps + warp;
-      // lane t finishes batch row t of rows g and g+8
-      float mine[2];
+      float* y = P.L[0].y;
+#pragma unroll
+      for (int q = 1; q < POLYQ_MAX_GROUP; ++q)
+        if (q == it.l) y = P.L[q].y;
+      const int N = S.N[it.l];
 #pragma unroll
       for (int r = 0; r < 2; ++r) {
-        mine[r] = 0.f;
+        const int n = it.tile * kRows + warp * 16 + g + 8 * r;
 #pragma unroll
         for (int b = 0; b < NB; ++b)
-          if (b == t) mine[r] = acc[r][b];
-      }
-      const bool active = t < P.batch;
-      if (T0 < lo) {
-        // not the owner: leave this piece for the CTA holding the tile's
-        // first step
-        if (active) {
-#pragma unroll
-          for (int r = 0; r < 2; ++r)
-            P.part[((size_t)blockIdx.x * kRows + warp * 16 + g + 8 * r) * NB + t] = mine[r];
-        }
-        __threadfence();
-        __syncwarp();
-        if (lane == 0) atomicAdd(cnt, 1u);
-      } else {
-        int c_last = blockIdx.x;
-        if (T1 >= hi) {
-          // the other pieces sit at the start of CTAs blockIdx.x+1 .. c_last
-          c_last = (int)(((long long)(T1 + 1) * C - 1) / I);
-          const uint32_t need = (uint32_t)(c_last - (int)blockIdx.x);
-          if (lane == 0 && !s_abort) {
-            const unsigned long long t_start = global_ns();
-            while (ld_acquire_u32(cnt) < need) {
-              __nanosleep(64);
-              if (global_ns() - t_start > kFixupWaitNs) {
-                atomicExch(P.status, kStatusFixupTimeout);
-                break;
-              }
-            }
-          }
-          __syncwarp();
-          __threadfence();
-        }
-        float* y = P.L[0].y;
-        const float* res = P.L[0].residual;
-#pragma unroll
-        for (int q = 1; q < POLYQ_MAX_GROUP; ++q)
-          if (q == l) {
-            y = P.L[q].y;
-            res = P.L[q].residual;
-          }
-#pragma unroll
-        for (int r = 0; r < 2; ++r) {
-          const int row = warp * 16 + g + 8 * r;
-          const int n = it.tile * kRows + row;
-          float v = mine[r];
-          if (active)
-            for (int c = (int)blockIdx.x + 1; c <= c_last; ++c)
-              v += __ldcg(P.part + ((size_t)c * kRows + row) * NB + t);
-          if (active && n < N) {
-            const size_t o = (size_t)t * N + n;
-            y[o] = (res ? res[o] : 0.f) + v;
-          }
-        }
-        if (c_last != (int)blockIdx.x) {
-          __syncwarp();
-          if (lane == 0) *cnt = 0u;
-        }
-      }
-#pragma unroll
-      for (int r = 0; r < 2; ++r)
+          if (b == t && b < P.batch && n < N) atomicAdd(y + (size_t)b * N + n, acc[r][b]);
 #pragma unroll
         for (int b = 0; b < NB; ++b) acc[r][b] = 0.f;
+      }
     }
     it.next(S, nl);
   }
@@ -844,44 +771,30 @@ int grid_for(int items, int* grid) {
   return POLYQ_OK;
 }
 
-// Workspace.  The tile counters sit at a fixed offset with a fixed capacity,
-// so that calls of different shapes can share one workspace without one
-// call's data landing on another's counters:
-//   [0, 256)               status word
-//   [256, +16*kMaxTiles)   tile piece counters (zero between calls)
-// then this call's activation records and piece sums.
-constexpr int kMaxRecs = 4096;
-constexpr int kMaxTiles = 8192;
+// Workspace: [0, 256) status word, then one activation record per step of
+// every layer of the call.
 struct WsLayout {
-  size_t cnt_off, rec_off, part_off, bytes;
-  int grid, tiles, items, recs;
+  size_t rec_off, bytes;
+  int grid, items, recs;
 };
 
 int workspace_layout(const polyq_dev_layer* const* L, int n, int batch, WsLayout* w) {
   const int nb = nb_of(batch);
-  long long items = 0, tiles = 0, recs = 0;
+  long long items = 0, recs = 0;
   for (int i = 0; i < n; ++i) {
     const long long t = (L[i]->N + kRows - 1) / kRows;
     const long long st = steps_of(L[i], nb, nullptr);
-    tiles += t;
     items += t * st;
     recs += st;
   }
-  if (items > (1ll << 30) || tiles > kMaxTiles || recs > kMaxRecs)
-    return polyq_set_error(POLYQ_EUNSUPPORTED,
-                           "polyq gemv: a call covers at most %d row tiles of 64 and %d steps "
-                           "(got %lld and %lld)",
-                           kMaxTiles, kMaxRecs, tiles, recs);
+  if (items > (1ll << 30) || recs > (1ll << 20))
+    return polyq_set_error(POLYQ_EUNSUPPORTED, "polyq gemv: too many work items (%lld)", items);
   w->items = (int)items;
-  w->tiles = (int)tiles;
   w->recs = (int)recs;
   int rc = grid_for(w->items, &w->grid);
   if (rc) return rc;
-  auto up = [](size_t v) { return (v + 255) / 256 * 256; };
-  w->cnt_off = 256;
-  w->rec_off = w->cnt_off + (size_t)kMaxTiles * kWarps * 4;
-  w->part_off = w->rec_off + up((size_t)recs * rec_bytes(nb));
-  w->bytes = w->part_off + (size_t)w->grid * kRows * nb * 4;
+  w->rec_off = 256;
+  w->bytes = w->rec_off + (size_t)recs * rec_bytes(nb);
   return POLYQ_OK;
 }
 
@@ -957,7 +870,7 @@ int gemv_group(const char* who, const polyq_dev_layer* const* L, int n, const vo
   const int nb = nb_of(batch);
   GvParams P;
   memset(&P, 0, sizeof P);
-  int items = 0, tiles = 0, recs = 0;
+  int items = 0, recs = 0;
   for (int i = 0; i < n; ++i) {
     GvLayer& G = P.L[i];
     const polyq_dev_layer* D = L[i];
@@ -980,14 +893,12 @@ int gemv_group(const char* who, const polyq_dev_layer* const* L, int n, const vo
     const int t = (int)((D->N + kRows - 1) / kRows);
     G.items = t * steps;
     G.item0 = items;
-    G.tile0 = tiles;
     G.rec0 = recs;
     G.x = (const __nv_bfloat16*)xs[i];
     G.gather = D->gather;
     G.y = ys[i];
     G.residual = res ? res[i] : nullptr;
     items += G.items;
-    tiles += t;
     recs += steps;
   }
   P.n_layers = n;
@@ -997,9 +908,7 @@ int gemv_group(const char* who, const polyq_dev_layer* const* L, int n, const vo
   P.magic = kMagic;
   uint8_t* ws = (uint8_t*)workspace;
   P.status = (int*)ws;
-  P.cnt = (uint32_t*)(ws + w.cnt_off);
   P.rec = ws + w.rec_off;
-  P.part = (float*)(ws + w.part_off);
   switch (nb) {
     case 1: return launch<1>(P, w.grid, st);
     case 2: return launch<2>(P, w.grid, st);
@@ -1120,10 +1029,10 @@ extern "C" int polyq_linear_gemv_noalloc(const polyq_dev_layer* L, const void* x
   void* scratch = nullptr;
   rc = noalloc_scratch(&scratch);
   if (rc) return rc;
-  // The status word and the tile counters must start at zero.  Finished
-  // calls leave them so, but one that gave up on a wait may not, and this
-  // caller cannot reset the library's array itself: clear them on every call.
-  cudaError_t e = cudaMemsetAsync(scratch, 0, w.rec_off, (cudaStream_t)stream);
+  // The status word must start at zero.  A call that gave up on a wait
+  // leaves it set, and this caller cannot reset the library's array itself:
+  // clear it on every call.
+  cudaError_t e = cudaMemsetAsync(scratch, 0, 256, (cudaStream_t)stream);
   if (e != cudaSuccess)
     return polyq_set_error(POLYQ_ECUDA, "%s: clearing the scratch counters: %s", who,
                            cudaGetErrorString(e));

@@ -21,8 +21,8 @@ def _x_dev(xb):
 
 
 def _same(got, ref):
-    # two runs of the GEMV kernels differ only in the order of the fp32 atomic
-    # additions of split tiles: the run-to-run tolerance of the GEMV tests
+    # two runs of the GEMV differ only in the order of the fp32 additions of
+    # split rows: the run-to-run tolerance of the GEMV tests
     assert torch.allclose(got, ref, rtol=1e-5, atol=1e-5 * float(ref.abs().max()))
 
 
@@ -63,9 +63,9 @@ def test_noalloc_matches_workspace_entry_on_two_calls(polyq_lib):
     _same(y2b, ref2)
 
 
-def _wide_layer(polyq_lib):
-    # one 64-row tile (16 rows) of K = 65536 all-8-bit channels
-    N, K = 16, 65536
+def _wide_layer(polyq_lib, K):
+    # one 64-row tile (16 rows) of K all-8-bit channels
+    N = 16
     W, a = synth.layer_weights(N, K, 74)
     bits = np.full(K, 8, dtype=np.uint8)
     dev = polyq_lib.DeviceLayer(polyq_lib.HostLayer.pack(W, a, 8.0, forced_bits=bits), "cuda")
@@ -73,9 +73,9 @@ def _wide_layer(polyq_lib):
 
 
 def test_noalloc_rejects_layers_beyond_the_scratch(polyq_lib):
-    # At batch 4 a step covers 128 channels, so this layer has 512 steps whose
+    # At batch 4 a step covers 128 channels, so K = 131072 has 1024 steps whose
     # activation records (1344 bytes each) do not fit the fixed 1 MiB.
-    dev, a = _wide_layer(polyq_lib)
+    dev, a = _wide_layer(polyq_lib, 131072)
     assert polyq_lib.gemv_workspace_bytes(dev, 4) > polyq_lib.NOALLOC_SCRATCH_BYTES
     xb, _ = synth.activations(a, 4, 74)
     y = torch.full((4, dev.N), 7.0, device="cuda")
@@ -88,14 +88,14 @@ def test_noalloc_rejects_layers_beyond_the_scratch(polyq_lib):
 
 
 def test_noalloc_wide_layer_many_pieces(polyq_lib):
-    # The same layer at batch 1 fits (256 steps of 256 channels).  Its one
-    # tile is split over every CTA, so one owner adds hundreds of pieces.
-    dev, a = _wide_layer(polyq_lib)
-    assert polyq_lib.gemv_workspace_bytes(dev, 1) <= polyq_lib.NOALLOC_SCRATCH_BYTES
-    xb, _ = synth.activations(a, 1, 74)
+    # K = 65536 fits at batch 4 (512 steps of 128 channels).  Its one tile is
+    # split over hundreds of CTAs, each adding its piece into y.
+    dev, a = _wide_layer(polyq_lib, 65536)
+    assert polyq_lib.gemv_workspace_bytes(dev, 4) <= polyq_lib.NOALLOC_SCRATCH_BYTES
+    xb, _ = synth.activations(a, 4, 74)
     x = _x_dev(xb)
     ref = polyq_lib.linear_gemv(dev, x)
-    y = torch.empty(1, dev.N, device="cuda")
+    y = torch.empty(4, dev.N, device="cuda")
     for _ in range(2):
         y.fill_(float("nan"))
         polyq_lib.linear_gemv_noalloc(dev, x, y)
