@@ -398,7 +398,7 @@ __device__ __forceinline__ void load_words(uint32_t* w, const uint8_t* codes, in
 // One step of a b<16 block for this warp's 16 rows; adds the chunk results,
 // scaled, into acc[row][batch].
 template <int NB, int BITS>
-__device__ __forceinline__ void step_mma(const GvParams& P, const GvBlock& B, int j,
+__device__ __forceinline__ void step_mma(const GvParams& P, int uvalid, int g0,
                                          const uint8_t* stage, const uint32_t* rec,
                                          const uint32_t* zeros, int warp, int lane,
                                          float (&acc)[2][NB]) {
@@ -428,7 +428,6 @@ __device__ __forceinline__ void step_mma(const GvParams& P, const GvBlock& B, in
   const int my_b = g / NGS, my_c = g % NGS;
   const int dc = my_b < P.batch ? my_c - lane_unit(BITS, NB, t, 0) / 64 : -1000;
   const uint32_t* brow = rec + (my_b * 4 + t) * LW;
-  const int uvalid = min(U, B.n_ch - j * U);
 
   float d[4][4];
 #pragma unroll
@@ -459,8 +458,8 @@ __device__ __forceinline__ void step_mma(const GvParams& P, const GvBlock& B, in
 #pragma unroll
   for (int v = 0; v < 4; ++v) D[v] = (d[0][v] + d[1][v]) + (d[2][v] + d[3][v]);
 
-  // epilogue: columns 2t, 2t+1 -> (batch, chunk) (col / NGS, col % NGS)
-  const int g0 = (B.grp_off + j * NGS) & 3;  // first group of the step in the meta box
+  // epilogue: columns 2t, 2t+1 -> (batch, chunk) (col / NGS, col % NGS);
+  // g0 is the step's first group in the meta box
   const float* recf = reinterpret_cast<const float*>(rec);
 #pragma unroll
   for (int cc = 0; cc < 2; ++cc) {
@@ -487,7 +486,7 @@ __device__ __forceinline__ void step_mma(const GvParams& P, const GvBlock& B, in
 // n of B is batch row n.  Lane t holds weights [16t, 16t+16) of each of the
 // two 64-weight boxes.
 template <int NB>
-__device__ __forceinline__ void step_16(const GvParams& P, const GvBlock& B, int j,
+__device__ __forceinline__ void step_16(const GvParams& P, int uvalid,
                                         const uint8_t* stage, const uint32_t* rec,
                                         const uint32_t* zeros, int warp, int lane,
                                         float (&acc)[2][NB]) {
@@ -496,7 +495,6 @@ __device__ __forceinline__ void step_16(const GvParams& P, const GvBlock& B, int
   static_assert(box_pitch(16, NB) == PITCH && nbox_of(16, NB) == 2, "16-bit geometry");
   const int g = lane >> 2, t = lane & 3;
   const int rA = warp * 16 + g, rB = rA + 8;
-  const int uvalid = min(128, B.n_ch - j * 128);
   const uint32_t* bsrc = g < P.batch ? rec + (g * 4 + t) * LW : zeros;
   float d[2][4];
 #pragma unroll
@@ -627,6 +625,19 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) gemv_main(const __grid_c
       }
       const uint32_t dst = smem_u32(stages + slot * kStageBytes);
       const uint32_t bar = full0 + 8 * slot;
+      {
+        // what the consumers need of this item: width, whether the item ends
+        // a tile piece, layer, valid units, first meta entry, tile
+        const int uvalid = min(B.units, B.n_ch - q.j * B.units);
+        const int g0 = (B.grp_off + q.j * (B.units / 64)) & 3;
+        const bool flush = q.tile_end(S) || k == n_mine - 1;
+        uint4 d;
+        d.x = (uint32_t)B.bits | ((uint32_t)flush << 8) | ((uint32_t)q.l << 16);
+        d.y = (uint32_t)uvalid | ((uint32_t)g0 << 16);
+        d.z = (uint32_t)q.tile;
+        d.w = 0u;
+        *reinterpret_cast<uint4*>(stages + slot * kStageBytes + kDescOff) = d;
+      }
       uint32_t bytes = nbx * pitch * kRows + RB;
       if (B.bits < 16) bytes += kMetaBytes;
       mbar_expect_tx(bar, bytes);
@@ -666,7 +677,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) gemv_main(const __grid_c
         issue_weights(k, it);
       }
       const int r = S.rec0[it.l] + it.s;
-      bulk_load(smem_u32(stages + slot * kStageBytes + kCodesBytes + kMetaBytes),
+      bulk_load(smem_u32(stages + slot * kStageBytes + kRecOff),
                 P.rec + (size_t)r * RB, RB, full0 + 8 * slot);
       it.next(S, nl);
     }
@@ -681,30 +692,34 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) gemv_main(const __grid_c
   for (int r = 0; r < 2; ++r)
 #pragma unroll
     for (int b = 0; b < NB; ++b) acc[r][b] = 0.f;
-  ItemPos it;
-  it.init(S, nl, lo);
+  int slot = 0;
+  uint32_t phase = 0;
   for (int k = 0; k < n_mine; ++k) {
-    const int slot = k % kStages;
-    if (s_abort || !mbar_wait(full0 + 8 * slot, (k / kStages) & 1)) {
+    if (s_abort || !mbar_wait(full0 + 8 * slot, phase)) {
       if (lane == 0 && !s_abort) atomicExch(P.status, kStatusTimeoutFull);
       s_abort = 1;
-      it.next(S, nl);
-      continue;
+      break;
     }
-    const GvBlock B = S.blk[it.l][it.bi];
     const uint8_t* stage = stages + slot * kStageBytes;
-    const uint32_t* rec = reinterpret_cast<const uint32_t*>(stage + kCodesBytes + kMetaBytes);
-    switch (B.bits) {
-      case 2: step_mma<NB, 2>(P, B, it.j, stage, rec, zeros, warp, lane, acc); break;
-      case 3: step_mma<NB, 3>(P, B, it.j, stage, rec, zeros, warp, lane, acc); break;
-      case 4: step_mma<NB, 4>(P, B, it.j, stage, rec, zeros, warp, lane, acc); break;
-      case 8: step_mma<NB, 8>(P, B, it.j, stage, rec, zeros, warp, lane, acc); break;
-      default: step_16<NB>(P, B, it.j, stage, rec, zeros, warp, lane, acc); break;
+    const uint32_t* rec = reinterpret_cast<const uint32_t*>(stage + kRecOff);
+    const uint4 desc = *reinterpret_cast<const uint4*>(stage + kDescOff);
+    const int bits = (int)(desc.x & 0xFFu);
+    const int uvalid = (int)(desc.y & 0xFFFFu), g0 = (int)(desc.y >> 16);
+    switch (bits) {
+      case 2: step_mma<NB, 2>(P, uvalid, g0, stage, rec, zeros, warp, lane, acc); break;
+      case 3: step_mma<NB, 3>(P, uvalid, g0, stage, rec, zeros, warp, lane, acc); break;
+      case 4: step_mma<NB, 4>(P, uvalid, g0, stage, rec, zeros, warp, lane, acc); break;
+      case 8: step_mma<NB, 8>(P, uvalid, g0, stage, rec, zeros, warp, lane, acc); break;
+      default: step_16<NB>(P, uvalid, stage, rec, zeros, warp, lane, acc); break;
     }
     __syncwarp();
     if (lane == 0) mbar_arrive(empty0 + 8 * slot);
+    if (++slot == kStages) {
+      slot = 0;
+      phase ^= 1u;
+    }
 
-    if (it.tile_end(S) || k == n_mine - 1) {
+    if (desc.x & 0x100u) {
       // ---- add this warp's 16 rows of the tile piece into y ----
       // Sum the four lanes of each row; lane t adds batch row t.  A tile
       // whose steps are split over CTAs gets one addition per piece.
@@ -717,14 +732,18 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) gemv_main(const __grid_c
           v += __shfl_xor_sync(0xffffffffu, v, 2);
           acc[r][b] = v;
         }
+      const int l = (int)(desc.x >> 16);
       float* y = P.L[0].y;
+      int N = P.L[0].N;
 #pragma unroll
       for (int q = 1; q < POLYQ_MAX_GROUP; ++q)
-        if (q == it.l) y = P.L[q].y;
-      const int N = S.N[it.l];
+        if (q == l) {
+          y = P.L[q].y;
+          N = P.L[q].N;
+        }
 #pragma unroll
       for (int r = 0; r < 2; ++r) {
-        const int n = it.tile * kRows + warp * 16 + g + 8 * r;
+        const int n = (int)desc.z * kRows + warp * 16 + g + 8 * r;
 #pragma unroll
         for (int b = 0; b < NB; ++b)
           if (b == t && b < P.batch && n < N) atomicAdd(y + (size_t)b * N + n, acc[r][b]);
@@ -732,9 +751,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) gemv_main(const __grid_c
         for (int b = 0; b < NB; ++b) acc[r][b] = 0.f;
       }
     }
-    it.next(S, nl);
   }
-
 }
 
 // ---------------------------------------------------------------------------

@@ -30,8 +30,11 @@ constexpr int kMetaBox = 12;       // meta entries per row loaded per step
 constexpr int kCodesBytes = 2 * kRows * kPitchSplit;  // largest codes area (2 boxes)
 constexpr int kMetaBytes = kRows * kMetaBox * 4;
 constexpr int kRecMax = 1344;      // largest activation record (NB = 4)
-// A stage holds an item's code boxes, its scale/zero box and its record.
-constexpr int kStageBytes = ((kCodesBytes + kMetaBytes + kRecMax) + 127) / 128 * 128;
+// A stage holds an item's code boxes, its scale/zero box, its record and a
+// 16-byte descriptor written by the producer.
+constexpr int kRecOff = kCodesBytes + kMetaBytes;
+constexpr int kDescOff = kRecOff + kRecMax;
+constexpr int kStageBytes = ((kDescOff + 16) + 127) / 128 * 128;
 constexpr uint32_t kMagic = 0x64006400u;  // two fp16 1024.0
 constexpr float kMagicF = 1024.0f;
 
