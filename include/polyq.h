@@ -245,6 +245,40 @@ int polyq_linear_gemv_group(const polyq_dev_layer* const* layers, int n,
                             const float* const* residuals, void* workspace,
                             size_t workspace_bytes, void* stream);
 
+/* Activation input of polyq_linear_gemv_input: the glue of a decoder layer
+ * (the residual stream's RMSNorm, SiLU(gate) * up, or a plain rounding to
+ * bf16) fused into the GEMV's record pre-pass.  These are elementwise up to
+ * a per-row scale, so they commute with the channel permutations
+ * (Section 4.3) and run on the gathered values.  Every kind produces the bf16
+ * activation x[b][k] that polyq_linear_gemv would take:
+ *   POLYQ_X_BF16      x = a                      a: bf16 [batch][K]
+ *   POLYQ_X_F32       x = bf16_rn(a)             a: fp32 [batch][K]
+ *   POLYQ_X_RMSNORM   x = bf16_rn(a[b][k] / sqrt(mean_k(a[b][k]^2) + eps))
+ *                                                a: fp32 [batch][K], unit gain
+ *   POLYQ_X_SILU_MUL  x = bf16_rn(a / (1 + exp(-a)) * b)
+ *                                                a, b: fp32 [batch][K]
+ * bf16_rn rounds the fp32 result to nearest even.  x_out (optional, device
+ * bf16 [batch][K]) receives x as computed, in source order. */
+#define POLYQ_X_BF16 0
+#define POLYQ_X_F32 1
+#define POLYQ_X_RMSNORM 2
+#define POLYQ_X_SILU_MUL 3
+typedef struct {
+  int32_t kind;      /* POLYQ_X_* */
+  float eps;         /* POLYQ_X_RMSNORM only */
+  const void* a;     /* device input, see kind */
+  const float* b;    /* device fp32 [batch][K] for POLYQ_X_SILU_MUL, else NULL */
+  uint16_t* x_out;   /* device bf16 [batch][K] or NULL */
+} polyq_gemv_input;
+
+/* polyq_linear_gemv_group with every layer reading the one input `in`
+ * (all layers must have the same K).  Workspace, outputs and residuals as
+ * for polyq_linear_gemv_group. */
+int polyq_linear_gemv_input(const polyq_dev_layer* const* layers, int n,
+                            const polyq_gemv_input* in, int batch, float* const* ys,
+                            const float* const* residuals, void* workspace,
+                            size_t workspace_bytes, void* stream);
+
 /* Device scratch bytes polyq_linear_gemm needs for this layer and M. */
 int polyq_gemm_workspace_bytes(const polyq_dev_layer* layer, int64_t M,
                                size_t* bytes);

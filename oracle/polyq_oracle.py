@@ -435,10 +435,57 @@ def bf16_rn(v):
 
 
 def rmsnorm(s, eps=1e-6):
+    """RMSNorm with unit gain over the last axis: s / sqrt(mean(s^2) + eps)."""
     s = np.asarray(s, dtype=np.float64)
     return s / np.sqrt(np.mean(s * s, axis=-1, keepdims=True) + eps)
 
 
 def silu(v):
+    """SiLU: v * sigmoid(v) = v / (1 + exp(-v))."""
     v = np.asarray(v, dtype=np.float64)
     return v / (1.0 + np.exp(-v))
+
+
+def merge_decoder_layer(lin):
+    """Apply the §4.3 merges of one decoder layer (reading R11): v emits in
+    o's input basis and gate/up emit in down's, so o and down read their
+    input without a gather; q, k, v, gate and up gather the natural-basis
+    stream.  ``lin`` maps q, k, v, o, gate, up, down to packed layers; the
+    result maps each name to (layer, gather) with gather None for identity."""
+    out = {}
+    for name in ("q", "k"):
+        out[name] = (lin[name], lin[name]["perm"])
+    out["v"] = (permute_rows(lin["v"], lin["o"]["perm"]), lin["v"]["perm"])
+    out["o"] = (lin["o"], None)
+    for name in ("gate", "up"):
+        out[name] = (permute_rows(lin[name], lin["down"]["perm"]), lin[name]["perm"])
+    out["down"] = (lin["down"], None)
+    return out
+
+
+def _linear_g(layer_gather, x):
+    layer, gather = layer_gather
+    g = np.arange(layer["K"]) if gather is None else gather
+    return linear(layer, x, gather=g)
+
+
+def decode_layer(s, merged, eps=1e-6):
+    """One decode step of a Llama-shaped layer at position 0 (reading R11):
+    h = bf16(rmsnorm(s)); q, k, v from h; attention over the single cached
+    key returns v, so s += o(bf16(v)); h2 = bf16(rmsnorm(s)); s +=
+    down(bf16(silu(gate(h2)) * up(h2))).  s is the fp32/fp64 residual stream
+    in the natural basis; ``merged`` comes from merge_decoder_layer.  Returns
+    the new stream and the intermediate values by name."""
+    s = np.asarray(s, dtype=np.float64)
+    h = bf16_rn(rmsnorm(s, eps))
+    q = _linear_g(merged["q"], h)
+    k = _linear_g(merged["k"], h)
+    v = _linear_g(merged["v"], h)
+    xo = bf16_rn(v)
+    s1 = s + _linear_g(merged["o"], xo)
+    h2 = bf16_rn(rmsnorm(s1, eps))
+    g = _linear_g(merged["gate"], h2)
+    u = _linear_g(merged["up"], h2)
+    xd = bf16_rn(silu(g) * u)
+    s2 = s1 + _linear_g(merged["down"], xd)
+    return s2, dict(h=h, q=q, k=k, v=v, xo=xo, s1=s1, h2=h2, gate=g, up=u, xd=xd)

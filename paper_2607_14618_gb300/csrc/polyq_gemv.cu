@@ -85,6 +85,13 @@ struct GvParams {
   // workspace
   int* status;     // sticky error word
   uint8_t* rec;    // [recs][rec_bytes(NB)] activation records
+  // input transform shared by all layers (POLYQ_X_*); with POLYQ_X_BF16 each
+  // layer reads its own L[l].x
+  int xkind;
+  float eps;
+  const float* xa;  // fp32 input of the transforms
+  const float* xb;  // second fp32 input of POLYQ_X_SILU_MUL
+  uint16_t* xout;   // optional bf16 copy of the transformed input
 };
 
 // Per-CTA shared copy of the scalars and block tables (runtime-indexed reads
@@ -285,7 +292,8 @@ __device__ __forceinline__ void rec_sources(const GvParams& P, const GvBlock& B,
 template <int NB>
 __device__ __forceinline__ void rec_build(const GvParams& P, const GvBlock& B, int l, int j,
                                           int warp, int lane, const uint32_t* p3,
-                                          const int (&src)[2][2], uint32_t* rec) {
+                                          const int (&src)[2][2], const float* rnorm,
+                                          uint32_t* rec) {
   constexpr int LW = rec_lane_words(NB);
   constexpr int PW = rec_pair_words(NB);
   constexpr int NGM = 8 / NB;
@@ -296,8 +304,27 @@ __device__ __forceinline__ void rec_build(const GvParams& P, const GvBlock& B, i
   for (int s = 0; s < 2; ++s) {
     const SlotGeom g = slot_geom<NB>(B.bits, warp, lane, threadIdx.x, s, j, p3);
 #pragma unroll
-    for (int h = 0; h < 2; ++h)
-      xv[s][h] = src[s][h] >= 0 ? __bfloat162float(x[(size_t)g.bb * K + src[s][h]]) : 0.f;
+    for (int h = 0; h < 2; ++h) {
+      if (src[s][h] < 0) {
+        xv[s][h] = 0.f;
+        continue;
+      }
+      const size_t o = (size_t)g.bb * K + src[s][h];
+      __nv_bfloat16 v;
+      switch (P.xkind) {
+        case POLYQ_X_F32: v = __float2bfloat16_rn(P.xa[o]); break;
+        case POLYQ_X_RMSNORM: v = __float2bfloat16_rn(P.xa[o] * rnorm[g.bb]); break;
+        case POLYQ_X_SILU_MUL: {
+          const float a = P.xa[o];
+          v = __float2bfloat16_rn(a / (1.f + expf(-a)) * P.xb[o]);
+          break;
+        }
+        default: v = x[o]; break;
+      }
+      // layer 0's records cover every source element once
+      if (P.xout && l == 0) P.xout[o] = __bfloat16_as_ushort(v);
+      xv[s][h] = __bfloat162float(v);
+    }
   }
   float* recf = reinterpret_cast<float*>(rec);
 #pragma unroll
@@ -556,7 +583,30 @@ __global__ void __launch_bounds__(kConsumers) gemv_prep(const __grid_constant__ 
   int src[2][2];
   rec_sources<NB>(P, S.blk[l][bi], l, j, warp, lane, s_p3, src);  // static layer data
   pdl_wait();  // x comes from the previous kernel; the records and y may still be in use
-  rec_build<NB>(P, S.blk[l][bi], l, j, warp, lane, s_p3, src,
+  __shared__ float s_rnorm[4];
+  if (P.xkind == POLYQ_X_RMSNORM) {
+    // 1 / sqrt(mean(a^2) + eps) of each batch row
+    __shared__ float s_part[4][kWarps];
+    const int K = P.L[0].K;
+    for (int bb = 0; bb < P.batch; ++bb) {
+      float acc = 0.f;
+      for (int i = threadIdx.x; i < K; i += kConsumers) {
+        const float v = P.xa[(size_t)bb * K + i];
+        acc = fmaf(v, v, acc);
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+      if (lane == 0) s_part[bb][warp] = acc;
+    }
+    __syncthreads();
+    if (threadIdx.x < P.batch) {
+      float t = 0.f;
+      for (int w = 0; w < kWarps; ++w) t += s_part[threadIdx.x][w];
+      s_rnorm[threadIdx.x] = rsqrtf(t / (float)K + P.eps);
+    }
+    __syncthreads();
+  }
+  rec_build<NB>(P, S.blk[l][bi], l, j, warp, lane, s_p3, src, s_rnorm,
                 reinterpret_cast<uint32_t*>(P.rec + (size_t)r * rec_bytes(NB)));
   // y starts as the residual (or zero); the main kernel adds its pieces
 #pragma unroll
@@ -870,9 +920,25 @@ int launch(const GvParams& P, int grid, cudaStream_t st) {
 
 int gemv_group(const char* who, const polyq_dev_layer* const* L, int n, const void* const* xs,
                int batch, float* const* ys, const float* const* res, void* workspace,
-               size_t ws_bytes, cudaStream_t st) {
+               size_t ws_bytes, cudaStream_t st, const polyq_gemv_input* in = nullptr) {
   int rc = check_group(who, L, n, batch);
   if (rc) return rc;
+  const void* shared_x[POLYQ_MAX_GROUP];
+  if (in) {
+    if (in->kind < POLYQ_X_BF16 || in->kind > POLYQ_X_SILU_MUL)
+      return polyq_set_error(POLYQ_EINVAL, "%s: unknown input kind %d", who, in->kind);
+    if (!in->a || (in->kind == POLYQ_X_SILU_MUL) != (in->b != nullptr))
+      return polyq_set_error(POLYQ_EINVAL, "%s: input pointers do not match kind %d", who,
+                             in->kind);
+    if (in->kind == POLYQ_X_RMSNORM && !(in->eps >= 0.f))
+      return polyq_set_error(POLYQ_EINVAL, "%s: eps must be >= 0", who);
+    for (int i = 0; i < n; ++i) {
+      if (L[i]->K != L[0]->K)
+        return polyq_set_error(POLYQ_EINVAL, "%s: layers sharing one input need the same K", who);
+      shared_x[i] = in->a;
+    }
+    xs = shared_x;
+  }
   if (!xs || !ys) return polyq_set_error(POLYQ_EINVAL, "%s: x or y is NULL", who);
   for (int i = 0; i < n; ++i)
     if (!xs[i] || !ys[i]) return polyq_set_error(POLYQ_EINVAL, "%s: x or y %d is NULL", who, i);
@@ -926,6 +992,11 @@ int gemv_group(const char* who, const polyq_dev_layer* const* L, int n, const vo
   uint8_t* ws = (uint8_t*)workspace;
   P.status = (int*)ws;
   P.rec = ws + w.rec_off;
+  P.xkind = in ? in->kind : POLYQ_X_BF16;
+  P.eps = in ? in->eps : 0.f;
+  P.xa = in ? (const float*)in->a : nullptr;
+  P.xb = in ? in->b : nullptr;
+  P.xout = in ? in->x_out : nullptr;
   switch (nb) {
     case 1: return launch<1>(P, w.grid, st);
     case 2: return launch<2>(P, w.grid, st);
@@ -972,6 +1043,16 @@ extern "C" int polyq_linear_gemv(const polyq_dev_layer* L, const void* x, int ba
   const float* rs[1] = {residual};
   return gemv_group("polyq_linear_gemv", one, 1, xs, batch, ys, rs, workspace, ws_bytes,
                     (cudaStream_t)stream);
+}
+
+extern "C" int polyq_linear_gemv_input(const polyq_dev_layer* const* layers, int n,
+                                       const polyq_gemv_input* in, int batch, float* const* ys,
+                                       const float* const* residuals, void* workspace,
+                                       size_t ws_bytes, void* stream) {
+  polyq_clear_error();
+  if (!in) return polyq_set_error(POLYQ_EINVAL, "polyq_linear_gemv_input: input is NULL");
+  return gemv_group("polyq_linear_gemv_input", layers, n, nullptr, batch, ys, residuals,
+                    workspace, ws_bytes, (cudaStream_t)stream, in);
 }
 
 extern "C" int polyq_linear_gemv_group(const polyq_dev_layer* const* layers, int n,

@@ -61,6 +61,14 @@ class Info(C.Structure):
                 ("meta_stride", C.c_int64)]
 
 
+X_BF16, X_F32, X_RMSNORM, X_SILU_MUL = 0, 1, 2, 3
+
+
+class GemvInput(C.Structure):
+    _fields_ = [("kind", C.c_int32), ("eps", C.c_float), ("a", C.c_void_p), ("b", C.c_void_p),
+                ("x_out", C.c_void_p)]
+
+
 class DevLayer(C.Structure):
     _fields_ = [("packed", C.c_void_p), ("meta", C.c_void_p), ("gather", C.c_void_p),
                 ("N", C.c_int64), ("K", C.c_int64), ("row_stride", C.c_int64),
@@ -87,6 +95,10 @@ _SIGS = {
                                                    C.c_int, C.POINTER(C.c_size_t)]),
     "polyq_linear_gemv_group": (C.c_int, [C.POINTER(C.POINTER(DevLayer)), C.c_int,
                                           C.POINTER(C.c_void_p), C.c_int,
+                                          C.POINTER(C.c_void_p), C.POINTER(C.c_void_p),
+                                          _P, C.c_size_t, _P]),
+    "polyq_linear_gemv_input": (C.c_int, [C.POINTER(C.POINTER(DevLayer)), C.c_int,
+                                          C.POINTER(GemvInput), C.c_int,
                                           C.POINTER(C.c_void_p), C.POINTER(C.c_void_p),
                                           _P, C.c_size_t, _P]),
     "polyq_gemm_workspace_bytes": (C.c_int, [C.POINTER(DevLayer), C.c_int64,
@@ -336,6 +348,40 @@ def linear_gemv_group(layers, xs, ys=None, residuals=None, workspace=None, strea
     if residuals is not None:
         ra = (C.c_void_p * n)(*[r.data_ptr() if r is not None else None for r in residuals])
     _check(_lib.polyq_linear_gemv_group(_layer_array(layers), n, xa, batch, ya, ra,
+                                        workspace.data_ptr(), workspace.numel(),
+                                        _stream_ptr(stream)))
+    return ys
+
+
+def linear_gemv_input(layers, kind, a, b=None, eps=1e-6, ys=None, residuals=None, x_out=None,
+                      workspace=None, stream=None):
+    """GEMVs of `layers` on one shared input with its transform fused into the
+    pre-pass (X_BF16, X_F32, X_RMSNORM or X_SILU_MUL, see polyq.h)."""
+    import torch
+    n = len(layers)
+    K = layers[0].K
+    want = torch.bfloat16 if kind == X_BF16 else torch.float32
+    if a.dtype != want or not a.is_cuda or a.dim() != 2 or a.shape[1] != K or not a.is_contiguous():
+        raise ValueError(f"a must be a contiguous CUDA {want} tensor [batch][K]")
+    batch = a.shape[0]
+    if (kind == X_SILU_MUL) != (b is not None):
+        raise ValueError("b is the second input of X_SILU_MUL only")
+    if b is not None and (b.dtype != torch.float32 or b.shape != a.shape or not b.is_contiguous()):
+        raise ValueError("b must be a contiguous fp32 tensor shaped like a")
+    if x_out is not None and (x_out.dtype != torch.bfloat16 or x_out.shape != a.shape):
+        raise ValueError("x_out must be a bf16 tensor shaped like a")
+    if ys is None:
+        ys = [torch.empty((batch, l.N), dtype=torch.float32, device=a.device) for l in layers]
+    need = gemv_group_workspace_bytes(layers, batch)
+    if workspace is None:
+        workspace = torch.zeros(need, dtype=torch.uint8, device=a.device)
+    inp = GemvInput(kind, eps, a.data_ptr(), b.data_ptr() if b is not None else None,
+                    x_out.data_ptr() if x_out is not None else None)
+    ya = (C.c_void_p * n)(*[y.data_ptr() for y in ys])
+    ra = None
+    if residuals is not None:
+        ra = (C.c_void_p * n)(*[r.data_ptr() if r is not None else None for r in residuals])
+    _check(_lib.polyq_linear_gemv_input(_layer_array(layers), n, C.byref(inp), batch, ya, ra,
                                         workspace.data_ptr(), workspace.numel(),
                                         _stream_ptr(stream)))
     return ys

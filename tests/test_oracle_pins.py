@@ -421,3 +421,74 @@ def test_w3_overhead_table():
     for model in ("Falcon-H1-3B", "Llama2-13B", "Qwen3-32B"):
         v = g[model]
         assert round(100 * (3 / v["B_min"] - 1), 1) == v["overhead"]
+
+
+# --------------------------------------------------------------------------
+# decode-step glue and the merged decoder layer (R11)
+# --------------------------------------------------------------------------
+def test_rmsnorm_closed_forms():
+    for c in (3.0, -0.25, 1e3):
+        v = O.rmsnorm(np.full(7, c), eps=1e-6)
+        assert np.allclose(v, np.sign(c) / np.sqrt(1.0 + 1e-6 / (c * c)), rtol=0, atol=1e-15)
+    s = np.random.default_rng(0).standard_normal((3, 50))
+    r = O.rmsnorm(s, eps=0.0)
+    assert np.allclose(np.mean(r * r, axis=-1), 1.0, atol=1e-13)        # unit mean square
+    assert np.allclose(O.rmsnorm(5.5 * s, eps=0.0), r, atol=1e-13)       # scale invariant
+
+
+def test_silu_identities():
+    assert O.silu(0.0) == 0.0
+    x = np.linspace(-8, 8, 33)
+    assert np.allclose(O.silu(x) - O.silu(-x), x, atol=1e-13)           # x*(s(x)+s(-x)) = x
+    assert abs(O.silu(40.0) - 40.0) < 1e-12
+    assert abs(O.silu(1.0) - 1.0 / (1.0 + np.exp(-1.0))) < 1e-15
+
+
+def _small_layer_set(hidden, ffn, seed, bits16=False):
+    lin = {}
+    for i, (name, N, K) in enumerate(O.llama_layer_linears(hidden, ffn)):
+        W, a = synth.layer_weights(N, K, seed + i)
+        bits = np.full(K, 16) if bits16 else None
+        lin[name] = O.pack_layer(W, a, 3.0, bits=bits)
+    return lin
+
+
+def test_merged_layer_equals_unmerged():
+    lin = _small_layer_set(64, 160, 300)
+    s = np.random.default_rng(1).standard_normal((2, 64))
+    merged = O.merge_decoder_layer(lin)
+    plain = {n: (L, L["perm"]) for n, L in lin.items()}
+    s_m, mid_m = O.decode_layer(s, merged)
+    s_p, mid_p = O.decode_layer(s, plain)
+    assert np.allclose(s_m, s_p, rtol=1e-12, atol=1e-12)
+    # v and gate/up come out permuted into o's and down's input orders
+    assert np.allclose(mid_m["v"], mid_p["v"][:, lin["o"]["perm"]], rtol=1e-12, atol=0)
+    assert np.allclose(mid_m["gate"], mid_p["gate"][:, lin["down"]["perm"]], rtol=1e-12, atol=0)
+
+
+def test_decoder_layer_matches_dense_graph():
+    # all-16-bit weights: the layer's weights are fp16(W) in natural order, so
+    # the step is the plain dense graph written out with matmuls
+    hidden, ffn, seed = 48, 96, 310
+    lin = _small_layer_set(hidden, ffn, seed, bits16=True)
+    Wd = {}
+    for i, (name, N, K) in enumerate(O.llama_layer_linears(hidden, ffn)):
+        W, _ = synth.layer_weights(N, K, seed + i)
+        Wd[name] = W.astype(np.float16).astype(np.float64)
+    s = np.random.default_rng(2).standard_normal((1, hidden)) * 3.0
+    out, _ = O.decode_layer(s, O.merge_decoder_layer(lin))
+
+    def bf16(v):
+        return O.bf16_rn(v)
+
+    def rms(v):
+        return v / np.sqrt(np.mean(v * v, axis=-1, keepdims=True) + 1e-6)
+
+    h = bf16(rms(s))
+    v = h @ Wd["v"].T
+    s1 = s + bf16(v) @ Wd["o"].T
+    h2 = bf16(rms(s1))
+    g = h2 @ Wd["gate"].T
+    u = h2 @ Wd["up"].T
+    ref = s1 + bf16(g / (1 + np.exp(-g)) * u) @ Wd["down"].T
+    assert np.allclose(out, ref, rtol=1e-12, atol=1e-12)
