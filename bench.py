@@ -306,6 +306,10 @@ def run_polyq(args):
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": e_steps,
                "ms_per_step": round(1e3 * (tb - ta) / e_steps, 4)}
 
+    decode = None
+    if not args.no_decode:
+        decode = bench_decode_step(polyq, synth, torch, device, stream, args, hbm)
+
     gemm = None
     if not args.no_gemm:
         gemm = bench_gemm(polyq, synth, torch, device, stream, args, tf_burst, tf_sus)
@@ -335,10 +339,133 @@ def run_polyq(args):
             "gpu_launches": args.steps * len(GROUPS) * kernels_per_call,
             "clocks": clk.summary(),
             "prefill_gemm": gemm,
+            "decode_step": decode,
         }
         print(json.dumps(out), flush=True)
     if ws > 1:
         dist.destroy_process_group()
+
+
+def bench_decode_step(polyq, synth, torch, device, stream, args, hbm):
+    """A whole batch-1 decode step of a Llama2-13B-shaped stack: for each of
+    the layers, RMSNorm -> q,k,v -> o (+ residual) -> RMSNorm -> gate,up ->
+    SiLU*up -> down (+ residual), attention at position 0 (output = v).  The
+    glue runs inside the GEMV pre-passes and the §4.3 merges make o and down
+    read their inputs without a gather.  Two modes: `separate` (seven linears,
+    v -> o and gate/up -> down merged) and `grouped` (q/k/v and gate/up each
+    allocated jointly over their stacked rows, sharing one permutation).
+    The layers are device copies of one packed layer set, so every step
+    streams all weights from HBM."""
+    hidden, ffn, L = 5120, 13824, args.decode_layers
+    W = {}
+    for i, (name, N, K) in enumerate(LLAMA):
+        W[name] = synth.layer_weights(N, K, synth.seed_for(5, i))
+    a_in = {"q": W["q"][1], "k": W["q"][1], "v": W["q"][1], "o": W["o"][1],
+            "gate": W["gate"][1], "up": W["gate"][1], "down": W["down"][1]}
+    gathered = {}
+    out = {}
+    for mode in ("separate", "grouped"):
+        if mode == "separate":
+            hosts = {n: polyq.HostLayer.pack(W[n][0], a_in[n], args.budget) for n in W}
+            p_o = hosts["o"].export()["perm"]
+            p_d = hosts["down"].export()["perm"]
+            hosts["v"].permute_rows(p_o)
+            hosts["gate"].permute_rows(p_d)
+            hosts["up"].permute_rows(p_d)
+            names = list(W)
+        else:
+            hosts = {"qkv": polyq.HostLayer.pack(np.vstack([W["q"][0], W["k"][0], W["v"][0]]),
+                                                 a_in["q"], args.budget),
+                     "o": polyq.HostLayer.pack(W["o"][0], a_in["o"], args.budget),
+                     "gu": polyq.HostLayer.pack(np.vstack([W["gate"][0], W["up"][0]]),
+                                                a_in["gate"], args.budget),
+                     "down": polyq.HostLayer.pack(W["down"][0], a_in["down"], args.budget)}
+            p_o = hosts["o"].export()["perm"]
+            p_d = hosts["down"].export()["perm"]
+            hosts["qkv"].permute_rows(np.concatenate([np.arange(2 * hidden), 2 * hidden + p_o]))
+            hosts["gu"].permute_rows(np.concatenate([p_d, ffn + p_d]))
+            names = list(hosts)
+        base = {n: polyq.DeviceLayer(hosts[n], device, identity_gather=n in ("o", "down"))
+                for n in names}
+        stack = [base] + [{n: base[n].clone() for n in names} for _ in range(L - 1)]
+        step_bytes = L * sum(base[n].info["packed_bytes"] + base[n].info["meta_bytes"]
+                             for n in names)
+        s = torch.zeros((1, hidden), dtype=torch.float32, device=device)
+        s0 = torch.from_numpy(np.random.default_rng(5).standard_normal((1, hidden))
+                              .astype(np.float32)).to(device)
+        if mode == "separate":
+            q, k, v = (torch.empty((1, hidden), dtype=torch.float32, device=device)
+                       for _ in range(3))
+            g, u = (torch.empty((1, ffn), dtype=torch.float32, device=device) for _ in range(2))
+            wsb = torch.zeros(max(polyq.gemv_group_workspace_bytes(
+                [base["gate"], base["up"]], 1), 1 << 20), dtype=torch.uint8, device=device)
+        else:
+            yqkv = torch.empty((1, 3 * hidden), dtype=torch.float32, device=device)
+            ygu = torch.empty((1, 2 * ffn), dtype=torch.float32, device=device)
+            wsb = torch.zeros(max(polyq.gemv_group_workspace_bytes([base["gu"]], 1), 1 << 20),
+                              dtype=torch.uint8, device=device)
+
+        def run_step():
+            for lay in stack:
+                if mode == "separate":
+                    polyq.linear_gemv_input([lay["q"], lay["k"], lay["v"]], polyq.X_RMSNORM, s,
+                                            ys=[q, k, v], workspace=wsb, stream=stream)
+                    polyq.linear_gemv_input([lay["o"]], polyq.X_F32, v, ys=[s], residuals=[s],
+                                            workspace=wsb, stream=stream)
+                    polyq.linear_gemv_input([lay["gate"], lay["up"]], polyq.X_RMSNORM, s,
+                                            ys=[g, u], workspace=wsb, stream=stream)
+                    polyq.linear_gemv_input([lay["down"]], polyq.X_SILU_MUL, g, b=u, ys=[s],
+                                            residuals=[s], workspace=wsb, stream=stream)
+                else:
+                    polyq.linear_gemv_input([lay["qkv"]], polyq.X_RMSNORM, s, ys=[yqkv],
+                                            workspace=wsb, stream=stream)
+                    polyq.linear_gemv_input([lay["o"]], polyq.X_F32, yqkv[:, 2 * hidden:],
+                                            ys=[s], residuals=[s], workspace=wsb, stream=stream)
+                    polyq.linear_gemv_input([lay["gu"]], polyq.X_RMSNORM, s, ys=[ygu],
+                                            workspace=wsb, stream=stream)
+                    polyq.linear_gemv_input([lay["down"]], polyq.X_SILU_MUL, ygu[:, :ffn],
+                                            b=ygu[:, ffn:], ys=[s], residuals=[s],
+                                            workspace=wsb, stream=stream)
+
+        with torch.cuda.stream(stream):
+            s.copy_(s0)
+            run_step()
+        stream.synchronize()
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=stream):
+            s.copy_(s0)  # every token starts from the same stream state
+            run_step()
+        reps = max(3, args.decode_steps)
+        with torch.cuda.stream(stream):
+            for _ in range(3):
+                graph.replay()
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for _ in range(reps):
+                graph.replay()
+            e1.record(stream)
+        stream.synchronize()
+        ms = e0.elapsed_time(e1) / reps
+        finite = bool(torch.isfinite(s).all())
+        tbs = step_bytes / (ms * 1e-3) / 1e12
+        gathered[mode] = (5 * hidden if mode == "separate" else 2 * hidden)
+        out[mode] = {"ms_per_token": round(ms, 4), "packed_bytes_per_token": step_bytes,
+                     "TB/s": round(tbs, 4), "frac_of_hbm": round(tbs * 1e3 / hbm, 4),
+                     "kernel_launches_per_token": 8 * L, "stream_finite": finite}
+        del stack, base, hosts
+        torch.cuda.empty_cache()
+    # §5.3 model of activation-reorder traffic per token (A16 read + write of
+    # each explicit shuffle): without merges every linear shuffles its input
+    no_merge = 4 * L * sum(k for _, _, k in LLAMA)
+    for mode in out:
+        kept = 4 * L * gathered[mode]
+        out[mode]["reorder_traffic_mib"] = round(kept / 2 ** 20, 3)
+        out[mode]["reorder_traffic_removed"] = round(1 - kept / no_merge, 4)
+    out["reorder_traffic_no_merge_mib"] = round(no_merge / 2 ** 20, 3)
+    out["workload"] = (f"llama2-13b decode step, {L} layers (device copies of one packed "
+                       f"layer set), batch 1, B={args.budget}, position 0")
+    return out
 
 
 def bench_gemm(polyq, synth, torch, device, stream, args, tf_burst, tf_sus):
@@ -461,6 +588,9 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-gemm", action="store_true")
+    ap.add_argument("--no-decode", action="store_true")
+    ap.add_argument("--decode-layers", type=int, default=40)
+    ap.add_argument("--decode-steps", type=int, default=20)
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

@@ -446,6 +446,17 @@ def silu(v):
     return v / (1.0 + np.exp(-v))
 
 
+def row_slice(layer, r0, r1):
+    """Rows [r0, r1) of a packed layer as a layer of their own (same channel
+    permutation and blocks): a jointly allocated stack of linears, split."""
+    out = dict(layer)
+    out["packed"] = layer["packed"][r0:r1].copy()
+    out["meta"] = layer["meta"][r0:r1].copy()
+    out["out_perm"] = np.arange(r1 - r0, dtype=np.int64)
+    out["N"] = r1 - r0
+    return out
+
+
 def merge_decoder_layer(lin):
     """Apply the §4.3 merges of one decoder layer (reading R11): v emits in
     o's input basis and gate/up emit in down's, so o and down read their

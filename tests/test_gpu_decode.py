@@ -143,3 +143,64 @@ def test_two_layer_decode_step(polyq_lib):
     got = s.cpu().numpy().astype(np.float64)
     rel = np.linalg.norm(got - s_ref) / np.linalg.norm(s_ref)
     assert rel <= 1e-2, rel
+
+
+def test_grouped_decode_layer(polyq_lib):
+    # q/k/v and gate/up each allocated jointly over their stacked rows (one
+    # permutation per group), v rows merged into o's basis, gate/up rows into
+    # down's; the library runs four calls, the oracle the same layer split
+    hidden, ffn = 256, 640
+    W = {}
+    for i, (name, N, K) in enumerate(O.llama_layer_linears(hidden, ffn)):
+        W[name] = synth.layer_weights(N, K, synth.seed_for(6, i))
+    Wqkv = np.vstack([W["q"][0], W["k"][0], W["v"][0]])
+    Wgu = np.vstack([W["gate"][0], W["up"][0]])
+    aq, ag = W["q"][1], W["gate"][1]
+    h_qkv, r_qkv = polyq_lib.HostLayer.pack(Wqkv, aq, 3.0), O.pack_layer(Wqkv, aq, 3.0)
+    h_gu, r_gu = polyq_lib.HostLayer.pack(Wgu, ag, 3.0), O.pack_layer(Wgu, ag, 3.0)
+    h_o, r_o = polyq_lib.HostLayer.pack(*W["o"], 3.0), O.pack_layer(*W["o"], 3.0)
+    h_d, r_d = polyq_lib.HostLayer.pack(*W["down"], 3.0), O.pack_layer(*W["down"], 3.0)
+    p_o, p_d = r_o["perm"], r_d["perm"]
+    rp_qkv = np.concatenate([np.arange(2 * hidden), 2 * hidden + p_o])
+    rp_gu = np.concatenate([p_d, ffn + p_d])
+    h_qkv.permute_rows(rp_qkv)
+    h_gu.permute_rows(rp_gu)
+    r_qkv = O.permute_rows(r_qkv, rp_qkv)
+    r_gu = O.permute_rows(r_gu, rp_gu)
+    merged = {"q": (O.row_slice(r_qkv, 0, hidden), r_qkv["perm"]),
+              "k": (O.row_slice(r_qkv, hidden, 2 * hidden), r_qkv["perm"]),
+              "v": (O.row_slice(r_qkv, 2 * hidden, 3 * hidden), r_qkv["perm"]),
+              "o": (r_o, None),
+              "gate": (O.row_slice(r_gu, 0, ffn), r_gu["perm"]),
+              "up": (O.row_slice(r_gu, ffn, 2 * ffn), r_gu["perm"]),
+              "down": (r_d, None)}
+    d_qkv = polyq_lib.DeviceLayer(h_qkv, "cuda")
+    d_gu = polyq_lib.DeviceLayer(h_gu, "cuda")
+    d_o = polyq_lib.DeviceLayer(h_o, "cuda", identity_gather=True)
+    d_d = polyq_lib.DeviceLayer(h_d, "cuda", identity_gather=True)
+
+    s0 = np.random.default_rng(6).standard_normal((1, hidden)).astype(np.float32)
+    s = torch.from_numpy(s0).cuda()
+    h = torch.empty((1, hidden), dtype=torch.bfloat16, device="cuda")
+    yqkv, = polyq_lib.linear_gemv_input([d_qkv], polyq_lib.X_RMSNORM, s, x_out=h)
+    xo = torch.empty((1, hidden), dtype=torch.bfloat16, device="cuda")
+    polyq_lib.linear_gemv_input([d_o], polyq_lib.X_F32, yqkv[:, 2 * hidden:], ys=[s],
+                                residuals=[s], x_out=xo)
+    h2 = torch.empty((1, hidden), dtype=torch.bfloat16, device="cuda")
+    ygu, = polyq_lib.linear_gemv_input([d_gu], polyq_lib.X_RMSNORM, s, x_out=h2)
+    xd = torch.empty((1, ffn), dtype=torch.bfloat16, device="cuda")
+    polyq_lib.linear_gemv_input([d_d], polyq_lib.X_SILU_MUL, ygu[:, :ffn], b=ygu[:, ffn:],
+                                ys=[s], residuals=[s], x_out=xd)
+    torch.cuda.synchronize()
+    hx, h2x = _bf16_vals(_bf16_bits(h)), _bf16_vals(_bf16_bits(h2))
+    y = yqkv.cpu().numpy()
+    for name, sl in (("q", slice(0, hidden)), ("k", slice(hidden, 2 * hidden)),
+                     ("v", slice(2 * hidden, 3 * hidden))):
+        L, gat = merged[name]
+        check_tolerance(y[:, sl], O.linear(L, hx, gather=gat), hx, hidden)
+    g = ygu.cpu().numpy()
+    check_tolerance(g[:, :ffn], O.linear(*merged["gate"][:1], h2x, gather=merged["gate"][1]),
+                    h2x, hidden)
+    s_ref, _ = O.decode_layer(s0.astype(np.float64), merged)
+    got = s.cpu().numpy().astype(np.float64)
+    assert np.linalg.norm(got - s_ref) / np.linalg.norm(s_ref) <= 1e-2

@@ -492,3 +492,14 @@ def test_decoder_layer_matches_dense_graph():
     u = h2 @ Wd["up"].T
     ref = s1 + bf16(g / (1 + np.exp(-g)) * u) @ Wd["down"].T
     assert np.allclose(out, ref, rtol=1e-12, atol=1e-12)
+
+
+def test_row_slice_of_stacked_layer():
+    # a stack allocated jointly, split by rows, multiplies like the stack
+    W1, a = synth.layer_weights(40, 96, 320)
+    W2, _ = synth.layer_weights(24, 96, 321)
+    Ls = O.pack_layer(np.vstack([W1, W2]), a, 3.0)
+    x = np.random.default_rng(3).standard_normal((2, 96))
+    y = O.linear(Ls, x)
+    assert np.array_equal(O.linear(O.row_slice(Ls, 0, 40), x), y[:, :40])
+    assert np.array_equal(O.linear(O.row_slice(Ls, 40, 64), x), y[:, 40:])
