@@ -264,19 +264,41 @@ __device__ __forceinline__ SlotGeom slot_geom(int bits, int warp, int lane, int 
   }
 }
 
-// A record is built once per call by the consumer warps of one CTA.
-// Pass 1: the gather indices (static layer data, so this may run before the
-// grid-dependency wait).
+// Where a record's activations come from: the layer's input (bf16 x, or the
+// fp32 inputs of a fused transform), its gather vector and its width K.
+struct XIn {
+  const __nv_bfloat16* x;
+  const float* xa;
+  const float* xb;
+  uint16_t* xout;  // written when not NULL
+  const int32_t* gather;
+  int kind, K, batch;
+};
+
+__device__ __forceinline__ XIn xin_of(const GvParams& P, int l) {
+  XIn in;
+  in.x = layer_x(P, l);
+  in.xa = P.xa;
+  in.xb = P.xb;
+  in.xout = l == 0 ? P.xout : nullptr;  // layer 0's records cover every source element
+  in.gather = layer_gather(P, l);
+  in.kind = P.xkind;
+  in.K = layer_K(P, l);
+  in.batch = P.batch;
+  return in;
+}
+
+// Pass 1 of a record: the gather indices (static layer data, so this may run
+// before the grid-dependency wait).
 template <int NB>
-__device__ __forceinline__ void rec_sources(const GvParams& P, const GvBlock& B, int l, int j,
-                                            int warp, int lane, const uint32_t* p3,
-                                            int (&src)[2][2]) {
-  const int32_t* gather = layer_gather(P, l);
+__device__ __forceinline__ void rec_sources(const XIn& in, const GvBlock& B, int j, int warp,
+                                            int lane, const uint32_t* p3, int (&src)[2][2]) {
+  const int32_t* gather = in.gather;
 #pragma unroll
   for (int s = 0; s < 2; ++s) {
     src[s][0] = src[s][1] = -1;
     const SlotGeom g = slot_geom<NB>(B.bits, warp, lane, threadIdx.x, s, j, p3);
-    if (g.valid && g.bb < P.batch) {
+    if (g.valid && g.bb < in.batch) {
 #pragma unroll
       for (int h = 0; h < 2; ++h)
         if (g.ch[h] < B.n_ch) {
@@ -290,15 +312,14 @@ __device__ __forceinline__ void rec_sources(const GvParams& P, const GvBlock& B,
 // Passes 2 and 3: load the activations, scale, round to fp16, store the
 // pairs and (b < 16) the per-chunk sums C1 = 1024 * sum x' and X = sum x.
 template <int NB>
-__device__ __forceinline__ void rec_build(const GvParams& P, const GvBlock& B, int l, int j,
-                                          int warp, int lane, const uint32_t* p3,
-                                          const int (&src)[2][2], const float* rnorm,
-                                          uint32_t* rec) {
+__device__ __forceinline__ void rec_build(const XIn& in, const GvBlock& B, int j, int warp,
+                                          int lane, const uint32_t* p3, const int (&src)[2][2],
+                                          const float* rnorm, uint32_t* rec) {
   constexpr int LW = rec_lane_words(NB);
   constexpr int PW = rec_pair_words(NB);
   constexpr int NGM = 8 / NB;
-  const __nv_bfloat16* x = layer_x(P, l);
-  const int K = layer_K(P, l);
+  const __nv_bfloat16* x = in.x;
+  const int K = in.K;
   float xv[2][2];
 #pragma unroll
   for (int s = 0; s < 2; ++s) {
@@ -311,18 +332,17 @@ __device__ __forceinline__ void rec_build(const GvParams& P, const GvBlock& B, i
       }
       const size_t o = (size_t)g.bb * K + src[s][h];
       __nv_bfloat16 v;
-      switch (P.xkind) {
-        case POLYQ_X_F32: v = __float2bfloat16_rn(P.xa[o]); break;
-        case POLYQ_X_RMSNORM: v = __float2bfloat16_rn(P.xa[o] * rnorm[g.bb]); break;
+      switch (in.kind) {
+        case POLYQ_X_F32: v = __float2bfloat16_rn(in.xa[o]); break;
+        case POLYQ_X_RMSNORM: v = __float2bfloat16_rn(in.xa[o] * rnorm[g.bb]); break;
         case POLYQ_X_SILU_MUL: {
-          const float a = P.xa[o];
-          v = __float2bfloat16_rn(a / (1.f + expf(-a)) * P.xb[o]);
+          const float a = in.xa[o];
+          v = __float2bfloat16_rn(a / (1.f + expf(-a)) * in.xb[o]);
           break;
         }
         default: v = x[o]; break;
       }
-      // layer 0's records cover every source element once
-      if (P.xout && l == 0) P.xout[o] = __bfloat16_as_ushort(v);
+      if (in.xout) in.xout[o] = __bfloat16_as_ushort(v);
       xv[s][h] = __bfloat162float(v);
     }
   }
@@ -425,7 +445,7 @@ __device__ __forceinline__ void load_words(uint32_t* w, const uint8_t* codes, in
 // One step of a b<16 block for this warp's 16 rows; adds the chunk results,
 // scaled, into acc[row][batch].
 template <int NB, int BITS>
-__device__ __forceinline__ void step_mma(const GvParams& P, int uvalid, int g0,
+__device__ __forceinline__ void step_mma(uint32_t magic, int batch, int uvalid, int g0,
                                          const uint8_t* stage, const uint32_t* rec,
                                          const uint32_t* zeros, int warp, int lane,
                                          float (&acc)[2][NB]) {
@@ -443,7 +463,6 @@ __device__ __forceinline__ void step_mma(const GvParams& P, int uvalid, int g0,
   const int g = lane >> 2, t = lane & 3;
   const int rA = warp * 16 + g, rB = rA + 8;
   const uint32_t* meta_s = reinterpret_cast<const uint32_t*>(stage + kCodesBytes);
-  const uint32_t magic = P.magic;
 
   uint32_t wa[NW], wb[NW];
   load_words<BITS, NB>(wa, stage, rA, t);
@@ -453,7 +472,7 @@ __device__ __forceinline__ void step_mma(const GvParams& P, int uvalid, int g0,
   // box h belong to chunk c_t + h*CPB, so only a matching lane loads its
   // activations, the others read zeros.
   const int my_b = g / NGS, my_c = g % NGS;
-  const int dc = my_b < P.batch ? my_c - lane_unit(BITS, NB, t, 0) / 64 : -1000;
+  const int dc = my_b < batch ? my_c - lane_unit(BITS, NB, t, 0) / 64 : -1000;
   const uint32_t* brow = rec + (my_b * 4 + t) * LW;
 
   float d[4][4];
@@ -492,7 +511,7 @@ __device__ __forceinline__ void step_mma(const GvParams& P, int uvalid, int g0,
   for (int cc = 0; cc < 2; ++cc) {
     const int col = 2 * t + cc;
     const int be = col / NGS, c = col % NGS;
-    if (be < P.batch) {
+    if (be < batch) {
       const float C1 = recf[PW + be * NGM + c];
       const float X = recf[PW + NB * NGM + be * NGM + c];
 #pragma unroll
@@ -513,7 +532,7 @@ __device__ __forceinline__ void step_mma(const GvParams& P, int uvalid, int g0,
 // n of B is batch row n.  Lane t holds weights [16t, 16t+16) of each of the
 // two 64-weight boxes.
 template <int NB>
-__device__ __forceinline__ void step_16(const GvParams& P, int uvalid,
+__device__ __forceinline__ void step_16(int batch, int uvalid,
                                         const uint8_t* stage, const uint32_t* rec,
                                         const uint32_t* zeros, int warp, int lane,
                                         float (&acc)[2][NB]) {
@@ -522,7 +541,7 @@ __device__ __forceinline__ void step_16(const GvParams& P, int uvalid,
   static_assert(box_pitch(16, NB) == PITCH && nbox_of(16, NB) == 2, "16-bit geometry");
   const int g = lane >> 2, t = lane & 3;
   const int rA = warp * 16 + g, rB = rA + 8;
-  const uint32_t* bsrc = g < P.batch ? rec + (g * 4 + t) * LW : zeros;
+  const uint32_t* bsrc = g < batch ? rec + (g * 4 + t) * LW : zeros;
   float d[2][4];
 #pragma unroll
   for (int q = 0; q < 2; ++q) d[q][0] = d[q][1] = d[q][2] = d[q][3] = 0.f;
@@ -581,7 +600,8 @@ __global__ void __launch_bounds__(kConsumers) gemv_prep(const __grid_constant__ 
   int l, bi, j;
   rec_pos(S, P.n_layers, r, &l, &bi, &j);
   int src[2][2];
-  rec_sources<NB>(P, S.blk[l][bi], l, j, warp, lane, s_p3, src);  // static layer data
+  const XIn in = xin_of(P, l);
+  rec_sources<NB>(in, S.blk[l][bi], j, warp, lane, s_p3, src);  // static layer data
   pdl_wait();  // x comes from the previous kernel; the records and y may still be in use
   __shared__ float s_rnorm[4];
   if (P.xkind == POLYQ_X_RMSNORM) {
@@ -606,7 +626,7 @@ __global__ void __launch_bounds__(kConsumers) gemv_prep(const __grid_constant__ 
     }
     __syncthreads();
   }
-  rec_build<NB>(P, S.blk[l][bi], l, j, warp, lane, s_p3, src, s_rnorm,
+  rec_build<NB>(in, S.blk[l][bi], j, warp, lane, s_p3, src, s_rnorm,
                 reinterpret_cast<uint32_t*>(P.rec + (size_t)r * rec_bytes(NB)));
   // y starts as the residual (or zero); the main kernel adds its pieces
 #pragma unroll
@@ -756,11 +776,11 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) gemv_main(const __grid_c
     const int bits = (int)(desc.x & 0xFFu);
     const int uvalid = (int)(desc.y & 0xFFFFu), g0 = (int)(desc.y >> 16);
     switch (bits) {
-      case 2: step_mma<NB, 2>(P, uvalid, g0, stage, rec, zeros, warp, lane, acc); break;
-      case 3: step_mma<NB, 3>(P, uvalid, g0, stage, rec, zeros, warp, lane, acc); break;
-      case 4: step_mma<NB, 4>(P, uvalid, g0, stage, rec, zeros, warp, lane, acc); break;
-      case 8: step_mma<NB, 8>(P, uvalid, g0, stage, rec, zeros, warp, lane, acc); break;
-      default: step_16<NB>(P, uvalid, stage, rec, zeros, warp, lane, acc); break;
+      case 2: step_mma<NB, 2>(P.magic, P.batch, uvalid, g0, stage, rec, zeros, warp, lane, acc); break;
+      case 3: step_mma<NB, 3>(P.magic, P.batch, uvalid, g0, stage, rec, zeros, warp, lane, acc); break;
+      case 4: step_mma<NB, 4>(P.magic, P.batch, uvalid, g0, stage, rec, zeros, warp, lane, acc); break;
+      case 8: step_mma<NB, 8>(P.magic, P.batch, uvalid, g0, stage, rec, zeros, warp, lane, acc); break;
+      default: step_16<NB>(P.batch, uvalid, stage, rec, zeros, warp, lane, acc); break;
     }
     __syncwarp();
     if (lane == 0) mbar_arrive(empty0 + 8 * slot);
