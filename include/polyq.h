@@ -65,6 +65,18 @@ extern "C" {
 #define POLYQ_ALLOC_WATERFILL 0 /* Section 3.2 max-heap waterfilling (default) */
 #define POLYQ_ALLOC_LADDER 1    /* descending saliency, each channel climbs */
 
+/* Section 3.1 error proxy E_b[k] that drives the allocation. */
+#define POLYQ_PROXY_SALIENCY 0 /* (a_k * ||W[:,k]||_2 / (2^b - 1))^2, E_16 = 0 */
+#define POLYQ_PROXY_QUANT 1    /* ||Q_b(W)[:,k] - W[:,k]||^2 * E[x_k^2], E_16 = 0:
+                                  the whole layer quantised at width b with groups
+                                  of 64 consecutive original channels; the sum
+                                  over rows in row order, fp64 */
+
+/* Default channel quanta of the Section 3.3 quanta matching, widths
+ * 2,3,4,8,16: one quantum of each width fills a whole number of 16-byte
+ * chunks, so blocks of these sizes need no segment padding. */
+#define POLYQ_GPU_QUANTA {64, 128, 32, 16, 8}
+
 /* Options of polyq_pack.  Zero-initialise, then set what you need;
  * polyq_pack_opts_default() gives the defaults. */
 typedef struct {
@@ -72,10 +84,48 @@ typedef struct {
   uint32_t palette_mask;     /* bit b set: width b allowed (b in 2,3,4,8,16);
                                 0 means all five */
   int32_t alloc_rule;        /* POLYQ_ALLOC_WATERFILL or POLYQ_ALLOC_LADDER */
-  int32_t snap_quanta;       /* must be 0 (quanta matching not built) */
+  int32_t snap_quanta;       /* 1: Section 3.3 quanta matching (below) */
   int32_t n_threads;         /* host threads, 0 = hardware concurrency */
-  const uint8_t* forced_bits;/* optional [K] width map; skips allocation */
+  const uint8_t* forced_bits;/* optional [K] width map; skips allocation
+                                (and then snap_quanta must be 0) */
+  int32_t proxy;             /* POLYQ_PROXY_SALIENCY (default) or
+                                POLYQ_PROXY_QUANT; POLYQ_ALLOC_LADDER needs
+                                the saliency proxy */
+  int32_t act_scaling;       /* 1: Section 3.4 bit-specific activation-aware
+                                scaling (below) */
+  int32_t quanta[5];         /* channels per quantum for widths 2,3,4,8,16
+                                (each > 0), or all 0 for POLYQ_GPU_QUANTA */
+  const float* act_sqmean;   /* [K] E[x_k^2] for POLYQ_PROXY_QUANT and the
+                                scaling search; NULL = act_absmean[k]^2 */
 } polyq_pack_opts;
+/* Quanta matching (snap_quanta = 1), Section 3.3, after the allocation:
+ *  1. target counts: for each palette width b the candidates are the
+ *     multiples q_b*(floor(c_b/q_b)+d), d in {-1,0,1,2}, inside [0,K]; of the
+ *     combinations summing to K the one with the smallest
+ *     |sum b*count - round(B*K)| is taken, then the one closest to the
+ *     allocation's counts (sum of |differences|), then the lexicographically
+ *     smallest count vector (widths ascending).  If no combination sums to K,
+ *     the narrowest width takes K minus the others' counts.
+ *  2. reassignment between neighbouring widths: with f_i the net number of
+ *     channels that must cross from widths <= w_i to widths > w_i, upward
+ *     crossings are made from the lowest boundary up, each promoting the
+ *     channels of width w_i with the largest gain per bit
+ *     (E_{w_i} - E_{w_i+1}) / (w_{i+1} - w_i) (ties: lower channel first),
+ *     then downward crossings from the top boundary down, each demoting the
+ *     channels of width w_{i+1} with the smallest gain (ties: higher channel
+ *     first).
+ * Activation-aware scaling (act_scaling = 1), Section 3.4, on the final map:
+ * m_k = a_k / mean(a) (a = act_absmean, mean summed in channel order); for
+ * each width b present the exponent alpha_b in {0, 0.1, ..., 1} (j/10) that
+ * minimises the mean over the block's channels of
+ * ||Q_b(W/t)[:,k]*t_k - W[:,k]||^2 * E[x_k^2] with t_k = fp32_rn(m_k^-alpha_b),
+ * evaluated with the block's own groups (ties: the smaller alpha; an alpha
+ * giving a non-finite or non-positive t_k or |W/t| > 65504 is skipped; for
+ * b = 16 alpha is 0).  The block is then packed from W/t (one fp64 division
+ * per weight) and the layer carries the activation factor t at each
+ * clustered position (polyq_layer_xscale): the GEMV and GEMM multiply the
+ * gathered activation by it, so the layer still computes y = x W'^T with
+ * W' = Q(W/t) * t. */
 
 /* One bit-homogeneous block (Section 4.2). */
 typedef struct {
@@ -100,6 +150,10 @@ typedef struct {
   int64_t meta_bytes;    /* N * n_groups * 4 */
   int64_t meta_stride;   /* device meta row stride in entries: n_groups
                             rounded up to a multiple of 4 (16-byte rows) */
+  int64_t pad_bytes;     /* segment padding bytes in one packed row */
+  double alpha[5];       /* Section 3.4 exponent of widths 2,3,4,8,16; -1 where
+                            the width is absent or the layer is not scaled */
+  int32_t has_xscale;    /* 1 when the layer carries activation factors */
 } polyq_info;
 
 /* A packed layer resident on the device.  Filled by polyq_dev_layer_fill()
@@ -114,6 +168,10 @@ typedef struct {
   int64_t meta_stride;    /* entries per meta row, multiple of 4, >= n_groups */
   int32_t n_blocks;
   polyq_block blocks[POLYQ_MAX_BLOCKS];
+  const float* xscale;    /* device fp32 [K], 16-byte aligned: Section 3.4
+                             activation factor at each clustered position,
+                             xs[p] = x[gather[p]] * xscale[p]; NULL = none
+                             (polyq_dev_layer_fill leaves it NULL) */
 } polyq_dev_layer;
 
 typedef struct polyq_layer polyq_layer; /* opaque host-side packed layer */
@@ -121,14 +179,19 @@ typedef struct polyq_layer polyq_layer; /* opaque host-side packed layer */
 const char* polyq_last_error(void);
 void polyq_pack_opts_default(polyq_pack_opts* opts);
 
-/* Allocate widths, cluster and pack one layer (Sections 3.1, 3.2, 4.1, 4.2).
+/* Allocate widths, cluster and pack one layer (Sections 3.1 to 3.4, 4.1,
+ * 4.2).
  * W: host fp32 [N][K] row-major (out x in), finite, |W| <= 65504.
- * act_absmean: host fp32 [K], per-input-channel activation magnitude used for
- * the saliency a_k * ||W[:,k]||_2 (Section 3.1 error proxy, E_16 = 0).
+ * act_absmean: host fp32 [K], per-input-channel activation magnitude: the
+ * saliency a_k * ||W[:,k]||_2 of the saliency proxy, the default E[x_k^2]
+ * (its square) and the metric m of the Section 3.4 scaling.  Needed unless
+ * forced_bits is given without act_scaling.
  * budget_bits: average width B in [2, 16] (Section 3.2).
  * Greedy waterfilling: all channels start at the narrowest palette width,
  * Delta = round(B*K) - b_min*K, upgrades popped from a max-heap by gain per
- * extra bit (ties: lower channel first); a step that does not fit is dropped.
+ * extra bit (E_b - E_b')/(b' - b) of the chosen proxy (ties: lower channel
+ * first); a step that does not fit is dropped.  Then, as the options ask,
+ * quanta matching and activation-aware scaling (see polyq_pack_opts).
  * On success *out owns a new layer (free with polyq_free). */
 int polyq_pack(const float* W, int64_t N, int64_t K, const float* act_absmean,
                double budget_bits, const polyq_pack_opts* opts,
@@ -148,6 +211,12 @@ int polyq_layer_info(const polyq_layer* layer, polyq_info* out);
 int polyq_layer_export(const polyq_layer* layer, uint8_t* packed,
                        uint32_t* meta, int64_t meta_stride, int32_t* perm,
                        uint8_t* bits, int32_t* out_perm);
+
+/* Section 3.4 activation factors of a scaled layer (act_scaling = 1):
+ * xscale [K] floats, xscale[p] = t at clustered position p (all 1.0 for a
+ * layer packed without scaling).  Upload them and set
+ * polyq_dev_layer.xscale; a scaled layer gives wrong results without them. */
+int polyq_layer_xscale(const polyq_layer* layer, float* xscale);
 
 /* Section 4.3 merge, producer side: permute whole output rows (packed bytes
  * and meta) so that afterwards the layer emits

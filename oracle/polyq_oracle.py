@@ -47,10 +47,40 @@ R5 packing: per (row, block) an LSB-first bitstream (code p at bits
    as two fp16, groups ordered by block then position.
 R6 merge: a producer basis beta means emitted[i] = y_orig[beta[i]]; the
    consumer gather is r = beta^-1 o P_c, i.e. xs[p] = x_emitted[r[p]].
+R13 quanta targets (§3.3): for each palette width b the candidates are the
+   multiples q_b*(floor(c_b/q_b)+d), d in {-1,0,1,2}, inside [0, K]; among
+   the combinations that sum to K, take the smallest |sum b*c^_b -
+   round(B*K)|, then the smallest sum |c^_b - c_b|, then the
+   lexicographically smallest count vector (widths ascending).  When no
+   combination sums to K (K not a multiple of the quanta's gcd, or the window
+   is too narrow), the narrowest width takes K minus the others' counts.
+R14 reassignment (§3.3): moves only between neighbouring palette widths.  The
+   net flow across boundary i (between widths w_i < w_{i+1}) is f_i =
+   sum_{j<=i} (c_j - c^_j).  Upward flows are applied boundary by boundary
+   from the bottom, each promoting the f_i channels of width w_i with the
+   largest gain G_{w_i->w_{i+1}} (ties: lower index); then downward flows from
+   the top, each demoting the |f_i| channels of width w_{i+1} with the
+   smallest gain (ties: higher index).
+R15 quantiser-in-the-loop proxy (§3.1, Eq. for E_b[j]): E_b[k] =
+   sum_n (Q_b(W)[n,k] - W[n,k])^2 * E[x_k^2] with Q_b the R1 quantiser applied
+   to the whole layer at width b, groups = 64 consecutive original channels of
+   a row; E_16 = 0.  The sum over n runs in row order in fp64.
+R16 bit-specific scaling (§3.4): m_k = a_k / mean(a) (a = the activation
+   magnitude, mean summed in channel order) and, for the channels of width b,
+   the activation factor t_k = fp32_rn(m_k^-alpha_b), i.e. s_k = 1/t_k.  A
+   block is quantised as Q_b(W / t) (one fp64 division per weight), so its
+   effective weight is Q_b(W/t) * t, and the layer multiplies its gathered
+   activation by t at each clustered position.  alpha_b is the grid value
+   j/10, j = 0..10, with the smallest mean of E_b over the block's channels,
+   evaluated with the block's own groups (64 consecutive clustered
+   positions); ties take the smaller alpha.  A value of alpha for which some
+   t_k is not finite and positive, or W/t leaves the fp16 range, is skipped
+   (alpha = 0 gives t = 1 and is always allowed).
 """
 from __future__ import annotations
 
 import heapq
+import itertools
 import math
 
 import numpy as np
@@ -500,3 +530,265 @@ def decode_layer(s, merged, eps=1e-6):
     xd = bf16_rn(silu(g) * u)
     s2 = s1 + _linear_g(merged["down"], xd)
     return s2, dict(h=h, q=q, k=k, v=v, xo=xo, s1=s1, h2=h2, gate=g, up=u, xd=xd)
+
+
+# ---------------------------------------------------------------------------
+# §3.1 full proxy (R15), §3.2 waterfilling on an error table, §3.3 quanta
+# matching (R13, R14), §3.4 bit-specific scaling (R16)
+# ---------------------------------------------------------------------------
+GPU_QUANTA = {2: 64, 3: 128, 4: 32, 8: 16, 16: 8}
+"""Channels per quantum: one quantum of each width is a whole number of
+16-byte chunks (64x2, 128x3, 32x4, 16x8 and 8x16 bits), so blocks whose sizes
+are multiples of these need no segment padding."""
+
+ALPHA_GRID = tuple(j / 10.0 for j in range(11))
+
+
+def saliency_error_table(sal, palette=PALETTE):
+    """E[b] = array over channels of the saliency proxy (R3)."""
+    return {b: np.array([proxy_error(float(v), b) for v in sal]) for b in palette}
+
+
+def _col_sq_err(Wq, W):
+    """sum_n (Wq[n,k] - W[n,k])^2 for each k, rows added in order, fp64."""
+    acc = np.zeros(W.shape[1], dtype=np.float64)
+    for n in range(W.shape[0]):
+        d = Wq[n] - W[n]
+        acc = acc + d * d
+    return acc
+
+
+def dequant_rows(Wb, b):
+    """Q_b applied to the columns of ``Wb`` (N x K_b, fp64) in groups of 64
+    consecutive columns (R1), dequantised: (q - z) * s, fp16(w) for b = 16."""
+    if b == 16:
+        return fp16_rn(Wb)
+    S, Z, Q = quantize_rows(Wb, b)
+    out = np.zeros_like(Wb)
+    for g in range(S.shape[1]):
+        cols = slice(g * GROUP, min((g + 1) * GROUP, Wb.shape[1]))
+        out[:, cols] = (Q[:, cols] - Z[:, g][:, None]) * S[:, g][:, None]
+    return out
+
+
+def quant_error_table(W, act_sqmean, palette=PALETTE):
+    """Quantiser-in-the-loop proxy (§3.1 channel-error equation, R15):
+    E[b][k] = ||Q_b(W)[:,k] - W[:,k]||^2 * E[x_k^2], the whole layer quantised
+    at width b with groups of 64 consecutive original channels; E[16] = 0."""
+    W = _check_weights(W).astype(np.float64)
+    x2 = np.asarray(act_sqmean, dtype=np.float64)
+    E = {}
+    for b in palette:
+        if b == 16:
+            E[b] = np.zeros(W.shape[1])
+        else:
+            E[b] = _col_sq_err(dequant_rows(W, b), W) * x2
+    return E
+
+
+def allocate_from_table(E, B, palette=PALETTE):
+    """§3.2 waterfilling with the gains of an error table: all channels start
+    at the narrowest width, Delta = round(B*K) - b_min*K, and the max-heap of
+    (gain per bit desc, channel asc) hands out upgrades to the next palette
+    width while they fit (a step that does not fit is dropped)."""
+    pal = tuple(sorted(palette))
+    K = len(E[pal[0]])
+    b_min = pal[0]
+    nxt = {pal[i]: pal[i + 1] for i in range(len(pal) - 1)}
+    bits = [b_min] * K
+    delta = residual_budget(B, K, b_min)
+    if delta <= 0 or len(pal) == 1:
+        return np.array(bits, dtype=np.int64)
+
+    def g(k, b, bn):
+        return (float(E[b][k]) - float(E[bn][k])) / float(bn - b)
+
+    heap = [(-g(k, b_min, nxt[b_min]), k, nxt[b_min]) for k in range(K)]
+    heapq.heapify(heap)
+    while delta > 0 and heap:
+        _, k, b_new = heapq.heappop(heap)
+        cost = b_new - bits[k]
+        if cost > delta:
+            continue
+        bits[k] = b_new
+        delta -= cost
+        if b_new in nxt:
+            heapq.heappush(heap, (-g(k, b_new, nxt[b_new]), k, nxt[b_new]))
+    return np.array(bits, dtype=np.int64)
+
+
+def quanta_targets(counts, quanta, B, K):
+    """§3.3 first step (R13): block sizes that are multiples of the quanta,
+    near the waterfilling counts, summing to K, budget kept closest to
+    round(B*K).  ``counts`` maps every palette width to its channel count."""
+    widths = sorted(counts)
+    T = int(math.floor(B * K + 0.5))
+    cand = []
+    for b in widths:
+        q = int(quanta[b])
+        base = int(counts[b]) // q
+        cand.append(sorted({q * (base + d) for d in (-1, 0, 1, 2) if 0 <= q * (base + d) <= K}))
+
+    def key(combo):
+        tb = sum(b * c for b, c in zip(widths, combo))
+        mv = sum(abs(c - int(counts[b])) for b, c in zip(widths, combo))
+        return (abs(tb - T), mv, tuple(combo))
+
+    best = None
+    for combo in itertools.product(*cand):
+        if sum(combo) != K:
+            continue
+        k = key(combo)
+        if best is None or k < best:
+            best = k
+    if best is None:
+        # the narrowest width fills the remainder
+        for rest in itertools.product(*cand[1:]):
+            c0 = K - sum(rest)
+            if c0 < 0:
+                continue
+            k = key((c0,) + tuple(rest))
+            if best is None or k < best:
+                best = k
+    return {b: int(c) for b, c in zip(widths, best[2])}
+
+
+def reassign_to_targets(bits, E, targets):
+    """§3.3 second step (R14): move channels between neighbouring widths until
+    the per-width counts equal ``targets``; promotions take the largest gain
+    per bit, demotions the smallest."""
+    bits = np.array(bits, dtype=np.int64)
+    pal = sorted(targets)
+    m = len(pal)
+    cur = [int(np.sum(bits == b)) for b in pal]
+    flow = []
+    acc = 0
+    for i in range(m - 1):
+        acc += cur[i] - int(targets[pal[i]])
+        flow.append(acc)
+
+    def g(k, i):
+        b, bn = pal[i], pal[i + 1]
+        return (float(E[b][k]) - float(E[bn][k])) / float(bn - b)
+
+    for i in range(m - 1):  # upward flows, bottom-up
+        if flow[i] > 0:
+            members = [k for k in range(len(bits)) if bits[k] == pal[i]]
+            members.sort(key=lambda k: (-g(k, i), k))
+            for k in members[:flow[i]]:
+                bits[k] = pal[i + 1]
+    for i in reversed(range(m - 1)):  # downward flows, top-down
+        if flow[i] < 0:
+            members = [k for k in range(len(bits)) if bits[k] == pal[i + 1]]
+            members.sort(key=lambda k: (g(k, i), -k))
+            for k in members[:-flow[i]]:
+                bits[k] = pal[i]
+    return bits
+
+
+def snap_to_quanta(bits, E, B, quanta=None, palette=PALETTE):
+    """Quanta matching (§3.3): R13 targets, then R14 reassignment."""
+    quanta = GPU_QUANTA if quanta is None else quanta
+    bits = np.asarray(bits, dtype=np.int64)
+    K = len(bits)
+    counts = {b: int(np.sum(bits == b)) for b in palette}
+    t = quanta_targets(counts, quanta, B, K)
+    return reassign_to_targets(bits, E, t)
+
+
+def padding_bytes_per_row(bits):
+    """Segment padding of one packed row: sum over blocks of the padded
+    segment bytes minus the bytes the codes need (R5)."""
+    bits = np.asarray(bits)
+    pad = 0
+    for b in PALETTE:
+        kb = int(np.sum(bits == b))
+        if kb:
+            raw = kb * 2 if b == 16 else (kb * b + 7) // 8
+            pad += seg_bytes(b, kb) - raw
+    return pad
+
+
+def act_metric(act_absmean):
+    """m_k = a_k / mean(a), the mean summed in channel order (R16)."""
+    a = np.asarray(act_absmean, dtype=np.float64)
+    tot = 0.0
+    for v in a:
+        tot = tot + float(v)
+    return a / (tot / len(a))
+
+
+def act_factor(m, alpha):
+    """t_k = fp32_rn(m_k^-alpha) (R16); None when some t_k is unusable."""
+    with np.errstate(divide="ignore", over="ignore", invalid="ignore"):
+        t = np.power(np.asarray(m, dtype=np.float64), -float(alpha))
+    t = t.astype(np.float32).astype(np.float64)
+    if not np.all(np.isfinite(t)) or np.any(t <= 0.0):
+        return None
+    return t
+
+
+def block_scaled_error(Wb, x2b, tb, b):
+    """Mean over the block's channels of ||Q_b(Wb/t)*t - Wb||^2 * E[x^2]
+    (R16), the block's groups being 64 consecutive clustered columns.  None
+    when Wb/t leaves the fp16 range."""
+    Ws = Wb / tb[None, :]
+    if np.max(np.abs(Ws)) > FP16_MAX:
+        return None
+    We = dequant_rows(Ws, b) * tb[None, :]
+    e = _col_sq_err(We, Wb) * x2b
+    tot = 0.0
+    for v in e:
+        tot = tot + float(v)
+    return tot / len(e)
+
+
+def choose_alphas(W, bits, act_absmean, act_sqmean, grid=ALPHA_GRID):
+    """§3.4 grid search (R16): per width present, the alpha with the smallest
+    mean scaled proxy error over the block; returns (alpha by width, t[K] in
+    original channel order)."""
+    W = _check_weights(W).astype(np.float64)
+    bits = np.asarray(bits, dtype=np.int64)
+    perm = cluster_perm(bits)
+    m = act_metric(act_absmean)
+    x2 = np.asarray(act_sqmean, dtype=np.float64)
+    t_all = np.ones(len(bits))
+    alphas = {}
+    for b in PALETTE:
+        idx = perm[bits[perm] == b]
+        if len(idx) == 0:
+            continue
+        if b == 16:
+            alphas[b] = 0.0  # E_16 = 0 for every alpha: the smallest wins
+            continue
+        best = None
+        for a in grid:
+            tb = act_factor(m[idx], a)
+            if tb is None:
+                continue
+            e = block_scaled_error(W[:, idx], x2[idx], tb, b)
+            if e is None:
+                continue
+            if best is None or e < best[0]:
+                best = (e, a, tb)
+        alphas[b] = best[1]
+        t_all[idx] = best[2]
+    return alphas, t_all
+
+
+def pack_layer_scaled(W, bits, t):
+    """Pack W / t (R16) with the width map ``bits``; the layer carries the
+    activation factors ``xscale`` in clustered order."""
+    W = _check_weights(W).astype(np.float64)
+    t = np.asarray(t, dtype=np.float64)
+    lay = pack_layer(W / t[None, :], None, 0.0, bits=bits)
+    lay["xscale"] = t[lay["perm"]]
+    return lay
+
+
+def linear_scaled(layer, x, gather=None):
+    """y[b][n'] = sum_p x[b][r[p]] * t[p] * W'[row(n')][p] (R16, fp64)."""
+    x = np.atleast_2d(np.asarray(x, dtype=np.float64))
+    r = layer["perm"] if gather is None else np.asarray(gather)
+    xs = x[:, r] * layer["xscale"][None, :]
+    return xs @ dequant(layer).T

@@ -74,6 +74,7 @@ struct GmParams {
   int has_meta;
   const __nv_bfloat16* x;
   const int32_t* gather;
+  const float* xscale;  // Section 3.4 activation factors (clustered order) or NULL
   __half* xg;
   float* y;
   int* status;
@@ -98,7 +99,8 @@ __host__ __device__ inline int slot_code(int bits, int s) {
 }
 
 // ---------------------------------------------------------------------------
-// pre-pass: Xg[m][kt*32 + s] = fp16(X[m][gather[pos0 + 32 h + slot_code(s)]])
+// pre-pass: Xg[m][kt*32 + s] = fp16(X[m][gather[p]] * xscale[p]) with
+// p = pos0 + 32 h + slot_code(s)
 // for the h-th 32-code half group of the block (tile kt); Y is zeroed when the
 // K range is split over CTAs
 // ---------------------------------------------------------------------------
@@ -141,6 +143,7 @@ __global__ void __launch_bounds__(256) gemm_prep(const __grid_constant__ GmParam
         const int p = B.pos0 + w;
         const int src = P.gather ? P.gather[p] : p;
         xv = __bfloat162float(P.x[(size_t)m * P.K + src]);
+        if (P.xscale) xv *= P.xscale[p];
       }
       v[h] = __float2half_rn(xv);
     }
@@ -555,6 +558,7 @@ extern "C" int polyq_linear_gemm(const polyq_dev_layer* L, const void* X, int64_
   P.units_n = (int)((L->N + BN - 1) / BN);
   P.x = (const __nv_bfloat16*)X;
   P.gather = L->gather;
+  P.xscale = L->xscale;
   P.xg = (__half*)workspace;
   P.y = Y;
   P.status = (int*)((uint8_t*)workspace + need - 256);

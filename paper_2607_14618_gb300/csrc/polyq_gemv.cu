@@ -2,7 +2,9 @@
 // the Section 4.2 bit blocks), one launch over all blocks of one or several
 // independent layers:
 //
-//   y[b][n] = residual[b][n] + sum_p x[b][gather[p]] * W'[n][p]
+//   y[b][n] = residual[b][n] + sum_p x[b][gather[p]] * t[p] * W'[n][p]
+//
+// (t = the Section 3.4 activation factors of a scaled layer, else 1.)
 //
 // Two kernels per call, chained with programmatic dependent launch:
 //  * gemv_prep, one CTA per (layer, step): gathers x through `gather`, scales
@@ -71,6 +73,7 @@ struct GvLayer {
   int rec0;   // first activation record of this layer (one per step)
   const __nv_bfloat16* x;
   const int32_t* gather;
+  const float* xscale;  // Section 3.4 activation factors or NULL
   float* y;
   const float* residual;
 };
@@ -180,6 +183,13 @@ __device__ __forceinline__ const int32_t* layer_gather(const GvParams& P, int l)
     if (q == l) g = P.L[q].gather;
   return g;
 }
+__device__ __forceinline__ const float* layer_xscale(const GvParams& P, int l) {
+  const float* f = P.L[0].xscale;
+#pragma unroll
+  for (int q = 1; q < POLYQ_MAX_GROUP; ++q)
+    if (q == l) f = P.L[q].xscale;
+  return f;
+}
 __device__ __forceinline__ int layer_K(const GvParams& P, int l) {
   int k = P.L[0].K;
 #pragma unroll
@@ -265,13 +275,15 @@ __device__ __forceinline__ SlotGeom slot_geom(int bits, int warp, int lane, int 
 }
 
 // Where a record's activations come from: the layer's input (bf16 x, or the
-// fp32 inputs of a fused transform), its gather vector and its width K.
+// fp32 inputs of a fused transform), its gather vector, its activation
+// factors and its width K.
 struct XIn {
   const __nv_bfloat16* x;
   const float* xa;
   const float* xb;
   uint16_t* xout;  // written when not NULL
   const int32_t* gather;
+  const float* xscale;
   int kind, K, batch;
 };
 
@@ -282,21 +294,24 @@ __device__ __forceinline__ XIn xin_of(const GvParams& P, int l) {
   in.xb = P.xb;
   in.xout = l == 0 ? P.xout : nullptr;  // layer 0's records cover every source element
   in.gather = layer_gather(P, l);
+  in.xscale = layer_xscale(P, l);
   in.kind = P.xkind;
   in.K = layer_K(P, l);
   in.batch = P.batch;
   return in;
 }
 
-// Pass 1 of a record: the gather indices (static layer data, so this may run
-// before the grid-dependency wait).
+// Pass 1 of a record: the gather indices and activation factors (static
+// layer data, so this may run before the grid-dependency wait).
 template <int NB>
 __device__ __forceinline__ void rec_sources(const XIn& in, const GvBlock& B, int j, int warp,
-                                            int lane, const uint32_t* p3, int (&src)[2][2]) {
+                                            int lane, const uint32_t* p3, int (&src)[2][2],
+                                            float (&fac)[2][2]) {
   const int32_t* gather = in.gather;
 #pragma unroll
   for (int s = 0; s < 2; ++s) {
     src[s][0] = src[s][1] = -1;
+    fac[s][0] = fac[s][1] = 1.f;
     const SlotGeom g = slot_geom<NB>(B.bits, warp, lane, threadIdx.x, s, j, p3);
     if (g.valid && g.bb < in.batch) {
 #pragma unroll
@@ -304,6 +319,7 @@ __device__ __forceinline__ void rec_sources(const XIn& in, const GvBlock& B, int
         if (g.ch[h] < B.n_ch) {
           const int p = B.pos0 + g.ch[h];
           src[s][h] = gather ? __ldg(gather + p) : p;
+          if (in.xscale) fac[s][h] = __ldg(in.xscale + p);
         }
     }
   }
@@ -314,7 +330,8 @@ __device__ __forceinline__ void rec_sources(const XIn& in, const GvBlock& B, int
 template <int NB>
 __device__ __forceinline__ void rec_build(const XIn& in, const GvBlock& B, int j, int warp,
                                           int lane, const uint32_t* p3, const int (&src)[2][2],
-                                          const float* rnorm, uint32_t* rec) {
+                                          const float (&fac)[2][2], const float* rnorm,
+                                          uint32_t* rec) {
   constexpr int LW = rec_lane_words(NB);
   constexpr int PW = rec_pair_words(NB);
   constexpr int NGM = 8 / NB;
@@ -343,7 +360,7 @@ __device__ __forceinline__ void rec_build(const XIn& in, const GvBlock& B, int j
         default: v = x[o]; break;
       }
       if (in.xout) in.xout[o] = __bfloat16_as_ushort(v);
-      xv[s][h] = __bfloat162float(v);
+      xv[s][h] = __bfloat162float(v) * fac[s][h];  // Section 3.4 factor (1 if none)
     }
   }
   float* recf = reinterpret_cast<float*>(rec);
@@ -600,8 +617,9 @@ __global__ void __launch_bounds__(kConsumers) gemv_prep(const __grid_constant__ 
   int l, bi, j;
   rec_pos(S, P.n_layers, r, &l, &bi, &j);
   int src[2][2];
+  float fac[2][2];
   const XIn in = xin_of(P, l);
-  rec_sources<NB>(in, S.blk[l][bi], j, warp, lane, s_p3, src);  // static layer data
+  rec_sources<NB>(in, S.blk[l][bi], j, warp, lane, s_p3, src, fac);  // static layer data
   pdl_wait();  // x comes from the previous kernel; the records and y may still be in use
   __shared__ float s_rnorm[4];
   if (P.xkind == POLYQ_X_RMSNORM) {
@@ -626,7 +644,7 @@ __global__ void __launch_bounds__(kConsumers) gemv_prep(const __grid_constant__ 
     }
     __syncthreads();
   }
-  rec_build<NB>(in, S.blk[l][bi], j, warp, lane, s_p3, src, s_rnorm,
+  rec_build<NB>(in, S.blk[l][bi], j, warp, lane, s_p3, src, fac, s_rnorm,
                 reinterpret_cast<uint32_t*>(P.rec + (size_t)r * rec_bytes(NB)));
   // y starts as the residual (or zero); the main kernel adds its pieces
 #pragma unroll
@@ -999,6 +1017,7 @@ int gemv_group(const char* who, const polyq_dev_layer* const* L, int n, const vo
     G.rec0 = recs;
     G.x = (const __nv_bfloat16*)xs[i];
     G.gather = D->gather;
+    G.xscale = D->xscale;
     G.y = ys[i];
     G.residual = res ? res[i] : nullptr;
     items += G.items;

@@ -1,6 +1,8 @@
-// Host side of the PolyQ library: width allocation (Section 3.2), clustering
-// permutation and bit blocks (Sections 4.1, 4.2), group quantisation and
-// packing, and the permutation merge rule (Section 4.3).
+// Host side of the PolyQ library: error proxies (Section 3.1), width
+// allocation (Section 3.2), quanta matching (Section 3.3), bit-specific
+// activation-aware scaling (Section 3.4), clustering permutation and bit
+// blocks (Sections 4.1, 4.2), group quantisation and packing, and the
+// permutation merge rule (Section 4.3).
 //
 // Build with -ffp-contract=off: every floating-point step below is a single
 // IEEE double operation in the order written, so the result is the same on
@@ -31,6 +33,8 @@ struct polyq_layer {
   std::vector<uint8_t> packed;    // [N][S]
   std::vector<uint32_t> meta;     // [N][G] scale | zero << 16
   std::vector<int32_t> out_perm;  // [N]
+  std::vector<float> xscale;      // [K] clustered order; empty = not scaled
+  double alpha[5] = {-1, -1, -1, -1, -1};
 };
 
 namespace {
@@ -53,10 +57,6 @@ double proxy_error(double sal, int b) {
   return e * e;
 }
 
-// Gain per extra bit, Section 3.2.
-double step_gain(double sal, int b, int bn) {
-  return (proxy_error(sal, b) - proxy_error(sal, bn)) / (double)(bn - b);
-}
 
 struct Cand {
   double g;
@@ -160,9 +160,27 @@ void saliency(const float* W, int64_t N, int64_t K, const float* a, std::vector<
   });
 }
 
+// Per-width error table E[width index][k] (Section 3.1).
+struct ErrTable {
+  std::vector<double> e[5];
+  double at(int b, int64_t k) const { return e[width_index(b)][k]; }
+  // gain per extra bit of the step b -> bn (Section 3.2)
+  double gain(int64_t k, int b, int bn) const {
+    return (at(b, k) - at(bn, k)) / (double)(bn - b);
+  }
+};
+
+void saliency_table(const std::vector<double>& sal, const std::vector<int>& pal, ErrTable& E) {
+  for (int b : pal) {
+    std::vector<double>& v = E.e[width_index(b)];
+    v.resize(sal.size());
+    for (size_t k = 0; k < sal.size(); ++k) v[k] = proxy_error(sal[k], b);
+  }
+}
+
 // Section 3.2 greedy allocation under budget B.
-void allocate(const std::vector<double>& sal, double B, const std::vector<int>& pal, int rule,
-              std::vector<uint8_t>& bits) {
+void allocate(const std::vector<double>& sal, const ErrTable& E, double B,
+              const std::vector<int>& pal, int rule, std::vector<uint8_t>& bits) {
   const int64_t K = (int64_t)sal.size();
   const int bmin = pal[0];
   bits.assign(K, (uint8_t)bmin);
@@ -192,7 +210,7 @@ void allocate(const std::vector<double>& sal, double B, const std::vector<int>& 
   std::vector<Cand> init;
   init.reserve(K);
   const int b1 = next_w(bmin);
-  for (int64_t k = 0; k < K; ++k) init.push_back({step_gain(sal[k], bmin, b1), (int32_t)k, b1});
+  for (int64_t k = 0; k < K; ++k) init.push_back({E.gain(k, bmin, b1), (int32_t)k, b1});
   std::priority_queue<Cand, std::vector<Cand>, CandLess> heap(CandLess(), std::move(init));
   while (delta > 0 && !heap.empty()) {
     Cand c = heap.top();
@@ -202,7 +220,7 @@ void allocate(const std::vector<double>& sal, double B, const std::vector<int>& 
     bits[c.k] = (uint8_t)c.bn;
     delta -= cost;
     int bn2 = next_w(c.bn);
-    if (bn2) heap.push({step_gain(sal[c.k], c.bn, bn2), c.k, bn2});
+    if (bn2) heap.push({E.gain(c.k, c.bn, bn2), c.k, bn2});
   }
 }
 
@@ -211,51 +229,63 @@ int64_t seg_bytes_for(int b, int64_t kb) {
   return (raw + 15) / 16 * 16;
 }
 
-// Quantise and pack rows [r0, r1) of the layer.
-void pack_rows(const float* W, int64_t K, polyq_layer& L, int64_t r0, int64_t r1) {
+// The group quantiser: scale and zero (fp16 values) and codes of the cn
+// weights w[0..cn) at width b < 16.
+void quant_group(const double* w, int cn, int b, double* s_out, double* z_out, uint32_t* q) {
+  const double qmax = (double)((1 << b) - 1);
+  double lo = INFINITY, hi = -INFINITY;
+  for (int i = 0; i < cn; ++i) {
+    lo = std::min(lo, w[i]);
+    hi = std::max(hi, w[i]);
+  }
+  double s = f16_to_f64(polyq_f64_to_f16((hi - lo) / qmax));
+  if (s == 0.0) {
+    double alt = std::max(std::max(std::fabs(lo), std::fabs(hi)), 6.103515625e-05);
+    s = f16_to_f64(polyq_f64_to_f16(alt));
+  }
+  double z = std::nearbyint((-lo) / s);
+  z = std::min(std::max(z, 0.0), qmax);
+  for (int i = 0; i < cn; ++i) {
+    double v = std::nearbyint(w[i] / s) + z;
+    v = std::min(std::max(v, 0.0), qmax);
+    q[i] = (uint32_t)v;
+  }
+  *s_out = s;
+  *z_out = z;
+}
+
+// Quantise and pack rows [r0, r1) of the layer.  With activation factors t
+// (original channel order) the packed weight is W / t.
+void pack_rows(const float* W, int64_t K, const double* t, polyq_layer& L, int64_t r0,
+               int64_t r1) {
   std::vector<double> w(POLYQ_GROUP);
   std::vector<uint32_t> q(POLYQ_GROUP);
   for (int64_t n = r0; n < r1; ++n) {
     const float* row = W + n * K;
     uint8_t* prow = L.packed.data() + n * L.S;
     uint32_t* mrow = L.meta.data() + n * L.G;
+    auto wv = [&](int32_t k) { return t ? (double)row[k] / t[k] : (double)row[k]; };
     for (const polyq_block& blk : L.blocks) {
       uint8_t* seg = prow + blk.seg_off;
       const int32_t* pp = L.perm.data() + blk.pos0;
       const int b = blk.bits;
       if (b == 16) {
         for (int32_t i = 0; i < blk.n_ch; ++i) {
-          uint16_t h = polyq_f64_to_f16((double)row[pp[i]]);
+          uint16_t h = polyq_f64_to_f16(wv(pp[i]));
           seg[2 * i] = (uint8_t)(h & 0xFF);
           seg[2 * i + 1] = (uint8_t)(h >> 8);
         }
         continue;
       }
-      const double qmax = (double)((1 << b) - 1);
       uint64_t acc = 0;  // LSB-first bit writer
       int nacc = 0;
       int64_t wb = 0;
       for (int32_t g = 0; g < blk.n_grp; ++g) {
         int32_t c0 = g * POLYQ_GROUP;
         int32_t cn = std::min<int32_t>(POLYQ_GROUP, blk.n_ch - c0);
-        double lo = INFINITY, hi = -INFINITY;
-        for (int32_t i = 0; i < cn; ++i) {
-          w[i] = (double)row[pp[c0 + i]];
-          lo = std::min(lo, w[i]);
-          hi = std::max(hi, w[i]);
-        }
-        double s = f16_to_f64(polyq_f64_to_f16((hi - lo) / qmax));
-        if (s == 0.0) {
-          double alt = std::max(std::max(std::fabs(lo), std::fabs(hi)), 6.103515625e-05);
-          s = f16_to_f64(polyq_f64_to_f16(alt));
-        }
-        double z = std::nearbyint((-lo) / s);
-        z = std::min(std::max(z, 0.0), qmax);
-        for (int32_t i = 0; i < cn; ++i) {
-          double v = std::nearbyint(w[i] / s) + z;
-          v = std::min(std::max(v, 0.0), qmax);
-          q[i] = (uint32_t)v;
-        }
+        for (int32_t i = 0; i < cn; ++i) w[i] = wv(pp[c0 + i]);
+        double s, z;
+        quant_group(w.data(), cn, b, &s, &z, q.data());
         mrow[blk.grp_off + g] =
             (uint32_t)polyq_f64_to_f16(s) | ((uint32_t)polyq_f64_to_f16(z) << 16);
         for (int32_t i = 0; i < cn; ++i) {
@@ -271,6 +301,219 @@ void pack_rows(const float* W, int64_t K, polyq_layer& L, int64_t r0, int64_t r1
       if (nacc > 0) seg[wb++] = (uint8_t)(acc & 0xFF);
       // remaining padding bytes are already zero (buffer zero-initialised)
     }
+  }
+}
+
+// Quantiser-in-the-loop proxy (Section 3.1): for each palette width b < 16
+// the whole layer is quantised at b with groups of 64 consecutive original
+// channels, and E_b[k] = sum_n (w'[n][k] - W[n][k])^2 * x2[k], rows added in
+// order; E_16 = 0.  Threads split the groups.
+void quant_table(const float* W, int64_t N, int64_t K, const std::vector<double>& x2,
+                 const std::vector<int>& pal, int nthreads, ErrTable& E) {
+  const int64_t ng = (K + POLYQ_GROUP - 1) / POLYQ_GROUP;
+  for (int b : pal) {
+    std::vector<double>& e = E.e[width_index(b)];
+    e.assign(K, 0.0);
+    if (b == 16) continue;
+    run_threads(ng, nthreads, [&](int64_t g0, int64_t g1) {
+      double w[POLYQ_GROUP];
+      uint32_t q[POLYQ_GROUP];
+      for (int64_t n = 0; n < N; ++n) {
+        const float* row = W + n * K;
+        for (int64_t g = g0; g < g1; ++g) {
+          const int64_t c0 = g * POLYQ_GROUP;
+          const int cn = (int)std::min<int64_t>(POLYQ_GROUP, K - c0);
+          for (int i = 0; i < cn; ++i) w[i] = (double)row[c0 + i];
+          double sc, z;
+          quant_group(w, cn, b, &sc, &z, q);
+          for (int i = 0; i < cn; ++i) {
+            double d = ((double)q[i] - z) * sc - w[i];
+            e[c0 + i] = e[c0 + i] + d * d;
+          }
+        }
+      }
+    });
+    for (int64_t k = 0; k < K; ++k) e[k] = e[k] * x2[k];
+  }
+}
+
+// Section 3.3, step 1: target block sizes, multiples of the quanta near the
+// allocation's counts, summing to K, with the realised budget closest to
+// round(B*K) (the rule is spelled out at polyq_pack_opts).
+std::vector<int64_t> quanta_targets(const std::vector<int>& pal, const std::vector<int64_t>& cnt,
+                                    const int32_t* quanta, double B, int64_t K) {
+  const int m = (int)pal.size();
+  const int64_t T = (int64_t)std::floor(B * (double)K + 0.5);
+  std::vector<std::vector<int64_t>> cand(m);
+  for (int i = 0; i < m; ++i) {
+    const int64_t q = quanta[width_index(pal[i])];
+    const int64_t base = cnt[i] / q;
+    for (int d = -1; d <= 2; ++d) {
+      const int64_t v = q * (base + d);
+      if (v >= 0 && v <= K && (cand[i].empty() || cand[i].back() != v)) cand[i].push_back(v);
+    }
+  }
+  // key: (|bits - T|, sum |c^ - c|, counts lexicographic)
+  bool have = false;
+  int64_t best_mis = 0, best_mv = 0;
+  std::vector<int64_t> best(m), cur(m);
+  auto consider = [&]() {
+    int64_t tb = 0, mv = 0;
+    for (int i = 0; i < m; ++i) {
+      tb += (int64_t)pal[i] * cur[i];
+      mv += std::llabs(cur[i] - cnt[i]);
+    }
+    const int64_t mis = std::llabs(tb - T);
+    if (!have || mis < best_mis || (mis == best_mis && (mv < best_mv || (mv == best_mv && cur < best)))) {
+      have = true;
+      best_mis = mis;
+      best_mv = mv;
+      best = cur;
+    }
+  };
+  // exact: every width a multiple of its quantum
+  std::vector<size_t> ix(m, 0);
+  for (;;) {
+    int64_t sum = 0;
+    for (int i = 0; i < m; ++i) sum += (cur[i] = cand[i][ix[i]]);
+    if (sum == K) consider();
+    int i = m - 1;
+    while (i >= 0 && ++ix[i] == cand[i].size()) ix[i--] = 0;
+    if (i < 0) break;
+  }
+  if (!have && m > 1) {
+    // the narrowest width takes the remainder
+    std::fill(ix.begin(), ix.end(), 0);
+    for (;;) {
+      int64_t rest = 0;
+      for (int i = 1; i < m; ++i) rest += (cur[i] = cand[i][ix[i]]);
+      cur[0] = K - rest;
+      if (cur[0] >= 0) consider();
+      int i = m - 1;
+      while (i >= 1 && ++ix[i] == cand[i].size()) ix[i--] = 0;
+      if (i < 1) break;
+    }
+  }
+  if (!have) best.assign(1, K);  // a one-width palette keeps every channel
+  return best;
+}
+
+// Section 3.3, step 2: move channels between neighbouring widths until the
+// per-width counts are the targets; promotions by largest gain per bit
+// (lower channel first), demotions by smallest gain (higher channel first).
+void reassign(const std::vector<int>& pal, const std::vector<int64_t>& target, const ErrTable& E,
+              std::vector<uint8_t>& bits) {
+  const int m = (int)pal.size();
+  const int64_t K = (int64_t)bits.size();
+  std::vector<int64_t> flow(m > 1 ? m - 1 : 0);
+  int64_t acc = 0;
+  for (int i = 0; i + 1 < m; ++i) {
+    int64_t c = 0;
+    for (int64_t k = 0; k < K; ++k) c += bits[k] == pal[i];
+    acc += c - target[i];
+    flow[i] = acc;
+  }
+  std::vector<int32_t> mem;
+  for (int i = 0; i + 1 < m; ++i) {
+    if (flow[i] <= 0) continue;
+    const int b = pal[i], bn = pal[i + 1];
+    mem.clear();
+    for (int64_t k = 0; k < K; ++k)
+      if (bits[k] == b) mem.push_back((int32_t)k);
+    std::stable_sort(mem.begin(), mem.end(), [&](int32_t x, int32_t y) {
+      const double gx = E.gain(x, b, bn), gy = E.gain(y, b, bn);
+      if (gx != gy) return gx > gy;
+      return x < y;
+    });
+    for (int64_t j = 0; j < flow[i]; ++j) bits[mem[j]] = (uint8_t)bn;
+  }
+  for (int i = m - 2; i >= 0; --i) {
+    if (flow[i] >= 0) continue;
+    const int b = pal[i], bn = pal[i + 1];
+    mem.clear();
+    for (int64_t k = 0; k < K; ++k)
+      if (bits[k] == bn) mem.push_back((int32_t)k);
+    std::stable_sort(mem.begin(), mem.end(), [&](int32_t x, int32_t y) {
+      const double gx = E.gain(x, b, bn), gy = E.gain(y, b, bn);
+      if (gx != gy) return gx < gy;
+      return x > y;
+    });
+    for (int64_t j = 0; j < -flow[i]; ++j) bits[mem[j]] = (uint8_t)b;
+  }
+}
+
+// Section 3.4: for each width present the exponent alpha (grid j/10) whose
+// activation factors t_k = fp32_rn(m_k^-alpha) give the smallest mean of
+// ||Q_b(W/t)[:,k]*t_k - W[:,k]||^2 * x2[k] over the block, with the block's
+// own groups.  Fills t (original order) and alpha per width index.
+void choose_alphas(const float* W, int64_t N, int64_t K, const std::vector<uint8_t>& bits,
+                   const float* a, const std::vector<double>& x2, int nthreads,
+                   std::vector<double>& t, double* alpha) {
+  std::vector<double> m(K);
+  double tot = 0.0;
+  for (int64_t k = 0; k < K; ++k) tot = tot + (double)a[k];
+  const double mean = tot / (double)K;
+  for (int64_t k = 0; k < K; ++k) m[k] = (double)a[k] / mean;
+  t.assign(K, 1.0);
+  for (int wi = 0; wi < 5; ++wi) alpha[wi] = -1.0;
+  for (int b : kPalette) {
+    std::vector<int32_t> idx;
+    for (int64_t k = 0; k < K; ++k)
+      if (bits[k] == b) idx.push_back((int32_t)k);
+    if (idx.empty()) continue;
+    if (b == 16) {  // E_16 = 0 for every alpha
+      alpha[width_index(b)] = 0.0;
+      continue;
+    }
+    const int64_t kb = (int64_t)idx.size();
+    const int64_t ng = (kb + POLYQ_GROUP - 1) / POLYQ_GROUP;
+    bool have = false;
+    double best_e = 0.0, best_a = 0.0;
+    std::vector<double> best_t, tb(kb), err(kb);
+    for (int j = 0; j <= 10; ++j) {
+      const double al = j / 10.0;
+      bool ok = true;
+      for (int64_t i = 0; i < kb; ++i) {
+        tb[i] = (double)(float)std::pow(m[idx[i]], -al);
+        if (!(std::isfinite(tb[i]) && tb[i] > 0.0)) ok = false;
+      }
+      if (!ok) continue;
+      std::atomic<bool> range_ok(true);
+      std::fill(err.begin(), err.end(), 0.0);
+      run_threads(ng, nthreads, [&](int64_t g0, int64_t g1) {
+        double w[POLYQ_GROUP];
+        uint32_t q[POLYQ_GROUP];
+        for (int64_t n = 0; n < N; ++n) {
+          const float* row = W + n * K;
+          for (int64_t g = g0; g < g1; ++g) {
+            const int64_t c0 = g * POLYQ_GROUP;
+            const int cn = (int)std::min<int64_t>(POLYQ_GROUP, kb - c0);
+            for (int i = 0; i < cn; ++i) {
+              w[i] = (double)row[idx[c0 + i]] / tb[c0 + i];
+              if (!(std::fabs(w[i]) <= 65504.0)) range_ok = false;
+            }
+            double sc, z;
+            quant_group(w, cn, b, &sc, &z, q);
+            for (int i = 0; i < cn; ++i) {
+              double d = ((double)q[i] - z) * sc * tb[c0 + i] - (double)row[idx[c0 + i]];
+              err[c0 + i] = err[c0 + i] + d * d;
+            }
+          }
+        }
+      });
+      if (!range_ok.load()) continue;
+      double s = 0.0;
+      for (int64_t i = 0; i < kb; ++i) s = s + err[i] * x2[idx[i]];
+      const double e = s / (double)kb;
+      if (!have || e < best_e) {
+        have = true;
+        best_e = e;
+        best_a = al;
+        best_t = tb;
+      }
+    }
+    alpha[width_index(b)] = best_a;  // alpha = 0 is always usable
+    for (int64_t i = 0; i < kb; ++i) t[idx[i]] = best_t[i];
   }
 }
 
@@ -307,10 +550,32 @@ extern "C" int polyq_pack(const float* W, int64_t N, int64_t K, const float* act
                            (long long)K);
   if (o.group_size != POLYQ_GROUP)
     return polyq_set_error(POLYQ_EUNSUPPORTED, "polyq_pack: group_size must be 64");
-  if (o.snap_quanta != 0)
-    return polyq_set_error(POLYQ_EUNSUPPORTED, "polyq_pack: quanta matching is not built");
   if (o.alloc_rule != POLYQ_ALLOC_WATERFILL && o.alloc_rule != POLYQ_ALLOC_LADDER)
     return polyq_set_error(POLYQ_EINVAL, "polyq_pack: unknown alloc_rule %d", o.alloc_rule);
+  if (o.proxy != POLYQ_PROXY_SALIENCY && o.proxy != POLYQ_PROXY_QUANT)
+    return polyq_set_error(POLYQ_EINVAL, "polyq_pack: unknown proxy %d", o.proxy);
+  if (o.proxy == POLYQ_PROXY_QUANT && o.alloc_rule == POLYQ_ALLOC_LADDER)
+    return polyq_set_error(POLYQ_EINVAL, "polyq_pack: the ladder rule needs the saliency proxy");
+  if (o.snap_quanta != 0 && o.snap_quanta != 1)
+    return polyq_set_error(POLYQ_EINVAL, "polyq_pack: snap_quanta must be 0 or 1");
+  if (o.act_scaling != 0 && o.act_scaling != 1)
+    return polyq_set_error(POLYQ_EINVAL, "polyq_pack: act_scaling must be 0 or 1");
+  if (o.snap_quanta && o.forced_bits)
+    return polyq_set_error(POLYQ_EINVAL, "polyq_pack: forced_bits cannot be snapped to quanta");
+  int32_t quanta[5] = POLYQ_GPU_QUANTA;
+  {
+    int nz = 0;
+    for (int i = 0; i < 5; ++i) nz += o.quanta[i] != 0;
+    if (nz == 5) {
+      for (int i = 0; i < 5; ++i) {
+        if (o.quanta[i] < 1 || o.quanta[i] > (1 << 24))
+          return polyq_set_error(POLYQ_EINVAL, "polyq_pack: quanta[%d] = %d", i, o.quanta[i]);
+        quanta[i] = o.quanta[i];
+      }
+    } else if (nz != 0) {
+      return polyq_set_error(POLYQ_EINVAL, "polyq_pack: set all five quanta or none");
+    }
+  }
   uint32_t mask = o.palette_mask ? o.palette_mask
                                  : ((1u << 2) | (1u << 3) | (1u << 4) | (1u << 8) | (1u << 16));
   std::vector<int> pal;
@@ -318,8 +583,9 @@ extern "C" int polyq_pack(const float* W, int64_t N, int64_t K, const float* act
     if (mask & (1u << b)) pal.push_back(b);
   if (pal.empty() || (mask & ~((1u << 2) | (1u << 3) | (1u << 4) | (1u << 8) | (1u << 16))))
     return polyq_set_error(POLYQ_EINVAL, "polyq_pack: bad palette mask 0x%x", mask);
+  if ((!o.forced_bits || o.act_scaling) && !act_absmean)
+    return polyq_set_error(POLYQ_EINVAL, "polyq_pack: act_absmean is NULL");
   if (!o.forced_bits) {
-    if (!act_absmean) return polyq_set_error(POLYQ_EINVAL, "polyq_pack: act_absmean is NULL");
     if (!(budget_bits >= 2.0 && budget_bits <= 16.0))
       return polyq_set_error(POLYQ_EINVAL, "polyq_pack: budget %g outside [2,16]", budget_bits);
   }
@@ -354,11 +620,43 @@ extern "C" int polyq_pack(const float* W, int64_t N, int64_t K, const float* act
           return polyq_set_error(POLYQ_EINVAL, "polyq_pack: forced width %d at %lld",
                                  (int)L->bits[k], (long long)k);
         }
-    } else {
-      std::vector<double> sal;
-      saliency(W, N, K, act_absmean, sal, o.n_threads);
-      allocate(sal, budget_bits, pal, o.alloc_rule, L->bits);
     }
+    // E[x^2] of the quantiser proxy and the scaling search
+    std::vector<double> x2;
+    if (o.proxy == POLYQ_PROXY_QUANT || o.act_scaling) {
+      x2.resize(K);
+      for (int64_t k = 0; k < K; ++k) {
+        const double v = o.act_sqmean ? (double)o.act_sqmean[k] : (double)act_absmean[k];
+        x2[k] = o.act_sqmean ? v : v * v;
+        if (!(x2[k] >= 0.0 && std::isfinite(x2[k]))) {
+          delete L;
+          return polyq_set_error(POLYQ_EINVAL, "polyq_pack: E[x^2] of channel %lld is not finite "
+                                 "and >= 0", (long long)k);
+        }
+      }
+    }
+    if (!o.forced_bits) {
+      std::vector<double> sal;
+      ErrTable E;
+      if (o.proxy == POLYQ_PROXY_QUANT) {
+        sal.assign(K, 0.0);  // unused by the waterfilling rule
+        quant_table(W, N, K, x2, pal, o.n_threads, E);
+      } else {
+        saliency(W, N, K, act_absmean, sal, o.n_threads);
+        saliency_table(sal, pal, E);
+      }
+      allocate(sal, E, budget_bits, pal, o.alloc_rule, L->bits);
+      if (o.snap_quanta) {
+        std::vector<int64_t> cnt(pal.size(), 0);
+        for (size_t i = 0; i < pal.size(); ++i)
+          for (int64_t k = 0; k < K; ++k) cnt[i] += L->bits[k] == pal[i];
+        const std::vector<int64_t> tgt = quanta_targets(pal, cnt, quanta, budget_bits, K);
+        reassign(pal, tgt, E, L->bits);
+      }
+    }
+    std::vector<double> tfac;
+    if (o.act_scaling)
+      choose_alphas(W, N, K, L->bits, act_absmean, x2, o.n_threads, tfac, L->alpha);
     // Section 4.1: stable clustering by width
     L->perm.reserve(K);
     for (int b : kPalette)
@@ -389,7 +687,12 @@ extern "C" int polyq_pack(const float* W, int64_t N, int64_t K, const float* act
     L->meta.assign((size_t)(N * L->G), 0);
     L->out_perm.resize(N);
     for (int64_t n = 0; n < N; ++n) L->out_perm[n] = (int32_t)n;
-    run_threads(N, o.n_threads, [&](int64_t a, int64_t b) { pack_rows(W, K, *L, a, b); });
+    const double* tp = o.act_scaling ? tfac.data() : nullptr;
+    run_threads(N, o.n_threads, [&](int64_t a, int64_t b) { pack_rows(W, K, tp, *L, a, b); });
+    if (o.act_scaling) {
+      L->xscale.resize(K);
+      for (int64_t p = 0; p < K; ++p) L->xscale[p] = (float)tfac[L->perm[p]];
+    }
   } catch (const std::bad_alloc&) {
     delete L;
     return polyq_set_error(POLYQ_ENOMEM, "polyq_pack: out of host memory");
@@ -417,6 +720,21 @@ extern "C" int polyq_layer_info(const polyq_layer* L, polyq_info* out) {
   out->packed_bytes = L->N * L->S;
   out->meta_bytes = L->N * L->G * 4;
   out->meta_stride = (L->G + 3) / 4 * 4;
+  int64_t pad = 0;
+  for (const polyq_block& b : L->blocks) {
+    const int64_t raw = b.bits == 16 ? 2 * (int64_t)b.n_ch : ((int64_t)b.n_ch * b.bits + 7) / 8;
+    pad += b.seg_bytes - raw;
+  }
+  out->pad_bytes = pad;
+  for (int i = 0; i < 5; ++i) out->alpha[i] = L->alpha[i];
+  out->has_xscale = L->xscale.empty() ? 0 : 1;
+  return POLYQ_OK;
+}
+
+extern "C" int polyq_layer_xscale(const polyq_layer* L, float* xscale) {
+  polyq_clear_error();
+  if (!L || !xscale) return polyq_set_error(POLYQ_EINVAL, "polyq_layer_xscale: NULL argument");
+  for (int64_t p = 0; p < L->K; ++p) xscale[p] = L->xscale.empty() ? 1.0f : L->xscale[p];
   return POLYQ_OK;
 }
 
@@ -503,8 +821,8 @@ int polyq_check_dev_layer(const polyq_dev_layer* L, const char* who) {
     return polyq_set_error(POLYQ_EINVAL, "%s: bad shape", who);
   if (L->row_stride <= 0 || L->row_stride % 16)
     return polyq_set_error(POLYQ_EINVAL, "%s: row_stride must be a positive multiple of 16", who);
-  if (((uintptr_t)L->packed) % 16 || ((uintptr_t)L->meta) % 16)
-    return polyq_set_error(POLYQ_EINVAL, "%s: packed/meta must be 16-byte aligned", who);
+  if (((uintptr_t)L->packed) % 16 || ((uintptr_t)L->meta) % 16 || ((uintptr_t)L->xscale) % 16)
+    return polyq_set_error(POLYQ_EINVAL, "%s: packed/meta/xscale must be 16-byte aligned", who);
   if (L->n_blocks < 1 || L->n_blocks > POLYQ_MAX_BLOCKS)
     return polyq_set_error(POLYQ_EINVAL, "%s: bad block count", who);
   int32_t pos = 0, off = 0, goff = 0, prev = 0;

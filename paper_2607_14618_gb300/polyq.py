@@ -25,6 +25,9 @@ MAX_GROUP = 4
 GROUP = 64
 NOALLOC_SCRATCH_BYTES = 1 << 20  # scratch compiled in for linear_gemv_noalloc
 ALLOC_WATERFILL = 0
+PROXY_SALIENCY = 0
+PROXY_QUANT = 1
+GPU_QUANTA = {2: 64, 3: 128, 4: 32, 8: 16, 16: 8}
 ALLOC_LADDER = 1
 
 if not os.path.exists(LIB_PATH):
@@ -41,7 +44,9 @@ class PolyqError(RuntimeError):
 class PackOpts(C.Structure):
     _fields_ = [("group_size", C.c_int32), ("palette_mask", C.c_uint32),
                 ("alloc_rule", C.c_int32), ("snap_quanta", C.c_int32),
-                ("n_threads", C.c_int32), ("forced_bits", C.POINTER(C.c_uint8))]
+                ("n_threads", C.c_int32), ("forced_bits", C.POINTER(C.c_uint8)),
+                ("proxy", C.c_int32), ("act_scaling", C.c_int32), ("quanta", C.c_int32 * 5),
+                ("act_sqmean", C.POINTER(C.c_float))]
 
 
 class Block(C.Structure):
@@ -58,7 +63,8 @@ class Info(C.Structure):
                 ("n_groups", C.c_int64), ("n_blocks", C.c_int32),
                 ("blocks", Block * MAX_BLOCKS), ("budget", C.c_double), ("b_real", C.c_double),
                 ("packed_bytes", C.c_int64), ("meta_bytes", C.c_int64),
-                ("meta_stride", C.c_int64)]
+                ("meta_stride", C.c_int64), ("pad_bytes", C.c_int64), ("alpha", C.c_double * 5),
+                ("has_xscale", C.c_int32)]
 
 
 X_BF16, X_F32, X_RMSNORM, X_SILU_MUL = 0, 1, 2, 3
@@ -73,7 +79,7 @@ class DevLayer(C.Structure):
     _fields_ = [("packed", C.c_void_p), ("meta", C.c_void_p), ("gather", C.c_void_p),
                 ("N", C.c_int64), ("K", C.c_int64), ("row_stride", C.c_int64),
                 ("n_groups", C.c_int64), ("meta_stride", C.c_int64), ("n_blocks", C.c_int32),
-                ("blocks", Block * MAX_BLOCKS)]
+                ("blocks", Block * MAX_BLOCKS), ("xscale", C.c_void_p)]
 
 
 _P = C.c_void_p
@@ -85,6 +91,7 @@ _SIGS = {
     "polyq_free": (None, [_P]),
     "polyq_layer_info": (C.c_int, [_P, C.POINTER(Info)]),
     "polyq_layer_export": (C.c_int, [_P, _P, _P, C.c_int64, _P, _P, _P]),
+    "polyq_layer_xscale": (C.c_int, [_P, _P]),
     "polyq_layer_permute_rows": (C.c_int, [_P, _P]),
     "polyq_permute_merge": (C.c_int, [_P, _P, C.c_int64, _P]),
     "polyq_dev_layer_fill": (C.c_int, [_P, _P, _P, _P, C.POINTER(DevLayer)]),
@@ -157,7 +164,14 @@ class HostLayer:
 
     @classmethod
     def pack(cls, W, act_absmean=None, budget=3.0, forced_bits=None,
-             rule=ALLOC_WATERFILL, palette=(2, 3, 4, 8, 16), n_threads=0):
+             rule=ALLOC_WATERFILL, palette=(2, 3, 4, 8, 16), n_threads=0,
+             proxy=PROXY_SALIENCY, snap_quanta=False, quanta=None, act_scaling=False,
+             act_sqmean=None):
+        """Allocate, (optionally) snap to quanta and scale, cluster and pack.
+
+        ``quanta`` maps widths 2, 3, 4, 8, 16 to channels per quantum (default
+        GPU_QUANTA); ``act_sqmean`` is E[x^2] per channel (default
+        act_absmean squared)."""
         W = np.ascontiguousarray(W, dtype=np.float32)
         if W.ndim != 2:
             raise ValueError("W must be [N][K]")
@@ -167,6 +181,18 @@ class HostLayer:
         opts.alloc_rule = int(rule)
         opts.palette_mask = _palette_mask(palette)
         opts.n_threads = int(n_threads)
+        opts.proxy = int(proxy)
+        opts.snap_quanta = 1 if snap_quanta else 0
+        opts.act_scaling = 1 if act_scaling else 0
+        if quanta is not None:
+            for i, b in enumerate((2, 3, 4, 8, 16)):
+                opts.quanta[i] = int(quanta[b])
+        keep_x2 = None
+        if act_sqmean is not None:
+            keep_x2 = np.ascontiguousarray(act_sqmean, dtype=np.float32)
+            if keep_x2.shape != (W.shape[1],):
+                raise ValueError("act_sqmean must be [K]")
+            opts.act_sqmean = keep_x2.ctypes.data_as(C.POINTER(C.c_float))
         keep = None
         if forced_bits is not None:
             keep = np.ascontiguousarray(forced_bits, dtype=np.uint8)
@@ -193,7 +219,15 @@ class HostLayer:
         _check(_lib.polyq_layer_info(self._h, C.byref(inf)))
         d = {f: getattr(inf, f) for f, _ in Info._fields_ if f != "blocks"}
         d["blocks"] = [inf.blocks[i].as_dict() for i in range(inf.n_blocks)]
+        d["alpha"] = {b: inf.alpha[i] for i, b in enumerate((2, 3, 4, 8, 16))}
         return d
+
+    def xscale(self):
+        """Section 3.4 activation factors [K] in clustered order (1.0 if the
+        layer is not scaled)."""
+        out = np.empty(self.info()["K"], np.float32)
+        _check(_lib.polyq_layer_xscale(self._h, out.ctypes.data))
+        return out
 
     def export(self, meta_stride=None) -> dict:
         """Host copies; meta rows have ``meta_stride`` entries (default: the
@@ -235,6 +269,10 @@ class DeviceLayer:
         _check(_lib.polyq_dev_layer_fill(
             host._h, self.packed.data_ptr(), self.meta.data_ptr() if self.meta.numel() else None,
             self.gather.data_ptr() if self.gather is not None else None, C.byref(self.desc)))
+        self.xscale = None
+        if self.info["has_xscale"]:
+            self.xscale = torch.from_numpy(host.xscale()).to(device)
+            self.desc.xscale = self.xscale.data_ptr()
         self.N = self.info["N"]
         self.K = self.info["K"]
 
@@ -245,6 +283,7 @@ class DeviceLayer:
         """A second device copy of the same packed layer (distinct memory)."""
         c = object.__new__(DeviceLayer)
         c.info, c.perm, c.out_perm, c.N, c.K = self.info, self.perm, self.out_perm, self.N, self.K
+        c.xscale = self.xscale
         c.packed = self.packed.clone()
         c.meta = self.meta.clone()
         c.gather = self.gather

@@ -198,6 +198,7 @@ def test_corrupt_descriptors_rejected_before_launch(polyq_lib):
         lambda d: setattr(d.blocks[3], "grp_off", 0),
         lambda d: setattr(d, "n_groups", d.n_groups - 1),
         lambda d: setattr(d, "meta_stride", d.meta_stride + 1),
+        lambda d: setattr(d, "xscale", 0x500004),
         lambda d: setattr(d, "meta_stride", d.n_groups - 1),
     ]
     for f in cases:
@@ -210,3 +211,127 @@ def test_corrupt_descriptors_rejected_before_launch(polyq_lib):
     assert gemv(d, batch=5) == polyq_lib.POLYQ_EUNSUPPORTED
     assert L.polyq_linear_gemv(C.byref(d), None, 1, C.c_void_p(0x400000), None, None, 0,
                                None) == polyq_lib.POLYQ_EINVAL
+
+
+# ---------------------------------------------------------------------------
+# Section 3.1 quantiser proxy, Section 3.3 quanta matching, Section 3.4
+# scaling: the library against the oracle, bit for bit
+# ---------------------------------------------------------------------------
+def _x2(a):
+    return np.asarray(a, np.float32).astype(np.float64) ** 2
+
+
+@pytest.mark.parametrize("N,K,B,seed", [
+    (256, 2048, 3.0, 1000),   # the 2048-channel decode layer's shape at B = 3
+    (64, 5120, 4.5, 2001),
+    (40, 1000, 3.7, 5),       # K a multiple of 8 only
+    (33, 777, 2.6, 6),        # no exact sum: the 2-bit block fills
+    (16, 13824, 3.0, 2006),
+])
+def test_snap_to_quanta_matches_oracle(polyq_lib, N, K, B, seed):
+    W, a = synth.layer_weights(N, K, seed)
+    host = polyq_lib.HostLayer.pack(W, a, B, snap_quanta=True)
+    sal = O.saliency(W, a)
+    bits = O.snap_to_quanta(O.allocate_bits(sal, B), O.saliency_error_table(sal), B)
+    _compare(host, O.pack_layer(W, a, B, bits=bits))
+    inf = host.info()
+    assert inf["pad_bytes"] == O.padding_bytes_per_row(bits)
+    if K % 128 == 0:
+        assert inf["pad_bytes"] == 0
+
+
+def test_snap_with_custom_quanta_and_ladder_matches_oracle(polyq_lib):
+    W, a = synth.layer_weights(24, 3000, 31)
+    q = {2: 96, 3: 32, 4: 48, 8: 8, 16: 8}
+    host = polyq_lib.HostLayer.pack(W, a, 3.3, snap_quanta=True, quanta=q,
+                                    rule=polyq_lib.ALLOC_LADDER)
+    sal = O.saliency(W, a)
+    bits = O.snap_to_quanta(O.allocate_bits(sal, 3.3, rule=O.SALIENCY_LADDER),
+                            O.saliency_error_table(sal), 3.3, quanta=q)
+    assert np.array_equal(host.export()["bits"], bits.astype(np.uint8))
+
+
+@pytest.mark.parametrize("N,K,B,seed", [
+    (128, 2048, 3.0, 1000),
+    (50, 777, 4.2, 7),
+    (20, 64, 2.5, 8),
+])
+def test_quant_proxy_allocation_matches_oracle(polyq_lib, N, K, B, seed):
+    W, a = synth.layer_weights(N, K, seed)
+    host = polyq_lib.HostLayer.pack(W, a, B, proxy=polyq_lib.PROXY_QUANT)
+    bits = O.allocate_from_table(O.quant_error_table(W, _x2(a)), B)
+    _compare(host, O.pack_layer(W, a, B, bits=bits))
+
+
+def test_quant_proxy_with_explicit_second_moments(polyq_lib):
+    W, a = synth.layer_weights(40, 900, 12)
+    x2 = (np.random.default_rng(1).random(900) * 3).astype(np.float32)
+    host = polyq_lib.HostLayer.pack(W, a, 3.2, proxy=polyq_lib.PROXY_QUANT, act_sqmean=x2)
+    bits = O.allocate_from_table(O.quant_error_table(W, x2.astype(np.float64)), 3.2)
+    assert np.array_equal(host.export()["bits"], bits.astype(np.uint8))
+
+
+def _compare_scaled(host, W, a, bits, x2):
+    alphas, t = O.choose_alphas(W, bits, a, x2)
+    ref = O.pack_layer_scaled(W, bits, t)
+    _compare(host, ref)
+    inf = host.info()
+    assert inf["has_xscale"] == 1
+    for b in O.PALETTE:
+        assert inf["alpha"][b] == (alphas[b] if b in alphas else -1.0)
+    assert np.array_equal(host.xscale(), ref["xscale"].astype(np.float32))
+
+
+@pytest.mark.parametrize("N,K,B,seed", [
+    (96, 2048, 3.0, 1000),
+    (40, 1000, 4.5, 9),
+])
+def test_scaled_pack_matches_oracle(polyq_lib, N, K, B, seed):
+    W, a = synth.layer_weights(N, K, seed)
+    host = polyq_lib.HostLayer.pack(W, a, B, proxy=polyq_lib.PROXY_QUANT, snap_quanta=True,
+                                    act_scaling=True)
+    E = O.quant_error_table(W, _x2(a))
+    bits = O.snap_to_quanta(O.allocate_from_table(E, B), E, B)
+    _compare_scaled(host, W, a, bits, _x2(a))
+
+
+def test_scaled_pack_with_forced_widths_matches_oracle(polyq_lib):
+    W, a = synth.layer_weights(30, 3001, 13)
+    bits = synth.random_codes_layer_bits(3001, 13)
+    host = polyq_lib.HostLayer.pack(W, a, 3.0, forced_bits=bits, act_scaling=True)
+    _compare_scaled(host, W, a, bits, _x2(a))
+
+
+def test_unscaled_layer_reports_no_factors(polyq_lib):
+    W, a = synth.layer_weights(8, 300, 14)
+    host = polyq_lib.HostLayer.pack(W, a, 3.0)
+    inf = host.info()
+    assert inf["has_xscale"] == 0 and all(v == -1.0 for v in inf["alpha"].values())
+    assert np.all(host.xscale() == 1.0)
+
+
+def test_new_pack_options_are_validated(polyq_lib):
+    W, a = synth.layer_weights(4, 128, 1)
+    bad = [
+        dict(snap_quanta=True, forced_bits=np.full(128, 3)),
+        dict(proxy=polyq_lib.PROXY_QUANT, rule=polyq_lib.ALLOC_LADDER),
+        dict(proxy=7),
+        dict(act_sqmean=np.full(128, -1.0, np.float32), proxy=polyq_lib.PROXY_QUANT),
+        dict(act_sqmean=np.full(128, np.nan, np.float32), act_scaling=True),
+    ]
+    for kw in bad:
+        with pytest.raises(polyq_lib.PolyqError) as ei:
+            polyq_lib.HostLayer.pack(W, a, 3.0, **kw)
+        assert ei.value.code == polyq_lib.POLYQ_EINVAL, kw
+    opts = polyq_lib.PackOpts()
+    polyq_lib._lib.polyq_pack_opts_default(C.byref(opts))
+    opts.snap_quanta = 1
+    opts.quanta[0] = 64  # one quantum set, the others zero
+    h = C.c_void_p()
+    W32 = np.ascontiguousarray(W, np.float32)
+    a32 = np.ascontiguousarray(a, np.float32)
+    rc = polyq_lib._lib.polyq_pack(W32.ctypes.data, 4, 128, a32.ctypes.data, 3.0,
+                                   C.byref(opts), C.byref(h))
+    assert rc == polyq_lib.POLYQ_EINVAL
+    with pytest.raises(polyq_lib.PolyqError):
+        polyq_lib.HostLayer.pack(W, None, 3.0, forced_bits=np.full(128, 3), act_scaling=True)
