@@ -372,8 +372,11 @@ __device__ __forceinline__ void rec_build(const XIn& in, const GvBlock& B, int j
     const __half hhi = __float2half_rn(ldexpf(xv[s][1], -g.p[1]));
     rec[(g.bb * 4 + g.t) * LW + g.jp] = pack_half2(hlo, hhi);
     if (B.bits != 16) {
+      // X sums the values the MMA multiplies (fp16 times 2^p), so that the
+      // zero-point term removes exactly what the codes' z adds; with
+      // activation factors these differ from the fp32 products x * t
       float s1 = __half2float(hlo) + __half2float(hhi);
-      float s2 = xv[s][0] + xv[s][1];
+      float s2 = ldexpf(__half2float(hlo), g.p[0]) + ldexpf(__half2float(hhi), g.p[1]);
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) {
         s1 += __shfl_xor_sync(0xffffffffu, s1, o);
