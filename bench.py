@@ -340,6 +340,7 @@ def run_polyq(args):
             "clocks": clk.summary(),
             "prefill_gemm": gemm,
             "decode_step": decode,
+            "permutation_plan": plan_report(polyq),
         }
         print(json.dumps(out), flush=True)
     if ws > 1:
@@ -465,6 +466,47 @@ def bench_decode_step(polyq, synth, torch, device, stream, args, hbm):
     out["reorder_traffic_no_merge_mib"] = round(no_merge / 2 ** 20, 3)
     out["workload"] = (f"llama2-13b decode step, {L} layers (device copies of one packed "
                        f"layer set), batch 1, B={args.budget}, position 0")
+    return out
+
+
+def plan_report(polyq):
+    """§4.4 planning of the whole decode graph (host, no GPU) on the
+    Llama2-13B and Qwen3-32B shapes: modelled activation-reorder traffic per
+    token (§5.3 model) without merges and with the library planner, for
+    separately allocated linears and for q/k/v and gate/up allocated jointly.
+    Every layer gets its own seeded permutations (distinct allocations)."""
+    shapes = {"llama2_13b": dict(layers=40, hidden=5120, ffn=13824, kv=None, qdim=None,
+                                 paper_polyq_mib=1.14, paper_no_merge_mib=6.80),
+              "qwen3_32b": dict(layers=64, hidden=5120, ffn=25600, kv=1024, qdim=8192,
+                                paper_polyq_mib=2.95, paper_no_merge_mib=14.50)}
+    out = {}
+    for name, c in shapes.items():
+        res = {}
+        for mode in ("separate", "grouped"):
+            rng = np.random.default_rng(7)
+            perms, ids = [], {}
+
+            def perm_of(l, nm):
+                key = (l, {"q": "qkv", "k": "qkv", "v": "qkv", "gate": "gu", "up": "gu"}
+                       .get(nm, nm) if mode == "grouped" else nm)
+                if key not in ids:
+                    width = {"o": c["qdim"] or c["hidden"], "down": c["ffn"]}.get(nm, c["hidden"])
+                    ids[key] = len(perms)
+                    perms.append(rng.permutation(width).astype(np.int32))
+                return ids[key]
+
+            nodes, dims, _ = polyq.decoder_plan_graph(c["layers"], c["hidden"], c["ffn"], perm_of,
+                                                      c["kv"], c["qdim"])
+            t0 = time.perf_counter()
+            _, cost = polyq.plan_graph(nodes, dims, perms)
+            dt = time.perf_counter() - t0
+            no_merge = 4 * sum(dims[i[0]] for k, i, o, p in nodes if k == polyq.NODE_LINEAR)
+            res[mode] = {"planned_mib": round(cost / 2 ** 20, 3),
+                         "removed": round(1 - cost / no_merge, 4), "planner_ms": round(dt * 1e3, 2)}
+        res["no_merge_mib"] = round(no_merge / 2 ** 20, 3)
+        res["paper_no_merge_mib"] = c["paper_no_merge_mib"]
+        res["paper_polyq_mib"] = c["paper_polyq_mib"]
+        out[name] = res
     return out
 
 

@@ -233,6 +233,59 @@ int polyq_permute_merge(const int32_t* producer_basis,
                         const int32_t* consumer_perm, int64_t n,
                         int32_t* gather_out);
 
+/* Section 4.4 graph-based permutation planning.  The model is a static DAG
+ * whose edges are activations and whose nodes are: */
+#define POLYQ_NODE_SOURCE_FIXED 0 /* no inputs; emits its output in natural order */
+#define POLYQ_NODE_SOURCE_FREE 1  /* no inputs; emits in any order at no cost
+                                     (e.g. an embedding table with permuted columns) */
+#define POLYQ_NODE_LINEAR 2       /* in[0] = x; reads x in any order through its
+                                     gather and emits any order by permuting its
+                                     output rows; `perm` = id of its clustering
+                                     permutation in the perms table */
+#define POLYQ_NODE_ELEMENTWISE 3  /* 1..3 inputs and the output share one order
+                                     (norms, activations, products, residual adds) */
+#define POLYQ_NODE_BOUNDARY 4     /* inputs read in natural order; the output, if
+                                     any, is natural (graph outputs, rotary q/k) */
+#define POLYQ_NODE_ATTENTION 5    /* in = q, k, v: q and k natural; the output keeps
+                                     v's order when both have the same width (the
+                                     kernel maps channels to heads through it),
+                                     otherwise v is read and the output written in
+                                     natural order */
+
+typedef struct {
+  int32_t kind;   /* POLYQ_NODE_* */
+  int32_t n_in;   /* inputs used in `in` (0..3) */
+  int32_t in[3];  /* input edge ids */
+  int32_t out;    /* output edge id, or -1 */
+  int32_t perm;   /* POLYQ_NODE_LINEAR: permutation id; otherwise -1 */
+} polyq_plan_node;
+
+/* Assign a channel order ("basis") to every edge so that the explicit
+ * activation shuffles the graph needs cost the least modelled traffic
+ * (Section 4.4; the traffic model is Section 5.3's A16 read + write, 4 bytes
+ * per channel per shuffle).  Edges joined by elementwise nodes (and by an
+ * attention node that keeps v's order) form regions that share one order;
+ * each region takes, among the natural order and the permutations of the
+ * linears reading it, the one with the smallest cost: one shuffle per
+ * distinct (edge, order wanted by a consumer) that differs from the region's
+ * order, shared by every consumer of that edge wanting that order, plus one
+ * per fixed-order producer that differs.  Ties go to the natural order, then
+ * to the lowest permutation id.  Permutations with equal contents count as
+ * one order, and an identity permutation as the natural order.
+ *   nodes [n_nodes], edge_dims [n_edges] (channels of each edge, >= 1).
+ *   perms [n_perms]: host int32 arrays, perms[i] of length perm_lens[i] (a
+ *   permutation; a linear's permutation must be as long as its input edge).
+ *   labels [n_edges] (out): -1 = natural order, else the id of the
+ *   permutation p (the smallest id with p's contents): the edge carries
+ *   emitted[i] = natural[p[i]].
+ *   bytes_per_token (out, may be NULL): the plan's modelled traffic.
+ * A linear then reads its input through polyq_permute_merge(label of its
+ * input edge, its permutation) (identity when equal) and has its rows
+ * permuted to its output edge's label (polyq_layer_permute_rows). */
+int polyq_plan_graph(const polyq_plan_node* nodes, int32_t n_nodes, const int64_t* edge_dims,
+                     int32_t n_edges, const int32_t* const* perms, const int64_t* perm_lens,
+                     int32_t n_perms, int32_t* labels, int64_t* bytes_per_token);
+
 /* Fill a device-layer descriptor from a host layer and the device copies of
  * its packed bytes and meta (uploaded by the caller from polyq_layer_export
  * with meta_stride = polyq_info.meta_stride) and an optional device gather

@@ -65,6 +65,19 @@ R15 quantiser-in-the-loop proxy (§3.1, Eq. for E_b[j]): E_b[k] =
    sum_n (Q_b(W)[n,k] - W[n,k])^2 * E[x_k^2] with Q_b the R1 quantiser applied
    to the whole layer at width b, groups = 64 consecutive original channels of
    a row; E_16 = 0.  The sum over n runs in row order in fp64.
+R17 graph planning (§4.4): edges carry a channel basis; linears absorb any
+   input basis into their gather and emit any output basis by permuting
+   rows; elementwise nodes (norms, activations, products, residual adds)
+   keep one basis for all their inputs and their output; attention passes
+   v's basis to its output when they have the same width (the kernel reads
+   the head of each channel from the basis) and otherwise, like graph
+   outputs and q/k under rotary embedding, needs the natural basis.  The
+   edges joined by basis-keeping nodes form regions; each region takes the
+   candidate basis (natural, or a consuming linear's permutation) with the
+   smallest modelled traffic, where one explicit shuffle of an edge into a
+   basis costs 4 bytes per channel (A16 read + write, §5.3) and is shared
+   by every consumer of that edge wanting that basis; ties go to natural,
+   then to the lowest permutation id.
 R16 bit-specific scaling (§3.4): m_k = a_k / mean(a) (a = the activation
    magnitude, mean summed in channel order) and, for the channels of width b,
    the activation factor t_k = fp32_rn(m_k^-alpha_b), i.e. s_k = 1/t_k.  A
@@ -792,3 +805,217 @@ def linear_scaled(layer, x, gather=None):
     r = layer["perm"] if gather is None else np.asarray(gather)
     xs = x[:, r] * layer["xscale"][None, :]
     return xs @ dequant(layer).T
+
+
+# ---------------------------------------------------------------------------
+# §4.4 graph-based permutation planning (R17)
+# ---------------------------------------------------------------------------
+NODE_SOURCE_FIXED = 0   # emits its edge in the natural basis
+NODE_SOURCE_FREE = 1    # emits in any basis at no cost (e.g. a permuted embedding)
+NODE_LINEAR = 2         # ins = [x]; absorbs its input basis, emits any basis
+NODE_ELEMENTWISE = 3    # ins and out share one basis (norm, activation, product, add)
+NODE_BOUNDARY = 4       # ins need the natural basis; out (if any) is natural
+NODE_ATTENTION = 5      # ins = [q, k, v]: q, k natural; out keeps v's basis if widths match
+NATURAL = -1
+
+
+def _basis_joins(nodes, edge_dims):
+    """Pairs of edges that one node forces into the same basis (R17)."""
+    joins = []
+    for kind, ins, out, _ in nodes:
+        if kind == NODE_ELEMENTWISE:
+            for e in ins:
+                joins.append((e, out))
+        elif kind == NODE_ATTENTION and out >= 0 and edge_dims[ins[2]] == edge_dims[out]:
+            joins.append((ins[2], out))
+    return joins
+
+
+def plan_regions(nodes, edge_dims):
+    """Region id of every edge: connected components of the basis joins."""
+    n = len(edge_dims)
+    parent = list(range(n))
+
+    def find(i):
+        while parent[i] != i:
+            i = parent[i]
+        return i
+
+    for a, b in _basis_joins(nodes, edge_dims):
+        ra, rb = find(a), find(b)
+        if ra != rb:
+            parent[max(ra, rb)] = min(ra, rb)
+    return [find(i) for i in range(n)]
+
+
+def _requests(nodes, edge_dims):
+    """(edge, wanted basis) pairs: what each consumer needs to read without a
+    shuffle, and the fixed bases producers emit."""
+    want = []   # (edge, basis) consumers
+    fixed = []  # (edge, basis) producers that cannot choose
+    for kind, ins, out, perm in nodes:
+        if kind == NODE_LINEAR:
+            want.append((ins[0], perm))
+        elif kind == NODE_BOUNDARY:
+            want.extend((e, NATURAL) for e in ins)
+            if out >= 0:
+                fixed.append((out, NATURAL))
+        elif kind == NODE_ATTENTION:
+            want.append((ins[0], NATURAL))
+            want.append((ins[1], NATURAL))
+            if out >= 0 and edge_dims[ins[2]] != edge_dims[out]:
+                want.append((ins[2], NATURAL))
+                fixed.append((out, NATURAL))
+        elif kind == NODE_SOURCE_FIXED:
+            fixed.append((out, NATURAL))
+    return want, fixed
+
+
+def basis_keys(perms):
+    """key[i]: NATURAL if permutation i is the identity, else the smallest id
+    whose permutation has the same contents (equal bases compare equal)."""
+    keys, seen = [], {}
+    for i, p in enumerate(perms):
+        p = np.asarray(p)
+        if np.array_equal(p, np.arange(len(p))):
+            keys.append(NATURAL)
+            continue
+        t = tuple(int(v) for v in p)
+        keys.append(seen.setdefault(t, i))
+    return keys
+
+
+def _key(keys, w):
+    return NATURAL if w == NATURAL else keys[w]
+
+
+def plan_cost(nodes, edge_dims, labels, perms, only_region=None, region=None, keys=None):
+    """Modelled bytes per token of the explicit shuffles a labelling needs
+    (R17): one shuffle per distinct (edge, wanted basis) that differs from
+    the edge's label, and one per fixed producer whose basis differs;
+    optionally only for the edges of one region."""
+    keys = basis_keys(perms) if keys is None else keys
+    want, fixed = _requests(nodes, edge_dims)
+    if only_region is not None:
+        want = [(e, w) for e, w in want if region[e] == only_region]
+        fixed = [(e, w) for e, w in fixed if region[e] == only_region]
+    need = set()
+    for e, w in want:
+        if _key(keys, labels[e]) != _key(keys, w):
+            need.add((e, _key(keys, w)))
+    cost = 4 * sum(edge_dims[e] for e, _ in need)
+    for e, w in fixed:
+        if _key(keys, labels[e]) != _key(keys, w):
+            cost += 4 * edge_dims[e]
+    return cost
+
+
+def plan_graph(nodes, edge_dims, perms):
+    """§4.4 planning (R17): the basis label of every edge.  ``nodes`` are
+    (kind, inputs, output edge or -1, permutation id or -1), ``perms[i]``
+    a linear's preferred input order (its clustering permutation).  Returns
+    (labels, modelled bytes per token)."""
+    keys = basis_keys(perms)
+    region = plan_regions(nodes, edge_dims)
+    want, _ = _requests(nodes, edge_dims)
+    labels = [NATURAL] * len(edge_dims)
+    for r in sorted(set(region)):
+        edges = [e for e in range(len(edge_dims)) if region[e] == r]
+        cands = [NATURAL] + sorted({keys[w] for e, w in want
+                                    if region[e] == r and w != NATURAL and keys[w] != NATURAL})
+        best = None
+        for c in cands:
+            for e in edges:
+                labels[e] = c
+            cost = plan_cost(nodes, edge_dims, labels, perms, only_region=r, region=region,
+                             keys=keys)
+            if best is None or cost < best[0]:
+                best = (cost, c)
+        for e in edges:
+            labels[e] = best[1]
+    return labels, plan_cost(nodes, edge_dims, labels, perms, keys=keys)
+
+
+def no_merge_traffic(nodes, edge_dims):
+    """The per-layer-gather baseline of §5.3: every linear input shuffled."""
+    return 4 * sum(edge_dims[i[0]] for k, i, o, p in nodes if k == NODE_LINEAR)
+
+
+def decoder_graph(n_layers, hidden, ffn, kv=None, perm_ids=None, qdim=None):
+    """The decode graph of a Llama/Qwen-style stack (R11 per layer, R17
+    kinds): nodes, edge widths and, per layer, the edge ids by name.  ``qdim``
+    is the width of q and of the attention output (heads x head width,
+    default ``hidden``), ``kv`` the k/v width (grouped-query attention when
+    below ``qdim``);
+    ``perm_ids(layer, name)`` gives each linear's permutation id.  The
+    stream enters from a fixed natural source and leaves through a boundary
+    (the output head reads natural order)."""
+    qdim = hidden if qdim is None else qdim
+    kv = qdim if kv is None else kv
+    nodes, dims, names = [], [], []
+
+    def edge(d):
+        dims.append(d)
+        return len(dims) - 1
+
+    s = edge(hidden)
+    nodes.append((NODE_SOURCE_FIXED, [], s, -1))
+    for l in range(n_layers):
+        e = {}
+        e["h"] = edge(hidden)
+        nodes.append((NODE_ELEMENTWISE, [s], e["h"], -1))           # RMSNorm
+        for nm, w in (("q", qdim), ("k", kv), ("v", kv)):
+            e[nm] = edge(w)
+            nodes.append((NODE_LINEAR, [e["h"]], e[nm], perm_ids(l, nm)))
+        e["att"] = edge(qdim)
+        nodes.append((NODE_ATTENTION, [e["q"], e["k"], e["v"]], e["att"], -1))
+        e["o"] = edge(hidden)
+        nodes.append((NODE_LINEAR, [e["att"]], e["o"], perm_ids(l, "o")))
+        e["s1"] = edge(hidden)
+        nodes.append((NODE_ELEMENTWISE, [s, e["o"]], e["s1"], -1))  # residual add
+        e["h2"] = edge(hidden)
+        nodes.append((NODE_ELEMENTWISE, [e["s1"]], e["h2"], -1))    # RMSNorm
+        for nm in ("gate", "up"):
+            e[nm] = edge(ffn)
+            nodes.append((NODE_LINEAR, [e["h2"]], e[nm], perm_ids(l, nm)))
+        e["m"] = edge(ffn)
+        nodes.append((NODE_ELEMENTWISE, [e["gate"], e["up"]], e["m"], -1))  # SiLU * up
+        e["down"] = edge(hidden)
+        nodes.append((NODE_LINEAR, [e["m"]], e["down"], perm_ids(l, "down")))
+        e["s2"] = edge(hidden)
+        nodes.append((NODE_ELEMENTWISE, [e["s1"], e["down"]], e["s2"], -1))
+        e["s_in"] = s
+        names.append(e)
+        s = e["s2"]
+    nodes.append((NODE_BOUNDARY, [s], -1, -1))
+    return nodes, dims, names
+
+
+DECODER_LINEAR_EDGES = (("q", "h", "q"), ("k", "h", "k"), ("v", "h", "v"), ("o", "att", "o"),
+                        ("gate", "h2", "gate"), ("up", "h2", "up"), ("down", "m", "down"))
+"""(linear, input edge, output edge) of one layer of ``decoder_graph``."""
+
+
+def merge_from_labels(lin, edges, labels, perms):
+    """The §4.3 merges a plan implies for one decoder layer (R17): each
+    linear's rows are permuted to its output edge's basis and it gathers from
+    its input edge's basis (gather None where that is its own order).
+    ``lin`` maps names to packed layers, ``edges`` is the layer's entry of
+    ``decoder_graph``'s names, ``labels`` and ``perms`` come from
+    ``plan_graph``; the result has merge_decoder_layer's form."""
+    def basis(e):
+        lab = labels[e]
+        return None if lab == NATURAL else np.asarray(perms[lab])
+
+    out = {}
+    for nm, ein, eout in DECODER_LINEAR_EDGES:
+        L = lin[nm]
+        bo = basis(edges[eout])
+        if bo is not None:
+            L = permute_rows(L, bo)
+        bi = basis(edges[ein])
+        g = L["perm"] if bi is None else permute_merge(bi, L["perm"])
+        if np.array_equal(g, np.arange(len(g))):
+            g = None
+        out[nm] = (L, g)
+    return out

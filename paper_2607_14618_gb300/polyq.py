@@ -75,6 +75,15 @@ class GemvInput(C.Structure):
                 ("x_out", C.c_void_p)]
 
 
+NODE_SOURCE_FIXED, NODE_SOURCE_FREE, NODE_LINEAR, NODE_ELEMENTWISE, NODE_BOUNDARY, \
+    NODE_ATTENTION = range(6)
+
+
+class PlanNode(C.Structure):
+    _fields_ = [("kind", C.c_int32), ("n_in", C.c_int32), ("in_", C.c_int32 * 3),
+                ("out", C.c_int32), ("perm", C.c_int32)]
+
+
 class DevLayer(C.Structure):
     _fields_ = [("packed", C.c_void_p), ("meta", C.c_void_p), ("gather", C.c_void_p),
                 ("N", C.c_int64), ("K", C.c_int64), ("row_stride", C.c_int64),
@@ -94,6 +103,9 @@ _SIGS = {
     "polyq_layer_xscale": (C.c_int, [_P, _P]),
     "polyq_layer_permute_rows": (C.c_int, [_P, _P]),
     "polyq_permute_merge": (C.c_int, [_P, _P, C.c_int64, _P]),
+    "polyq_plan_graph": (C.c_int, [C.POINTER(PlanNode), C.c_int32, _P, C.c_int32,
+                                   C.POINTER(C.c_void_p), _P, C.c_int32, _P,
+                                   C.POINTER(C.c_int64)]),
     "polyq_dev_layer_fill": (C.c_int, [_P, _P, _P, _P, C.POINTER(DevLayer)]),
     "polyq_gemv_workspace_bytes": (C.c_int, [C.POINTER(DevLayer), C.c_int, C.POINTER(C.c_size_t)]),
     "polyq_linear_gemv": (C.c_int, [C.POINTER(DevLayer), _P, C.c_int, _P, _P, _P, C.c_size_t, _P]),
@@ -147,6 +159,29 @@ def permute_merge(producer_basis, consumer_perm):
     out = np.empty_like(c)
     _check(_lib.polyq_permute_merge(b.ctypes.data, c.ctypes.data, c.shape[0], out.ctypes.data))
     return out
+
+
+def plan_graph(nodes, edge_dims, perms):
+    """Section 4.4 planning: ``nodes`` as (kind, input edges, output edge or
+    -1, permutation id or -1), ``perms`` the linears' permutations.  Returns
+    (labels [n_edges] int32, -1 = natural order, modelled bytes per token)."""
+    arr = (PlanNode * len(nodes))()
+    for i, (kind, ins, out, perm) in enumerate(nodes):
+        arr[i].kind = int(kind)
+        arr[i].n_in = len(ins)
+        for j, e in enumerate(ins):
+            arr[i].in_[j] = int(e)
+        arr[i].out = int(out)
+        arr[i].perm = int(perm)
+    dims = np.ascontiguousarray(edge_dims, dtype=np.int64)
+    keep = [np.ascontiguousarray(p, dtype=np.int32) for p in perms]
+    ptrs = (C.c_void_p * max(1, len(keep)))(*[k.ctypes.data for k in keep])
+    lens = np.array([len(k) for k in keep] or [0], dtype=np.int64)
+    labels = np.empty(len(dims), np.int32)
+    cost = C.c_int64()
+    _check(_lib.polyq_plan_graph(arr, len(nodes), dims.ctypes.data, len(dims), ptrs,
+                                 lens.ctypes.data, len(keep), labels.ctypes.data, C.byref(cost)))
+    return labels, int(cost.value)
 
 
 def _palette_mask(palette):
@@ -464,3 +499,49 @@ def gemv_launches_per_call(layer: DeviceLayer, batch: int) -> int:
     """Kernels one polyq_linear_gemv (or _group) call enqueues: the activation
     record pre-pass and the streaming kernel."""
     return 2
+
+
+def decoder_plan_graph(n_layers, hidden, ffn, perm_of, kv=None, qdim=None):
+    """Planner input for a decoder stack's decode step: per layer RMSNorm ->
+    q, k, v -> attention -> o -> residual add -> RMSNorm -> gate, up ->
+    SiLU * up -> down -> residual add; the stream enters in natural order and
+    leaves through a natural-order boundary.  ``perm_of(layer, name)``
+    returns the permutation id of each linear.  Returns (nodes, edge widths,
+    per-layer edge ids by name)."""
+    qdim = hidden if qdim is None else qdim
+    kv = qdim if kv is None else kv
+    nodes, dims, names = [], [], []
+
+    def edge(w):
+        dims.append(w)
+        return len(dims) - 1
+
+    s = edge(hidden)
+    nodes.append((NODE_SOURCE_FIXED, [], s, -1))
+    for l in range(n_layers):
+        e = {"s_in": s, "h": edge(hidden)}
+        nodes.append((NODE_ELEMENTWISE, [s], e["h"], -1))
+        for nm, w in (("q", qdim), ("k", kv), ("v", kv)):
+            e[nm] = edge(w)
+            nodes.append((NODE_LINEAR, [e["h"]], e[nm], perm_of(l, nm)))
+        e["att"] = edge(qdim)
+        nodes.append((NODE_ATTENTION, [e["q"], e["k"], e["v"]], e["att"], -1))
+        e["o"] = edge(hidden)
+        nodes.append((NODE_LINEAR, [e["att"]], e["o"], perm_of(l, "o")))
+        e["s1"] = edge(hidden)
+        nodes.append((NODE_ELEMENTWISE, [s, e["o"]], e["s1"], -1))
+        e["h2"] = edge(hidden)
+        nodes.append((NODE_ELEMENTWISE, [e["s1"]], e["h2"], -1))
+        for nm in ("gate", "up"):
+            e[nm] = edge(ffn)
+            nodes.append((NODE_LINEAR, [e["h2"]], e[nm], perm_of(l, nm)))
+        e["m"] = edge(ffn)
+        nodes.append((NODE_ELEMENTWISE, [e["gate"], e["up"]], e["m"], -1))
+        e["down"] = edge(hidden)
+        nodes.append((NODE_LINEAR, [e["m"]], e["down"], perm_of(l, "down")))
+        e["s2"] = edge(hidden)
+        nodes.append((NODE_ELEMENTWISE, [e["s1"], e["down"]], e["s2"], -1))
+        names.append(e)
+        s = e["s2"]
+    nodes.append((NODE_BOUNDARY, [s], -1, -1))
+    return nodes, dims, names
