@@ -341,6 +341,7 @@ def run_polyq(args):
             "prefill_gemm": gemm,
             "decode_step": decode,
             "permutation_plan": plan_report(polyq),
+            "quanta_matching": quanta_report(polyq, synth),
         }
         print(json.dumps(out), flush=True)
     if ws > 1:
@@ -507,6 +508,30 @@ def plan_report(polyq):
         res["paper_no_merge_mib"] = c["paper_no_merge_mib"]
         res["paper_polyq_mib"] = c["paper_polyq_mib"]
         out[name] = res
+    return out
+
+
+def quanta_report(polyq, synth):
+    """§3.3 quanta matching on the synthetic layer generator (host, no GPU):
+    realised mean width and segment padding before and after snapping to
+    the GPU quanta (one 16-byte chunk per quantum), over the §5.2 budget
+    sweep, for the input widths of the Llama2-13B and Qwen3-32B linears
+    (256 rows each: the allocation depends on the rows only through the
+    column norms)."""
+    out = {}
+    for K in (5120, 8192, 13824, 25600):
+        W, a = synth.layer_weights(256, K, 40000 + K)
+        rows = []
+        for B in (3.0, 3.5, 4.0, 4.5, 5.0, 5.5, 6.0):
+            raw = polyq.HostLayer.pack(W, a, B).info()
+            snap = polyq.HostLayer.pack(W, a, B, snap_quanta=True).info()
+            rows.append({"B": B, "b_real_raw": round(raw["b_real"], 5),
+                         "b_real_snapped": round(snap["b_real"], 5),
+                         "pad_pct_raw": round(100 * raw["pad_bytes"] / raw["row_stride"], 3),
+                         "pad_pct_snapped": round(100 * snap["pad_bytes"] / snap["row_stride"], 3)})
+        out[f"K{K}"] = {"max_abs_mismatch": round(max(abs(r["b_real_snapped"] - r["B"])
+                                                      for r in rows), 5),
+                        "sweep": rows}
     return out
 
 
