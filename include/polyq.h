@@ -401,6 +401,74 @@ int polyq_linear_gemv_input(const polyq_dev_layer* const* layers, int n,
                             const float* const* residuals, void* workspace,
                             size_t workspace_bytes, void* stream);
 
+/* ---- chained decode GEMVs in one persistent launch ----
+ * A decoder's decode step is a chain of dependent GEMV phases (q/k/v, o,
+ * gate/up, down, then the next layer's q/k/v, ...), each the product of
+ * Section 4.1 for one to four layers that share an input.  A chain runs all
+ * of its phases in one launch: one CTA per resident slot (three per SM)
+ * streams the packed weights of every phase through its TMA ring without
+ * stopping at phase boundaries, while its consumer warps wait at a grid-wide
+ * barrier between phases (phase p+1 reads what phase p wrote), then gather
+ * their activation records in shared memory and continue.  Work items of a
+ * phase are (layer, step, 64-row tile) in step-major order, split into
+ * contiguous ranges of equal modelled cost; each item adds its rows into y
+ * with fp32 atomics (the order of those additions varies from run to run).
+ * Every device-side wait is bounded; on a timeout the kernel records a
+ * status and returns. */
+typedef struct polyq_gemv_chain polyq_gemv_chain; /* opaque, host-owned */
+
+typedef struct {
+  int32_t n_layers;                              /* 1..POLYQ_MAX_GROUP */
+  const polyq_dev_layer* layers[POLYQ_MAX_GROUP];
+  polyq_gemv_input in;    /* the phase's input and its transform (as for
+                             polyq_linear_gemv_input); with POLYQ_X_BF16 a
+                             non-NULL xs[i] overrides in.a for layer i */
+  const void* xs[POLYQ_MAX_GROUP];
+  float* ys[POLYQ_MAX_GROUP];                    /* fp32 [batch][N_i] */
+  const float* residuals[POLYQ_MAX_GROUP];       /* NULL = none; may equal ys[i] */
+} polyq_gemv_phase;
+
+/* Scratch every chained launch needs: a status word and the grid-barrier
+ * counters.  Zero-filled before first use; a launch leaves it zeroed unless
+ * it reports a timeout (then zero it again). */
+#define POLYQ_CHAIN_WORKSPACE_BYTES 256u
+
+/* Build a chain of n_phases phases (1..65536) at one batch size (1..4).
+ * The phase descriptors and the layer descriptors are copied (device memory
+ * they point to must stay valid while the chain is used).  Rules, checked
+ * here (POLYQ_EINVAL):
+ *   - every layer of a phase has the phase input's width K;
+ *   - a phase's outputs do not overlap its inputs (a residual may be the
+ *     output itself: y += W'x in place);
+ *   - the outputs of phase p+1 other than in-place ones overlap nothing that
+ *     phase p reads or writes (they are initialised while phase p runs).
+ * *out owns a host plan; upload it to device memory with
+ * polyq_gemv_chain_upload before launching. */
+int polyq_gemv_chain_create(const polyq_gemv_phase* phases, int n_phases, int batch,
+                            polyq_gemv_chain** out);
+
+/* Bytes of device memory the chain's plan needs (tensor maps, block tables
+ * and per-CTA work ranges for the current device). */
+int polyq_gemv_chain_plan_bytes(const polyq_gemv_chain* chain, size_t* bytes);
+
+/* Copy the plan into plan_dev (device memory of at least
+ * polyq_gemv_chain_plan_bytes, owned by the caller) with a
+ * copy on `stream` (the call waits for it); the chain then launches from
+ * plan_dev.  plan_dev must be 128-byte aligned. */
+int polyq_gemv_chain_upload(polyq_gemv_chain* chain, void* plan_dev, size_t bytes,
+                            void* stream);
+
+/* Run every phase of the chain, in order, in one cooperative launch on
+ * `stream`.  workspace: device, 256-byte aligned, at least
+ * POLYQ_CHAIN_WORKSPACE_BYTES, zero-filled before first use; one workspace
+ * serves consecutive launches on one stream but not launches that run at the
+ * same time.  Launch errors (including a device that cannot hold every CTA
+ * at once) are POLYQ_ECUDA. */
+int polyq_linear_gemv_chain(const polyq_gemv_chain* chain, void* workspace,
+                            size_t workspace_bytes, void* stream);
+
+void polyq_gemv_chain_free(polyq_gemv_chain* chain);
+
 /* Device scratch bytes polyq_linear_gemm needs for this layer and M. */
 int polyq_gemm_workspace_bytes(const polyq_dev_layer* layer, int64_t M,
                                size_t* bytes);

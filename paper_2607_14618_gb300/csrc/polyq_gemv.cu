@@ -41,6 +41,7 @@
 
 #include "polyq.h"
 #include "polyq_dev.cuh"
+#include "polyq_gemv_dev.cuh"
 #include "polyq_gemv_layout.cuh"
 #include "polyq_internal.h"
 
@@ -51,14 +52,7 @@ using namespace polyq::gv;
 
 constexpr int kCtasPerSm = 3;
 constexpr int kMaxGrid = 1024;  // persistent CTAs at most
-constexpr int kThreads = 32 * (kWarps + 1);
-constexpr int kConsumers = 32 * kWarps;
 
-struct GvBlock {
-  int bits, n_ch, pos0, seg_off, grp_off;
-  int step0, n_steps;  // step range of this block inside its layer
-  int units;           // units per step
-};
 
 // One layer of a call.  Tensor maps first (64-byte aligned).
 struct GvLayer {
@@ -199,94 +193,6 @@ __device__ __forceinline__ int layer_K(const GvParams& P, int l) {
 }
 
 
-__device__ __forceinline__ uint32_t pack_half2(__half lo, __half hi) {
-  return (uint32_t)__half_as_ushort(lo) | ((uint32_t)__half_as_ushort(hi) << 16);
-}
-
-// ---------------------------------------------------------------------------
-// activation records (consumer warps, shared memory)
-// ---------------------------------------------------------------------------
-// Which activation values one consumer thread contributes to a record.  A
-// record has at most two slots per thread:
-//  * b < 16: slot s is the (batch, chunk) pair bc = warp + 4s of the step;
-//    lane q of the warp makes the q-th of the chunk's 32 lane pairs.
-//  * 16-bit: slot s is entry e = tid + 128s of the [batch][lane][16] pairs.
-struct SlotGeom {
-  bool valid;
-  int bb, c, t, jp;
-  int ch[2];  // channels (inside the block) of the pair's low and high half
-  int p[2];   // power-of-two scale exponents of the two halves
-};
-
-template <int NB, int BITS>
-__device__ __forceinline__ SlotGeom slot_geom_t(int warp, int lane, int tid, int s, int j,
-                                                const uint32_t* p3) {
-  SlotGeom g;
-  if constexpr (BITS == 16) {
-    const int e = tid + kConsumers * s;
-    g.valid = e < NB * 64;
-    g.bb = e / 64;
-    g.t = (e / 16) % 4;
-    g.jp = e % 16;
-    g.c = 0;
-    g.ch[0] = j * 128 + lane_weight16(g.t, 2 * g.jp);
-    g.ch[1] = j * 128 + lane_weight16(g.t, 2 * g.jp + 1);
-    g.p[0] = g.p[1] = 0;
-  } else {
-    constexpr int U = step_units(BITS, NB), NGS = U / 64;
-    constexpr int GP = group_pairs(BITS), GU = group_units(BITS);
-    const int bc = warp + kWarps * s;
-    g.valid = bc < NB * NGS;
-    g.bb = bc / NGS;
-    g.c = bc - g.bb * NGS;
-    chunk_pair(BITS, NB, g.c, lane, &g.t, &g.jp);
-    const int jj = g.jp % GP, base = (g.jp / GP) * GU;
-    int lo, hi;
-    if constexpr (BITS == 3) {
-      const uint32_t e = p3[jj];  // lo | hi << 8 | (win + 16) << 16
-      lo = (int)(e & 0xFF);
-      hi = (int)((e >> 8) & 0xFF);
-      const int win = (int)(e >> 16) - 16;
-      g.p[0] = 3 * lo - win;
-      g.p[1] = 3 * hi - win - 16;
-    } else {
-      const PairDef d = pair_def(BITS, jj);
-      lo = d.lo;
-      hi = d.hi;
-      g.p[0] = d.plo;
-      g.p[1] = d.phi;
-    }
-    g.ch[0] = j * U + lane_unit(BITS, NB, g.t, base + lo);
-    g.ch[1] = j * U + lane_unit(BITS, NB, g.t, base + hi);
-  }
-  return g;
-}
-
-template <int NB>
-__device__ __forceinline__ SlotGeom slot_geom(int bits, int warp, int lane, int tid, int s,
-                                              int j, const uint32_t* p3) {
-  switch (bits) {
-    case 2: return slot_geom_t<NB, 2>(warp, lane, tid, s, j, p3);
-    case 3: return slot_geom_t<NB, 3>(warp, lane, tid, s, j, p3);
-    case 4: return slot_geom_t<NB, 4>(warp, lane, tid, s, j, p3);
-    case 8: return slot_geom_t<NB, 8>(warp, lane, tid, s, j, p3);
-    default: return slot_geom_t<NB, 16>(warp, lane, tid, s, j, p3);
-  }
-}
-
-// Where a record's activations come from: the layer's input (bf16 x, or the
-// fp32 inputs of a fused transform), its gather vector, its activation
-// factors and its width K.
-struct XIn {
-  const __nv_bfloat16* x;
-  const float* xa;
-  const float* xb;
-  uint16_t* xout;  // written when not NULL
-  const int32_t* gather;
-  const float* xscale;
-  int kind, K, batch;
-};
-
 __device__ __forceinline__ XIn xin_of(const GvParams& P, int l) {
   XIn in;
   in.x = layer_x(P, l);
@@ -301,95 +207,6 @@ __device__ __forceinline__ XIn xin_of(const GvParams& P, int l) {
   return in;
 }
 
-// Pass 1 of a record: the gather indices and activation factors (static
-// layer data, so this may run before the grid-dependency wait).
-template <int NB>
-__device__ __forceinline__ void rec_sources(const XIn& in, const GvBlock& B, int j, int warp,
-                                            int lane, const uint32_t* p3, int (&src)[2][2],
-                                            float (&fac)[2][2]) {
-  const int32_t* gather = in.gather;
-#pragma unroll
-  for (int s = 0; s < 2; ++s) {
-    src[s][0] = src[s][1] = -1;
-    fac[s][0] = fac[s][1] = 1.f;
-    const SlotGeom g = slot_geom<NB>(B.bits, warp, lane, threadIdx.x, s, j, p3);
-    if (g.valid && g.bb < in.batch) {
-#pragma unroll
-      for (int h = 0; h < 2; ++h)
-        if (g.ch[h] < B.n_ch) {
-          const int p = B.pos0 + g.ch[h];
-          src[s][h] = gather ? __ldg(gather + p) : p;
-          if (in.xscale) fac[s][h] = __ldg(in.xscale + p);
-        }
-    }
-  }
-}
-
-// Passes 2 and 3: load the activations, scale, round to fp16, store the
-// pairs and (b < 16) the per-chunk sums C1 = 1024 * sum x' and X = sum x.
-template <int NB>
-__device__ __forceinline__ void rec_build(const XIn& in, const GvBlock& B, int j, int warp,
-                                          int lane, const uint32_t* p3, const int (&src)[2][2],
-                                          const float (&fac)[2][2], const float* rnorm,
-                                          uint32_t* rec) {
-  constexpr int LW = rec_lane_words(NB);
-  constexpr int PW = rec_pair_words(NB);
-  constexpr int NGM = 8 / NB;
-  const __nv_bfloat16* x = in.x;
-  const int K = in.K;
-  float xv[2][2];
-#pragma unroll
-  for (int s = 0; s < 2; ++s) {
-    const SlotGeom g = slot_geom<NB>(B.bits, warp, lane, threadIdx.x, s, j, p3);
-#pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      if (src[s][h] < 0) {
-        xv[s][h] = 0.f;
-        continue;
-      }
-      const size_t o = (size_t)g.bb * K + src[s][h];
-      __nv_bfloat16 v;
-      switch (in.kind) {
-        case POLYQ_X_F32: v = __float2bfloat16_rn(in.xa[o]); break;
-        case POLYQ_X_RMSNORM: v = __float2bfloat16_rn(in.xa[o] * rnorm[g.bb]); break;
-        case POLYQ_X_SILU_MUL: {
-          const float a = in.xa[o];
-          v = __float2bfloat16_rn(a / (1.f + expf(-a)) * in.xb[o]);
-          break;
-        }
-        default: v = x[o]; break;
-      }
-      if (in.xout) in.xout[o] = __bfloat16_as_ushort(v);
-      xv[s][h] = __bfloat162float(v) * fac[s][h];  // Section 3.4 factor (1 if none)
-    }
-  }
-  float* recf = reinterpret_cast<float*>(rec);
-#pragma unroll
-  for (int s = 0; s < 2; ++s) {
-    const SlotGeom g = slot_geom<NB>(B.bits, warp, lane, threadIdx.x, s, j, p3);
-    if (!g.valid) continue;  // uniform over the warp for b < 16
-    const __half hlo = __float2half_rn(ldexpf(xv[s][0], -g.p[0]));
-    const __half hhi = __float2half_rn(ldexpf(xv[s][1], -g.p[1]));
-    rec[(g.bb * 4 + g.t) * LW + g.jp] = pack_half2(hlo, hhi);
-    if (B.bits != 16) {
-      // X sums the values the MMA multiplies (fp16 times 2^p), so that the
-      // zero-point term removes exactly what the codes' z adds; with
-      // activation factors these differ from the fp32 products x * t
-      float s1 = __half2float(hlo) + __half2float(hhi);
-      float s2 = ldexpf(__half2float(hlo), g.p[0]) + ldexpf(__half2float(hhi), g.p[1]);
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        s1 += __shfl_xor_sync(0xffffffffu, s1, o);
-        s2 += __shfl_xor_sync(0xffffffffu, s2, o);
-      }
-      if (lane == 0) {
-        recf[PW + g.bb * NGM + g.c] = kMagicF * s1;
-        recf[PW + NB * NGM + g.bb * NGM + g.c] = s2;
-      }
-    }
-  }
-}
-
 // Layer, block and block step of record r.
 __device__ __forceinline__ void rec_pos(const GvShared& S, int nl, int r, int* l, int* bi,
                                         int* j) {
@@ -401,200 +218,6 @@ __device__ __forceinline__ void rec_pos(const GvShared& S, int nl, int r, int* l
   *l = q;
   *bi = b;
   *j = s - S.blk[q][b].step0;
-}
-
-// ---------------------------------------------------------------------------
-// MMA steps
-// ---------------------------------------------------------------------------
-template <int BITS>
-__device__ __forceinline__ uint32_t window(const uint32_t* w, int off) {
-  // bits [off, off+32) of the little-endian stream held in w[]
-  if (off < 0) return w[0] << (-off);
-  const int k = off >> 5, r = off & 31;
-  if (r == 0) return w[k];
-  if (k + 1 >= group_words(BITS)) return w[k] >> r;
-  return __funnelshift_r(w[k], w[k + 1], r);
-}
-
-// Pair register for lane pair j of one row's words: one LOP3 with the mask
-// as its immediate and `magic` in a register, plus the window's shift, which
-// the pairs sharing a window share.
-template <int BITS>
-__device__ __forceinline__ uint32_t make_pair(const uint32_t* words, int j, uint32_t magic) {
-  constexpr int GP = group_pairs(BITS);
-  constexpr int GW = group_words(BITS);
-  constexpr uint32_t QM = (1u << BITS) - 1u;
-  const PairDef d = pair_def(BITS, j % GP);
-  const uint32_t* g = words + (j / GP) * GW;
-  const uint32_t win = window<BITS>(g, d.win);
-  const uint32_t m = (QM << d.plo) | ((QM << d.phi) << 16);
-  return lop3_and_or(win, m, magic);
-}
-
-// Load the lane's words of tile row r from the stage's codes area (box h at
-// h * 64 rows * pitch, row r at r * pitch, lane t at t * LB).
-template <int BITS, int NB>
-__device__ __forceinline__ void load_words(uint32_t* w, const uint8_t* codes, int r, int t) {
-  constexpr int NBX = nbox_of(BITS, NB);
-  constexpr int PITCH = box_pitch(BITS, NB);
-  constexpr int LB = lane_box_bytes(BITS, NB);
-  constexpr int WPB = LB / 4;
-#pragma unroll
-  for (int h = 0; h < NBX; ++h) {
-    const uint8_t* p = codes + h * kRows * PITCH + r * PITCH + t * LB;
-    uint32_t* o = w + h * WPB;
-    if constexpr (LB % 16 == 0) {
-#pragma unroll
-      for (int k = 0; k < WPB / 4; ++k) {
-        const uint4 a = reinterpret_cast<const uint4*>(p)[k];
-        o[4 * k] = a.x; o[4 * k + 1] = a.y; o[4 * k + 2] = a.z; o[4 * k + 3] = a.w;
-      }
-    } else if constexpr (LB % 8 == 0) {
-#pragma unroll
-      for (int k = 0; k < WPB / 2; ++k) {
-        const uint2 a = reinterpret_cast<const uint2*>(p)[k];
-        o[2 * k] = a.x; o[2 * k + 1] = a.y;
-      }
-    } else {
-#pragma unroll
-      for (int k = 0; k < WPB; ++k) o[k] = reinterpret_cast<const uint32_t*>(p)[k];
-    }
-  }
-}
-
-// One step of a b<16 block for this warp's 16 rows; adds the chunk results,
-// scaled, into acc[row][batch].
-template <int NB, int BITS>
-__device__ __forceinline__ void step_mma(uint32_t magic, int batch, int uvalid, int g0,
-                                         const uint8_t* stage, const uint32_t* rec,
-                                         const uint32_t* zeros, int warp, int lane,
-                                         float (&acc)[2][NB]) {
-  constexpr int U = step_units(BITS, NB);
-  constexpr int NGS = step_chunks(BITS, NB);
-  constexpr int NGM = 8 / NB;
-  constexpr int NW = lane_words(BITS, NB);
-  constexpr int LW = rec_lane_words(NB);
-  constexpr int PW = rec_pair_words(NB);
-  constexpr int GP = group_pairs(BITS), GW = group_words(BITS);
-  constexpr int NBX = nbox_of(BITS, NB);
-  constexpr int GPB = NW / GW / NBX;      // groups per box
-  constexpr int CPB = U / NBX / 64;       // chunks per box
-  static_assert(GP % 4 == 0 && GPB * GW * NBX == NW, "step geometry");
-  const int g = lane >> 2, t = lane & 3;
-  const int rA = warp * 16 + g, rB = rA + 8;
-  const uint32_t* meta_s = reinterpret_cast<const uint32_t*>(stage + kCodesBytes);
-
-  uint32_t wa[NW], wb[NW];
-  load_words<BITS, NB>(wa, stage, rA, t);
-  load_words<BITS, NB>(wb, stage, rB, t);
-
-  // Column g of the B fragment is (batch my_b, chunk my_c); lane t's codes in
-  // box h belong to chunk c_t + h*CPB, so only a matching lane loads its
-  // activations, the others read zeros.
-  const int my_b = g / NGS, my_c = g % NGS;
-  const int dc = my_b < batch ? my_c - lane_unit(BITS, NB, t, 0) / 64 : -1000;
-  const uint32_t* brow = rec + (my_b * 4 + t) * LW;
-
-  float d[4][4];
-#pragma unroll
-  for (int q = 0; q < 4; ++q) d[q][0] = d[q][1] = d[q][2] = d[q][3] = 0.f;
-#pragma unroll
-  for (int h = 0; h < NBX; ++h) {
-    if (h == 1 && uvalid <= U / 2) break;  // the second half of the step is empty
-    const uint32_t* bsrc = dc == h * CPB ? brow + h * GPB * GP : zeros;
-#pragma unroll
-    for (int qq = 0; qq < GPB; ++qq) {
-      const int q = h * GPB + qq;
-#pragma unroll
-      for (int m2 = 0; m2 < GP / 4; ++m2) {  // two MMAs per 16-byte activation load
-        const uint4 bv = *reinterpret_cast<const uint4*>(bsrc + qq * GP + 4 * m2);
-#pragma unroll
-        for (int hh = 0; hh < 2; ++hh) {
-          const int jp = q * GP + 4 * m2 + 2 * hh;  // lane pair index
-          const uint32_t a0 = make_pair<BITS>(wa, jp, magic);
-          const uint32_t a1 = make_pair<BITS>(wb, jp, magic);
-          const uint32_t a2 = make_pair<BITS>(wa, jp + 1, magic);
-          const uint32_t a3 = make_pair<BITS>(wb, jp + 1, magic);
-          mma_f16_16816(d[(jp / 2) & 3], a0, a1, a2, a3, hh ? bv.z : bv.x, hh ? bv.w : bv.y);
-        }
-      }
-    }
-  }
-  float D[4];
-#pragma unroll
-  for (int v = 0; v < 4; ++v) D[v] = (d[0][v] + d[1][v]) + (d[2][v] + d[3][v]);
-
-  // epilogue: columns 2t, 2t+1 -> (batch, chunk) (col / NGS, col % NGS);
-  // g0 is the step's first group in the meta box
-  const float* recf = reinterpret_cast<const float*>(rec);
-#pragma unroll
-  for (int cc = 0; cc < 2; ++cc) {
-    const int col = 2 * t + cc;
-    const int be = col / NGS, c = col % NGS;
-    if (be < batch) {
-      const float C1 = recf[PW + be * NGM + c];
-      const float X = recf[PW + NB * NGM + be * NGM + c];
-#pragma unroll
-      for (int r = 0; r < 2; ++r) {
-        const uint32_t m = meta_s[(r ? rB : rA) * kMetaBox + g0 + c];
-        const float sc = __half2float(__ushort_as_half((uint16_t)(m & 0xFFFFu)));
-        const float ze = __half2float(__ushort_as_half((uint16_t)(m >> 16)));
-        const float v = sc * fmaf(-ze, X, D[2 * r + cc] - C1);
-#pragma unroll
-        for (int b = 0; b < NB; ++b)
-          if (b == be) acc[r][b] += v;
-      }
-    }
-  }
-}
-
-// One 16-bit step: the fp16 weights are the MMA's A operand as stored; column
-// n of B is batch row n.  Lane t holds weights [16t, 16t+16) of each of the
-// two 64-weight boxes.
-template <int NB>
-__device__ __forceinline__ void step_16(int batch, int uvalid,
-                                        const uint8_t* stage, const uint32_t* rec,
-                                        const uint32_t* zeros, int warp, int lane,
-                                        float (&acc)[2][NB]) {
-  constexpr int LW = rec_lane_words(NB);
-  constexpr int PITCH = kPitchSplit;
-  static_assert(box_pitch(16, NB) == PITCH && nbox_of(16, NB) == 2, "16-bit geometry");
-  const int g = lane >> 2, t = lane & 3;
-  const int rA = warp * 16 + g, rB = rA + 8;
-  const uint32_t* bsrc = g < batch ? rec + (g * 4 + t) * LW : zeros;
-  float d[2][4];
-#pragma unroll
-  for (int q = 0; q < 2; ++q) d[q][0] = d[q][1] = d[q][2] = d[q][3] = 0.f;
-#pragma unroll
-  for (int h = 0; h < 2; ++h) {
-    if (h == 1 && uvalid <= 64) break;
-    const uint4* pa = reinterpret_cast<const uint4*>(stage + h * kRows * PITCH + rA * PITCH + 32 * t);
-    const uint4* pb = reinterpret_cast<const uint4*>(stage + h * kRows * PITCH + rB * PITCH + 32 * t);
-    const uint4 a0 = pa[0], a1 = pa[1], b0 = pb[0], b1 = pb[1];
-    const uint32_t wa[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
-    const uint32_t wb[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
-#pragma unroll
-    for (int m2 = 0; m2 < 2; ++m2) {
-      const uint4 bv = *reinterpret_cast<const uint4*>(bsrc + 8 * h + 4 * m2);
-#pragma unroll
-      for (int hh = 0; hh < 2; ++hh) {
-        const int k = 4 * m2 + 2 * hh;
-        mma_f16_16816(d[hh], wa[k], wb[k], wa[k + 1], wb[k + 1], hh ? bv.z : bv.x,
-                      hh ? bv.w : bv.y);
-      }
-    }
-  }
-#pragma unroll
-  for (int cc = 0; cc < 2; ++cc) {
-    const int be = 2 * t + cc;
-#pragma unroll
-    for (int r = 0; r < 2; ++r) {
-      const float v = d[0][2 * r + cc] + d[1][2 * r + cc];
-#pragma unroll
-      for (int b = 0; b < NB; ++b)
-        if (b == be) acc[r][b] += v;
-    }
-  }
 }
 
 __device__ __forceinline__ void fence_proxy_async_global() {
@@ -624,30 +247,12 @@ __global__ void __launch_bounds__(kConsumers) gemv_prep(const __grid_constant__ 
   const XIn in = xin_of(P, l);
   rec_sources<NB>(in, S.blk[l][bi], j, warp, lane, s_p3, src, fac);  // static layer data
   pdl_wait();  // x comes from the previous kernel; the records and y may still be in use
+  float ra[2][2], rb[2][2];
+  rec_load<NB>(in, S.blk[l][bi], j, warp, lane, s_p3, src, ra, rb);
   __shared__ float s_rnorm[4];
-  if (P.xkind == POLYQ_X_RMSNORM) {
-    // 1 / sqrt(mean(a^2) + eps) of each batch row
-    __shared__ float s_part[4][kWarps];
-    const int K = P.L[0].K;
-    for (int bb = 0; bb < P.batch; ++bb) {
-      float acc = 0.f;
-      for (int i = threadIdx.x; i < K; i += kConsumers) {
-        const float v = P.xa[(size_t)bb * K + i];
-        acc = fmaf(v, v, acc);
-      }
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-      if (lane == 0) s_part[bb][warp] = acc;
-    }
-    __syncthreads();
-    if (threadIdx.x < P.batch) {
-      float t = 0.f;
-      for (int w = 0; w < kWarps; ++w) t += s_part[threadIdx.x][w];
-      s_rnorm[threadIdx.x] = rsqrtf(t / (float)K + P.eps);
-    }
-    __syncthreads();
-  }
-  rec_build<NB>(in, S.blk[l][bi], j, warp, lane, s_p3, src, fac, s_rnorm,
+  __shared__ float s_part[4][kWarps];
+  if (P.xkind == POLYQ_X_RMSNORM) rms_rnorm(P.xa, P.L[0].K, P.batch, P.eps, s_part, s_rnorm);
+  rec_store<NB>(in, S.blk[l][bi], j, warp, lane, s_p3, src, fac, ra, rb, s_rnorm,
                 reinterpret_cast<uint32_t*>(P.rec + (size_t)r * rec_bytes(NB)));
   // y starts as the residual (or zero); the main kernel adds its pieces
 #pragma unroll

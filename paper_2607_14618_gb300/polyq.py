@@ -91,6 +91,14 @@ class DevLayer(C.Structure):
                 ("blocks", Block * MAX_BLOCKS), ("xscale", C.c_void_p)]
 
 
+class GemvPhase(C.Structure):
+    _fields_ = [("n_layers", C.c_int32), ("layers", C.POINTER(DevLayer) * MAX_GROUP),
+                ("in_", GemvInput), ("xs", C.c_void_p * MAX_GROUP),
+                ("ys", C.c_void_p * MAX_GROUP), ("residuals", C.c_void_p * MAX_GROUP)]
+
+
+CHAIN_WORKSPACE_BYTES = 256
+
 _P = C.c_void_p
 _SIGS = {
     "polyq_last_error": (C.c_char_p, []),
@@ -120,6 +128,12 @@ _SIGS = {
                                           C.POINTER(GemvInput), C.c_int,
                                           C.POINTER(C.c_void_p), C.POINTER(C.c_void_p),
                                           _P, C.c_size_t, _P]),
+    "polyq_gemv_chain_create": (C.c_int, [C.POINTER(GemvPhase), C.c_int, C.c_int,
+                                          C.POINTER(C.c_void_p)]),
+    "polyq_gemv_chain_plan_bytes": (C.c_int, [_P, C.POINTER(C.c_size_t)]),
+    "polyq_gemv_chain_upload": (C.c_int, [_P, _P, C.c_size_t, _P]),
+    "polyq_linear_gemv_chain": (C.c_int, [_P, _P, C.c_size_t, _P]),
+    "polyq_gemv_chain_free": (None, [_P]),
     "polyq_gemm_workspace_bytes": (C.c_int, [C.POINTER(DevLayer), C.c_int64,
                                              C.POINTER(C.c_size_t)]),
     "polyq_linear_gemm": (C.c_int, [C.POINTER(DevLayer), _P, C.c_int64, _P, _P, C.c_size_t, _P]),
@@ -545,3 +559,57 @@ def decoder_plan_graph(n_layers, hidden, ffn, perm_of, kv=None, qdim=None):
         s = e["s2"]
     nodes.append((NODE_BOUNDARY, [s], -1, -1))
     return nodes, dims, names
+
+
+class GemvChain:
+    """A chain of dependent GEMV phases run in one persistent launch
+    (polyq_linear_gemv_chain).  Each phase is a dict with ``layers`` (one to
+    four DeviceLayer reading one input), ``kind`` (X_BF16, X_F32, X_RMSNORM,
+    X_SILU_MUL), ``a`` (and ``b`` for X_SILU_MUL) CUDA tensors [batch][K],
+    ``ys`` fp32 CUDA tensors [batch][N], optional ``residuals``, ``eps``,
+    ``x_out`` and, for X_BF16, per-layer inputs ``xs``.  The tensors must
+    stay alive and in place while the chain is used."""
+
+    def __init__(self, phases, batch, stream=None):
+        import torch
+        self._keep = []
+        arr = (GemvPhase * len(phases))()
+        for i, ph in enumerate(phases):
+            layers = ph["layers"]
+            arr[i].n_layers = len(layers)
+            for j, L in enumerate(layers):
+                arr[i].layers[j] = C.pointer(L.desc)
+                self._keep.append(L)
+            kind = ph.get("kind", X_BF16)
+            a, b, xo = ph.get("a"), ph.get("b"), ph.get("x_out")
+            arr[i].in_ = GemvInput(kind, float(ph.get("eps", 1e-6)),
+                                   a.data_ptr() if a is not None else None,
+                                   b.data_ptr() if b is not None else None,
+                                   xo.data_ptr() if xo is not None else None)
+            for j, x in enumerate(ph.get("xs") or []):
+                arr[i].xs[j] = x.data_ptr() if x is not None else None
+            for j, y in enumerate(ph["ys"]):
+                arr[i].ys[j] = y.data_ptr()
+            for j, r in enumerate(ph.get("residuals") or []):
+                arr[i].residuals[j] = r.data_ptr() if r is not None else None
+            self._keep.append(ph)
+        h = C.c_void_p()
+        _check(_lib.polyq_gemv_chain_create(arr, len(phases), int(batch), C.byref(h)))
+        self._h = h
+        nbytes = C.c_size_t()
+        _check(_lib.polyq_gemv_chain_plan_bytes(self._h, C.byref(nbytes)))
+        self.plan = torch.empty(max(1, nbytes.value), dtype=torch.uint8, device="cuda")
+        _check(_lib.polyq_gemv_chain_upload(self._h, self.plan.data_ptr(), self.plan.numel(),
+                                            _stream_ptr(stream)))
+        self.workspace = torch.zeros(CHAIN_WORKSPACE_BYTES, dtype=torch.uint8, device="cuda")
+        self.n_phases = len(phases)
+
+    def run(self, stream=None, workspace=None):
+        ws = self.workspace if workspace is None else workspace
+        _check(_lib.polyq_linear_gemv_chain(self._h, ws.data_ptr(), ws.numel(),
+                                            _stream_ptr(stream)))
+
+    def __del__(self):
+        if getattr(self, "_h", None) and self._h.value:
+            _lib.polyq_gemv_chain_free(self._h)
+            self._h = C.c_void_p()

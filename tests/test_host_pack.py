@@ -335,3 +335,47 @@ def test_new_pack_options_are_validated(polyq_lib):
     assert rc == polyq_lib.POLYQ_EINVAL
     with pytest.raises(polyq_lib.PolyqError):
         polyq_lib.HostLayer.pack(W, None, 3.0, forced_bits=np.full(128, 3), act_scaling=True)
+
+
+def test_chain_overlap_rules_checked_before_any_device_work(polyq_lib):
+    """polyq_gemv_chain_create rejects hazards between and inside phases on
+    the host (fake, never dereferenced device addresses)."""
+    W, a = synth.layer_weights(64, 128, 3)
+    host = polyq_lib.HostLayer.pack(W, a, 3.0)
+    d = _desc_from(polyq_lib, host)
+    L = polyq_lib._lib
+    base = 0x10000000
+
+    def phase(x, y, res=None, kind=polyq_lib.X_F32):
+        ph = polyq_lib.GemvPhase()
+        ph.n_layers = 1
+        ph.layers[0] = C.pointer(d)
+        ph.in_ = polyq_lib.GemvInput(kind, 1e-6, x, None, None)
+        ph.ys[0] = y
+        ph.residuals[0] = res
+        return ph
+
+    def create(*phs):
+        arr = (polyq_lib.GemvPhase * len(phs))(*phs)
+        h = C.c_void_p()
+        rc = L.polyq_gemv_chain_create(arr, len(phs), 1, C.byref(h))
+        if rc == 0:
+            L.polyq_gemv_chain_free(h)
+        return rc
+
+    x0, y0, y1 = base, base + 0x10000, base + 0x20000
+    # output overlapping its own input
+    assert create(phase(x0, x0 + 256)) == polyq_lib.POLYQ_EINVAL
+    # phase 1's fresh output overlapping phase 0's input
+    assert create(phase(x0, y0), phase(y0, x0)) == polyq_lib.POLYQ_EINVAL
+    # phase 1's fresh output overlapping phase 0's output
+    assert create(phase(x0, y0), phase(x0, y0 + 64)) == polyq_lib.POLYQ_EINVAL
+    # a residual overlapping (but not equal to) its output
+    assert create(phase(x0, y0, y0 + 4)) == polyq_lib.POLYQ_EINVAL
+    # bad phase count and batch
+    assert L.polyq_gemv_chain_create(None, 0, 1, C.byref(C.c_void_p())) == polyq_lib.POLYQ_EINVAL
+    # a legal chain passes the host checks: in place (y == residual) after a
+    # phase that read y, then a fresh output elsewhere.  Without a GPU the
+    # first device query fails instead.
+    rc = create(phase(x0, y0), phase(y0, x0, x0), phase(y0, y1))
+    assert rc in (0, polyq_lib.POLYQ_ECUDA)
