@@ -455,6 +455,41 @@ def bench_decode_step(polyq, synth, torch, device, stream, args, hbm):
         out[mode] = {"ms_per_token": round(ms, 4), "packed_bytes_per_token": step_bytes,
                      "TB/s": round(tbs, 4), "frac_of_hbm": round(tbs * 1e3 / hbm, 4),
                      "kernel_launches_per_token": 8 * L, "stream_finite": finite}
+        if mode == "grouped":
+            # the same token as one persistent launch (polyq_linear_gemv_chain)
+            phases = []
+            for lay in stack:
+                phases += [
+                    dict(layers=[lay["qkv"]], kind=polyq.X_RMSNORM, a=s, eps=1e-6, ys=[yqkv]),
+                    dict(layers=[lay["o"]], kind=polyq.X_F32, a=yqkv[:, 2 * hidden:], ys=[s],
+                         residuals=[s]),
+                    dict(layers=[lay["gu"]], kind=polyq.X_RMSNORM, a=s, eps=1e-6, ys=[ygu]),
+                    dict(layers=[lay["down"]], kind=polyq.X_SILU_MUL, a=ygu[:, :ffn],
+                         b=ygu[:, ffn:], ys=[s], residuals=[s])]
+            chain = polyq.GemvChain(phases, batch=1, stream=stream)
+            s_graph = s.clone()  # the graph's token (every replay starts from s0)
+            with torch.cuda.stream(stream):
+                s.copy_(s0)
+                chain.run(stream=stream)
+            stream.synchronize()
+            agree = float((s - s_graph).norm() / s_graph.norm())
+            with torch.cuda.stream(stream):
+                c0 = torch.cuda.Event(enable_timing=True)
+                c1 = torch.cuda.Event(enable_timing=True)
+                c0.record(stream)
+                for _ in range(reps):
+                    s.copy_(s0)
+                    chain.run(stream=stream)
+                c1.record(stream)
+            stream.synchronize()
+            cms = c0.elapsed_time(c1) / reps
+            out[mode]["chained"] = {
+                "ms_per_token": round(cms, 4),
+                "TB/s": round(step_bytes / (cms * 1e-3) / 1e12, 4),
+                "kernel_launches_per_token": 1, "phases": len(phases),
+                "rel_diff_vs_graph": round(agree, 6),
+                "status": int(chain.workspace[:4].view(torch.int32).item())}
+            del chain
         del stack, base, hosts
         torch.cuda.empty_cache()
     # §5.3 model of activation-reorder traffic per token (A16 read + write of

@@ -407,14 +407,14 @@ int polyq_linear_gemv_input(const polyq_dev_layer* const* layers, int n,
  * Section 4.1 for one to four layers that share an input.  A chain runs all
  * of its phases in one launch: one CTA per resident slot (three per SM)
  * streams the packed weights of every phase through its TMA ring without
- * stopping at phase boundaries, while its consumer warps wait at a grid-wide
- * barrier between phases (phase p+1 reads what phase p wrote), then gather
- * their activation records in shared memory and continue.  Work items of a
- * phase are (layer, step, 64-row tile) in step-major order, split into
- * contiguous ranges of equal modelled cost; each item adds its rows into y
- * with fp32 atomics (the order of those additions varies from run to run).
- * Every device-side wait is bounded; on a timeout the kernel records a
- * status and returns. */
+ * stopping at phase boundaries.  Between phases the consumer warps of all
+ * CTAs meet at a grid-wide barrier (phase p+1 reads what phase p wrote),
+ * then build the phase's activation records in the workspace, one per CTA.
+ * Work items of a phase are (layer, 64-row tile, step) in tile-major order,
+ * split into contiguous ranges of equal modelled cost; each tile piece adds
+ * its rows into y with fp32 atomics (the order of those additions varies
+ * from run to run).  Every device-side wait is bounded; on a timeout the
+ * kernel records a status and returns. */
 typedef struct polyq_gemv_chain polyq_gemv_chain; /* opaque, host-owned */
 
 typedef struct {
@@ -428,10 +428,6 @@ typedef struct {
   const float* residuals[POLYQ_MAX_GROUP];       /* NULL = none; may equal ys[i] */
 } polyq_gemv_phase;
 
-/* Scratch every chained launch needs: a status word and the grid-barrier
- * counters.  Zero-filled before first use; a launch leaves it zeroed unless
- * it reports a timeout (then zero it again). */
-#define POLYQ_CHAIN_WORKSPACE_BYTES 256u
 
 /* Build a chain of n_phases phases (1..65536) at one batch size (1..4).
  * The phase descriptors and the layer descriptors are copied (device memory
@@ -449,6 +445,11 @@ int polyq_gemv_chain_create(const polyq_gemv_phase* phases, int n_phases, int ba
 
 /* Bytes of device memory the chain's plan needs (tensor maps, block tables
  * and per-CTA work ranges for the current device). */
+/* Bytes of the workspace a launch of the chain needs: a status word, the
+ * grid-barrier and launch counters, one record-ready counter per phase and
+ * the activation records of the largest phase. */
+int polyq_gemv_chain_workspace_bytes(const polyq_gemv_chain* chain, size_t* bytes);
+
 int polyq_gemv_chain_plan_bytes(const polyq_gemv_chain* chain, size_t* bytes);
 
 /* Copy the plan into plan_dev (device memory of at least
@@ -460,10 +461,13 @@ int polyq_gemv_chain_upload(polyq_gemv_chain* chain, void* plan_dev, size_t byte
 
 /* Run every phase of the chain, in order, in one cooperative launch on
  * `stream`.  workspace: device, 256-byte aligned, at least
- * POLYQ_CHAIN_WORKSPACE_BYTES, zero-filled before first use; one workspace
- * serves consecutive launches on one stream but not launches that run at the
- * same time.  Launch errors (including a device that cannot hold every CTA
- * at once) are POLYQ_ECUDA. */
+ * polyq_gemv_chain_workspace_bytes, zero-filled before first use and then
+ * kept for this chain (its counters carry over from launch to launch); one
+ * workspace serves consecutive launches on one stream but not launches that
+ * run at the same time.  Its first 4 bytes are a status word that stays zero
+ * unless a bounded wait gave up (then zero the whole workspace again).
+ * Launch errors (including a device that cannot hold every CTA at once) are
+ * POLYQ_ECUDA. */
 int polyq_linear_gemv_chain(const polyq_gemv_chain* chain, void* workspace,
                             size_t workspace_bytes, void* stream);
 

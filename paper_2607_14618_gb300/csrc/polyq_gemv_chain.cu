@@ -4,22 +4,21 @@
 //
 // One CTA per resident slot (3 per SM, all co-resident: cooperative launch).
 //  * Warp 4, one thread, streams the packed codes and scale/zero boxes of
-//    the CTA's items of phase 0, 1, 2, ... through a 3-stage TMA ring and
-//    never waits for a phase boundary: the weights are static, so the ring
-//    is already full when the consumers reach the next phase.
-//  * Warps 0-3 (16 rows each) run the phases in order.  At the start of a
-//    phase they gather, transform (RMSNorm, SiLU * up, rounding to bf16) and
-//    round to fp16 the activation records of the steps their items touch,
-//    into shared-memory slots, then decode and multiply items exactly as the
-//    per-call kernel does, adding each item's rows into y with fp32 atomics.
-//    They also set the next phase's outputs to its residual (or zero).
-//    Between phases the consumers of all CTAs meet at a grid-wide barrier
-//    (an arrival counter in the workspace), because phase p+1 reads what
-//    phase p wrote.
-// Items of a phase are (layer, step, tile) in step-major order, so a CTA's
-// contiguous range touches few steps and its records fit in shared memory;
-// the host splits each phase into ranges of equal modelled cost (the steps
-// of the widths differ in bytes).  Every wait is bounded; a wait that gives
+//    the CTA's items of phase 0, 1, 2, ... through a 3-stage TMA ring without
+//    stopping at phase boundaries (the weights are static), and adds each
+//    item's activation record once every record of its phase has been built
+//    (a per-phase counter in the workspace).
+//  * Warps 0-3 (16 rows each) run the phases in order.  A grid-wide barrier
+//    (an arrival counter) separates phases, because phase p+1 reads what
+//    phase p wrote.  After it, CTA b builds record b (b+G, ...) of the phase
+//    into the workspace: gather, transform (RMSNorm, SiLU * up, rounding to
+//    bf16), activation factor, fp16 rounding, per-chunk sums.  The warps then
+//    set the next phase's outputs to its residual (or zero) and decode and
+//    multiply their items exactly as the per-call kernel does, adding each
+//    tile piece's rows into y with fp32 atomics.
+// Items of a phase are (layer, tile, step) in tile-major order, split into
+// contiguous ranges of equal modelled cost, so each CTA streams the rows of
+// a few tiles from start to end.  Every wait is bounded; a wait that gives
 // up records a status, makes the CTA skip the rest, waits (bounded) for its
 // own copies in flight and returns.
 #include <cuda.h>
@@ -45,12 +44,14 @@ using namespace polyq::gv;
 
 constexpr int kChCtasPerSm = 3;
 constexpr int kChMaxGrid = 1024;
-constexpr int kRecSlots = 4;  // activation records a CTA holds at once
-constexpr int kChDescOff = kCodesBytes + kMetaBytes;
-constexpr int kChStageBytes = ((kChDescOff + 16) + 127) / 128 * 128;
 constexpr uint32_t kGridWaitLimit = 1u << 23;  // barrier polls (each sleeps >= 256 ns)
 constexpr int kStatusTimeoutGrid = 3;
+constexpr int kStatusTimeoutRecords = 4;
 constexpr int kItemFixedCost = 2048;  // per-item overhead in the cost model, bytes
+// workspace: status word at 0; barrier arrivals, CTAs done and the launch
+// count at 64; per-phase record-ready counters from 256; then the records
+constexpr size_t kWsCounters = 64;
+constexpr size_t kWsReady = 256;
 
 struct ChLayer {
   CUtensorMap tm_codes[POLYQ_MAX_BLOCKS];
@@ -80,21 +81,21 @@ struct ChParams {
   int n_phases, batch;
   uint32_t magic;
   int* status;
-  unsigned int* bar;  // [0] barrier arrivals, [1] CTAs done
+  unsigned int* bar;    // [0] barrier arrivals, [1] CTAs done, [2] launches completed
+  unsigned int* ready;  // [n_phases] records built, summed over launches
+  uint8_t* rec;         // records of the current phase
 };
 
 // Consumer-side copy of one phase's tables.
 struct ChShared {
   GvBlock blk[POLYQ_MAX_GROUP][POLYQ_MAX_BLOCKS];
   int n_blocks[POLYQ_MAX_GROUP], N[POLYQ_MAX_GROUP], K[POLYQ_MAX_GROUP];
-  int tiles[POLYQ_MAX_GROUP];
   int item0[POLYQ_MAX_GROUP + 1], rec0[POLYQ_MAX_GROUP + 1];
   const __nv_bfloat16* x[POLYQ_MAX_GROUP];
   const int32_t* gather[POLYQ_MAX_GROUP];
   const float* xscale[POLYQ_MAX_GROUP];
   float* y[POLYQ_MAX_GROUP];
-  const float* residual[POLYQ_MAX_GROUP];
-  int n_layers, kind;
+  int n_layers, kind, recs;
   float eps;
   const float* xa;
   const float* xb;
@@ -105,6 +106,10 @@ __device__ __forceinline__ unsigned ld_acquire_gpu(const unsigned* p) {
   unsigned v;
   asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
   return v;
+}
+
+__device__ __forceinline__ void fence_proxy_async_global() {
+  asm volatile("fence.proxy.async.global;" ::: "memory");
 }
 
 // The tensor maps live in global memory, written by a host copy: make the
@@ -126,32 +131,24 @@ __device__ void load_phase(const ChPhase* ph, ChShared* S) {
     S->n_blocks[t] = L.n_blocks;
     S->N[t] = L.N;
     S->K[t] = L.K;
-    S->tiles[t] = L.tiles;
     S->item0[t] = L.item0;
     S->rec0[t] = L.rec0;
     S->x[t] = L.x;
     S->gather[t] = L.gather;
     S->xscale[t] = L.xscale;
     S->y[t] = L.y;
-    S->residual[t] = L.residual;
   }
   if (t == 32) {
     S->n_layers = nl;
     S->item0[nl] = ph->items;
     S->rec0[nl] = ph->recs;
+    S->recs = ph->recs;
     S->kind = ph->kind;
     S->eps = ph->eps;
     S->xa = ph->xa;
     S->xb = ph->xb;
     S->xout = ph->xout;
   }
-}
-
-// Flat record index (layer's rec0 + step) of item `it` of a phase.
-__device__ __forceinline__ int item_rec(const ChShared& S, int it) {
-  int l = 0;
-  while (l + 1 < S.n_layers && it >= S.item0[l + 1]) ++l;
-  return S.rec0[l] + (it - S.item0[l]) / S.tiles[l];
 }
 
 // Layer, block and block step of flat record f.
@@ -180,41 +177,20 @@ __device__ __forceinline__ XIn chain_xin(const ChShared& S, int l, int batch) {
   return in;
 }
 
-// Records of flat steps f0 .. f0+n-1 into slots 0..n-1, two at a time: the
-// gathers and loads of a pair first (and, once per phase, the RMSNorm
-// factors while they are in flight), then the pair's fp16 records.
+// One activation record of the phase (flat index f) into global memory.
 template <int NB>
-__device__ __noinline__ void build_round(const ChShared& S, int f0, int n, int batch, bool need_rnorm,
-                            const uint32_t* p3, float (*s_part)[kWarps], float* s_rnorm,
-                            uint8_t* slots) {
+__device__ __noinline__ void build_record(const ChShared& S, int f, int batch, const uint32_t* p3,
+                                          const float* s_rnorm, uint8_t* dst) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  for (int q0 = 0; q0 < kRecSlots; q0 += 2) {
-    if (q0 >= n) break;  // n is the same for every consumer thread
-    int src[2][2][2];
-    float fac[2][2][2], ra[2][2][2], rb[2][2][2];
-#pragma unroll
-    for (int u = 0; u < 2; ++u) {
-      if (q0 + u < n) {
-        int l, bi, j;
-        rec_where(S, f0 + q0 + u, &l, &bi, &j);
-        const XIn in = chain_xin(S, l, batch);
-        rec_sources<NB>(in, S.blk[l][bi], j, warp, lane, p3, src[u], fac[u]);
-        rec_load<NB>(in, S.blk[l][bi], j, warp, lane, p3, src[u], ra[u], rb[u]);
-      }
-    }
-    if (need_rnorm && q0 == 0) rms_rnorm(S.xa, S.K[0], batch, S.eps, s_part, s_rnorm);
-#pragma unroll
-    for (int u = 0; u < 2; ++u) {
-      if (q0 + u < n) {
-        int l, bi, j;
-        rec_where(S, f0 + q0 + u, &l, &bi, &j);
-        const XIn in = chain_xin(S, l, batch);
-        rec_store<NB>(in, S.blk[l][bi], j, warp, lane, p3, src[u], fac[u], ra[u], rb[u],
-                      s_rnorm, reinterpret_cast<uint32_t*>(slots + (q0 + u) * kRecMax));
-      }
-    }
-  }
-  consumer_sync();
+  int l, bi, j;
+  rec_where(S, f, &l, &bi, &j);
+  const XIn in = chain_xin(S, l, batch);
+  int src[2][2];
+  float fac[2][2], ra[2][2], rb[2][2];
+  rec_sources<NB>(in, S.blk[l][bi], j, warp, lane, p3, src, fac);
+  rec_load<NB>(in, S.blk[l][bi], j, warp, lane, p3, src, ra, rb);
+  rec_store<NB>(in, S.blk[l][bi], j, warp, lane, p3, src, fac, ra, rb, s_rnorm,
+                reinterpret_cast<uint32_t*>(dst));
 }
 
 // Outputs of a phase start as the residual (or zero); grid-stride over all
@@ -235,9 +211,9 @@ __device__ void init_outputs(const ChPhase* ph, int batch) {
 template <int NB>
 __global__ void __launch_bounds__(kThreads, kChCtasPerSm) gemv_chain(const __grid_constant__ ChParams P) {
   extern __shared__ __align__(128) uint8_t smem[];
+  constexpr int RB = rec_bytes(NB);
   uint8_t* stages = smem;
-  uint8_t* slots = smem + kStages * kChStageBytes;
-  uint32_t* zeros = reinterpret_cast<uint32_t*>(slots + kRecSlots * kRecMax);
+  uint32_t* zeros = reinterpret_cast<uint32_t*>(smem + kStages * kStageBytes);
   uint64_t* bars = reinterpret_cast<uint64_t*>(zeros + 64);
   __shared__ ChShared S;
   __shared__ uint32_t s_p3[16];
@@ -245,12 +221,14 @@ __global__ void __launch_bounds__(kThreads, kChCtasPerSm) gemv_chain(const __gri
   __shared__ float s_part[4][kWarps];
   __shared__ volatile int s_abort;
   __shared__ int s_ok;
+  __shared__ unsigned s_epoch;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t full0 = smem_u32(bars), empty0 = smem_u32(bars + kStages);
   const int G = gridDim.x;
 
   if (threadIdx.x == 0) {
     s_abort = 0;
+    s_epoch = ld_acquire_gpu(P.bar + 2);  // launches completed on this workspace
     for (int s = 0; s < kStages; ++s) {
       mbar_init(full0 + 8 * s, 1);
       mbar_init(empty0 + 8 * s, kWarps);
@@ -266,9 +244,44 @@ __global__ void __launch_bounds__(kThreads, kChCtasPerSm) gemv_chain(const __gri
 
   if (warp == kWarps) {
     // ---------------- producer ----------------
+    // Weights are issued as soon as a stage is free, across phase
+    // boundaries; an item's activation record is issued once its phase's
+    // records are all built (a counter per phase, summed over launches).
     if (lane != 0) return;
-    int kg = 0;  // ring position over all phases
-    for (int p = 0; p < P.n_phases && !s_abort; ++p) {
+    const unsigned epoch = s_epoch;
+    int kg = 0, kr = 0;           // items whose weights / records were issued
+    int ready_phase = -1;         // phases whose records are known to be built
+    const uint8_t* rsrc[kStages]; // record source of each pending item, by slot
+    int rphase[kStages];
+    auto wait_ready = [&](int p) -> bool {
+      const unsigned target = (epoch + 1u) * (unsigned)P.ph[p].recs;
+      uint32_t it = 0;
+      while (ld_acquire_gpu(P.ready + p) < target) {
+        if (++it > kGridWaitLimit || s_abort) return false;
+        __nanosleep(128);
+      }
+      fence_proxy_async_global();  // the builders wrote through the generic proxy
+      return true;
+    };
+    // issue the records of items kr..upto (blocking until their phases are built)
+    auto issue_records = [&](int upto) -> bool {
+      while (kr <= upto) {
+        const int sl = kr % kStages;
+        if (rphase[sl] > ready_phase) {
+          if (!wait_ready(rphase[sl])) {
+            if (!s_abort) atomicExch(P.status, kStatusTimeoutRecords);
+            s_abort = 1;
+            return false;
+          }
+          ready_phase = rphase[sl];
+        }
+        bulk_load(smem_u32(stages + sl * kStageBytes + kRecOff), rsrc[sl], RB, full0 + 8 * sl);
+        ++kr;
+      }
+      return true;
+    };
+    bool go = true;
+    for (int p = 0; p < P.n_phases && go; ++p) {
       const ChPhase* ph = P.ph + p;
       const int lo = __ldg(P.ranges + p * (G + 1) + blockIdx.x);
       const int hi = __ldg(P.ranges + p * (G + 1) + blockIdx.x + 1);
@@ -278,15 +291,21 @@ __global__ void __launch_bounds__(kThreads, kChCtasPerSm) gemv_chain(const __gri
         for (int b = 0; b < ph->L[q].n_blocks; ++b) tmap_acquire(&ph->L[q].tm_codes[b]);
         tmap_acquire(&ph->L[q].tm_meta);
       }
-      // position of item lo: layer, step, tile
+      // position of item lo: layer, tile, step (tile-major)
       int l = 0;
       while (l + 1 < nl && lo >= ph->L[l + 1].item0) ++l;
-      int tiles = ph->L[l].tiles;
-      int s = (lo - ph->L[l].item0) / tiles;
-      int tile = lo - ph->L[l].item0 - s * tiles;
-      for (int it = lo; it < hi; ++it) {
+      int steps = ph->L[l].steps;
+      int tile = (lo - ph->L[l].item0) / steps;
+      int s = lo - ph->L[l].item0 - tile * steps;
+      for (int it = lo; it < hi && go; ++it) {
         const int slot = kg % kStages;
         if (kg >= kStages) {
+          // the consumers free this stage only after the item it holds, so
+          // that item's record goes first
+          if (!issue_records(kg - kStages)) {
+            go = false;
+            break;
+          }
           const uint32_t bar = empty0 + 8 * slot, par = ((kg / kStages) - 1) & 1;
           bool ok = false;
           for (uint32_t w = 0; w < kWaitLimit && !s_abort; ++w)
@@ -297,6 +316,7 @@ __global__ void __launch_bounds__(kThreads, kChCtasPerSm) gemv_chain(const __gri
           if (!ok) {
             if (!s_abort) atomicExch(P.status, kStatusTimeoutEmpty);
             s_abort = 1;
+            go = false;
             break;
           }
         }
@@ -305,17 +325,7 @@ __global__ void __launch_bounds__(kThreads, kChCtasPerSm) gemv_chain(const __gri
         while (bi + 1 < L.n_blocks && s >= L.blk[bi + 1].step0) ++bi;
         const GvBlock B = L.blk[bi];
         const int j = s - B.step0;
-        // next item: same layer and tile only when the layer has one tile
-        int nl2 = l, ns = s, nt = tile + 1;
-        if (nt == tiles) {
-          nt = 0;
-          ++ns;
-          if (ns == L.steps) {
-            ns = 0;
-            ++nl2;
-          }
-        }
-        const bool flush = !(it + 1 < hi && nl2 == l && nt == tile);
+        const bool flush = s == steps - 1 || it == hi - 1;
         int sb, nbx, pitch;
         switch (B.bits) {
           case 2: sb = step_bytes(2, NB); nbx = nbox_of(2, NB); pitch = box_pitch(2, NB); break;
@@ -324,7 +334,7 @@ __global__ void __launch_bounds__(kThreads, kChCtasPerSm) gemv_chain(const __gri
           case 8: sb = step_bytes(8, NB); nbx = nbox_of(8, NB); pitch = box_pitch(8, NB); break;
           default: sb = step_bytes(16, NB); nbx = nbox_of(16, NB); pitch = box_pitch(16, NB); break;
         }
-        uint8_t* st = stages + slot * kChStageBytes;
+        uint8_t* st = stages + slot * kStageBytes;
         const uint32_t dst = smem_u32(st);
         const uint32_t bar = full0 + 8 * slot;
         {
@@ -334,10 +344,10 @@ __global__ void __launch_bounds__(kThreads, kChCtasPerSm) gemv_chain(const __gri
           d.x = (uint32_t)B.bits | ((uint32_t)flush << 8) | ((uint32_t)l << 16);
           d.y = (uint32_t)uvalid | ((uint32_t)g0 << 16);
           d.z = (uint32_t)tile;
-          d.w = (uint32_t)(L.rec0 + s);
-          *reinterpret_cast<uint4*>(st + kChDescOff) = d;
+          d.w = 0u;
+          *reinterpret_cast<uint4*>(st + kDescOff) = d;
         }
-        uint32_t bytes = nbx * pitch * kRows;
+        uint32_t bytes = nbx * pitch * kRows + RB;
         if (B.bits < 16) bytes += kMetaBytes;
         mbar_expect_tx(bar, bytes);
         for (int h = 0; h < nbx; ++h)
@@ -347,16 +357,31 @@ __global__ void __launch_bounds__(kThreads, kChCtasPerSm) gemv_chain(const __gri
           const int x0 = (B.grp_off + j * (B.units / 64)) & ~3;
           tma_load_2d(dst + kCodesBytes, &L.tm_meta, x0, tile * kRows, bar);
         }
+        rsrc[slot] = P.rec + (size_t)(L.rec0 + s) * RB;
+        rphase[slot] = p;
         ++kg;
-        if (nl2 != l) {
-          l = nl2;
-          if (l < nl) tiles = ph->L[l].tiles;
+        if (p <= ready_phase && !issue_records(kg - 1)) {
+          go = false;
+          break;
         }
-        s = ns;
-        tile = nt;
+        // next item
+        if (++s == steps) {
+          s = 0;
+          if (++tile == L.tiles) {
+            tile = 0;
+            if (++l < nl) steps = ph->L[l].steps;
+          }
+        }
       }
     }
-    // wait (bounded) for the copies still in flight before leaving
+    if (go) issue_records(kg - 1);
+    // After a give-up, records still missing are issued anyway (their
+    // contents no longer matter) so that every issued stage completes; then
+    // wait (bounded) for the copies in flight before leaving.
+    for (; kr < kg; ++kr) {
+      const int sl = kr % kStages;
+      bulk_load(smem_u32(stages + sl * kStageBytes + kRecOff), rsrc[sl], RB, full0 + 8 * sl);
+    }
     for (int k = max(0, kg - kStages); k < kg; ++k)
       mbar_wait(full0 + 8 * (k % kStages), (k / kStages) & 1);
     return;
@@ -410,25 +435,22 @@ __global__ void __launch_bounds__(kThreads, kChCtasPerSm) gemv_chain(const __gri
     const ChPhase* ph = P.ph + p;
     load_phase(ph, &S);
     consumer_sync();
+    // this CTA's share of the phase's records (the inputs are complete)
+    if (blockIdx.x < S.recs) {
+      if (S.kind == POLYQ_X_RMSNORM) rms_rnorm(S.xa, S.K[0], P.batch, S.eps, s_part, s_rnorm);
+      int built = 0;
+      for (int f = blockIdx.x; f < S.recs; f += G, ++built)
+        build_record<NB>(S, f, P.batch, s_p3, s_rnorm, P.rec + (size_t)f * RB);
+      consumer_sync();
+      if (threadIdx.x == 0) {
+        __threadfence();
+        atomicAdd(P.ready + p, (unsigned)built);
+      }
+    }
+    if (p + 1 < P.n_phases) init_outputs(P.ph + p + 1, P.batch);
     const int lo = __ldg(P.ranges + p * (G + 1) + blockIdx.x);
     const int hi = __ldg(P.ranges + p * (G + 1) + blockIdx.x + 1);
-    if (p + 1 < P.n_phases) init_outputs(P.ph + p + 1, P.batch);
-    int f_lo = 0, f_last = -1, round = -1;
-    if (lo < hi) {
-      f_lo = item_rec(S, lo);
-      f_last = item_rec(S, hi - 1);
-    }
     for (int it = lo; it < hi; ++it) {
-      const int r = item_rec(S, it) - f_lo;
-      if (r / kRecSlots != round) {
-        // the next records (at a later round, every warp is done with the
-        // current ones)
-        if (round >= 0) consumer_sync();
-        round = r / kRecSlots;
-        const int f0 = f_lo + round * kRecSlots;
-        build_round<NB>(S, f0, min(kRecSlots, f_last - f0 + 1), P.batch,
-                        round == 0 && S.kind == POLYQ_X_RMSNORM, s_p3, s_part, s_rnorm, slots);
-      }
       bool ok = false;
       for (uint32_t w = 0; w < kWaitLimit && !s_abort; ++w)
         if (mbar_try_wait(full0 + 8 * slot, phase)) {
@@ -440,10 +462,9 @@ __global__ void __launch_bounds__(kThreads, kChCtasPerSm) gemv_chain(const __gri
         s_abort = 1;
       }
       if (ok) {
-        const uint8_t* stage = stages + slot * kChStageBytes;
-        const uint4 desc = *reinterpret_cast<const uint4*>(stage + kChDescOff);
-        const uint32_t* rec =
-            reinterpret_cast<const uint32_t*>(slots + (r % kRecSlots) * kRecMax);
+        const uint8_t* stage = stages + slot * kStageBytes;
+        const uint32_t* rec = reinterpret_cast<const uint32_t*>(stage + kRecOff);
+        const uint4 desc = *reinterpret_cast<const uint4*>(stage + kDescOff);
         const int bits = (int)(desc.x & 0xFFu);
         const int uvalid = (int)(desc.y & 0xFFFFu), g0 = (int)(desc.y >> 16);
         switch (bits) {
@@ -456,8 +477,8 @@ __global__ void __launch_bounds__(kThreads, kChCtasPerSm) gemv_chain(const __gri
         __syncwarp();
         if (lane == 0) mbar_arrive(empty0 + 8 * slot);
         if (desc.x & 0x100u) {
-          // add this warp's 16 rows of the item (or of consecutive items of
-          // the same tile) into y; lane t adds batch row t
+          // add this warp's 16 rows of the tile piece into y; lane t adds
+          // batch row t
 #pragma unroll
           for (int rr = 0; rr < 2; ++rr)
 #pragma unroll
@@ -488,13 +509,14 @@ __global__ void __launch_bounds__(kThreads, kChCtasPerSm) gemv_chain(const __gri
     }
     if (p + 1 < P.n_phases) alive = grid_sync();
   }
-  // the last CTA to finish clears the barrier counters for the next launch
+  // the last CTA to finish clears the barrier counters and counts the launch
   consumer_sync();
   if (threadIdx.x == 0 && !s_abort) {
     __threadfence();
     if (atomicAdd(P.bar + 1, 1u) == (unsigned)G - 1) {
       atomicExch(P.bar, 0u);
       atomicExch(P.bar + 1, 0u);
+      atomicAdd(P.bar + 2, 1u);
     }
   }
 }
@@ -502,8 +524,7 @@ __global__ void __launch_bounds__(kThreads, kChCtasPerSm) gemv_chain(const __gri
 // ---------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------
-constexpr size_t kChSmemBytes =
-    (size_t)kStages * kChStageBytes + (size_t)kRecSlots * kRecMax + 64 * 4 + 2 * kStages * 8;
+constexpr size_t kChSmemBytes = (size_t)kStages * kStageBytes + 64 * 4 + 2 * kStages * 8;
 
 int nb_of_batch(int batch) { return batch == 1 ? 1 : batch == 2 ? 2 : 4; }
 
@@ -527,6 +548,7 @@ struct polyq_gemv_chain {
   std::vector<ChPhase> ph;
   std::vector<int> ranges;
   size_t ranges_off = 0, plan_bytes = 0;
+  size_t rec_off = 0, ws_bytes = 0;  // workspace: records region, total
   void* plan_dev = nullptr;
 };
 
@@ -639,46 +661,27 @@ int fill_phase(const polyq_gemv_phase& P, int nb, ChPhase* C) {
 }
 
 // Contiguous item ranges of equal modelled cost (bytes streamed plus a fixed
-// per-item cost) for `grid` CTAs; items are (layer, step, tile) step-major.
+// per-item cost) for `grid` CTAs; items are (layer, tile, step) tile-major.
 void split_phase(const ChPhase& C, int nb, int grid, int* out) {
-  std::vector<long long> cost;  // per step of every layer, in item order
-  std::vector<int> count;
-  long long total = 0;
+  std::vector<long long> prefix(1, 0);  // cost of items [0, i)
+  prefix.reserve((size_t)C.items + 1);
   for (int l = 0; l < C.n_layers; ++l) {
     const ChLayer& L = C.L[l];
+    std::vector<long long> per;
     for (int b = 0; b < L.n_blocks; ++b) {
       const GvBlock& B = L.blk[b];
-      const long long per = (long long)kRows * step_bytes(B.bits, nb) +
-                            (B.bits < 16 ? kRows * 4LL * (B.units / 64) : 0) + kItemFixedCost;
-      for (int j = 0; j < B.n_steps; ++j) {
-        cost.push_back(per);
-        count.push_back(L.tiles);
-        total += per * L.tiles;
-      }
+      const long long c = (long long)kRows * step_bytes(B.bits, nb) +
+                          (B.bits < 16 ? kRows * 4LL * (B.units / 64) : 0) + kItemFixedCost;
+      for (int j = 0; j < B.n_steps; ++j) per.push_back(c);
     }
+    for (int t = 0; t < L.tiles; ++t)
+      for (long long c : per) prefix.push_back(prefix.back() + c);
   }
-  // boundary b: first item whose cost prefix reaches b * total / grid
+  const long long total = prefix.back();
   int item = 0;
-  long long prefix = 0;
-  size_t st = 0;
-  int in_step = 0;  // items of step st already passed
-  out[0] = 0;
-  for (int b = 1; b <= grid; ++b) {
+  for (int b = 0; b <= grid; ++b) {
     const long long goal = (long long)((__int128)total * b / grid);
-    while (st < cost.size() && prefix + cost[st] <= goal) {
-      // advance whole items of this step while they fit
-      const long long room = (goal - prefix) / cost[st];
-      const int take = (int)std::min<long long>(room, count[st] - in_step);
-      item += take;
-      in_step += take;
-      prefix += take * cost[st];
-      if (in_step == count[st]) {
-        ++st;
-        in_step = 0;
-      } else {
-        break;
-      }
-    }
+    while (item < C.items && prefix[item + 1] <= goal) ++item;
     out[b] = item;
   }
   out[grid] = C.items;
@@ -710,7 +713,9 @@ int launch_chain(const polyq_gemv_chain* ch, void* ws, cudaStream_t st) {
   P.batch = ch->batch;
   P.magic = kMagic;
   P.status = static_cast<int*>(ws);
-  P.bar = reinterpret_cast<unsigned int*>(static_cast<char*>(ws) + 64);
+  P.bar = reinterpret_cast<unsigned int*>(static_cast<char*>(ws) + kWsCounters);
+  P.ready = reinterpret_cast<unsigned int*>(static_cast<char*>(ws) + kWsReady);
+  P.rec = static_cast<uint8_t*>(ws) + ch->rec_off;
   cudaLaunchAttribute at[1];
   at[0].id = cudaLaunchAttributeCooperative;
   at[0].val.cooperative = 1;
@@ -801,7 +806,19 @@ extern "C" int polyq_gemv_chain_create(const polyq_gemv_phase* phases, int n_pha
   }
   ch->ranges_off = (size_t)n_phases * sizeof(ChPhase);
   ch->plan_bytes = ch->ranges_off + ch->ranges.size() * sizeof(int);
+  int max_recs = 0;
+  for (const ChPhase& c : ch->ph) max_recs = std::max(max_recs, c.recs);
+  ch->rec_off = (kWsReady + 4 * (size_t)n_phases + 255) / 256 * 256;
+  ch->ws_bytes = ch->rec_off + (size_t)max_recs * rec_bytes(ch->nb);
   *out = ch;
+  return POLYQ_OK;
+}
+
+extern "C" int polyq_gemv_chain_workspace_bytes(const polyq_gemv_chain* ch, size_t* bytes) {
+  polyq_clear_error();
+  if (!ch || !bytes)
+    return polyq_set_error(POLYQ_EINVAL, "polyq_gemv_chain_workspace_bytes: NULL argument");
+  *bytes = ch->ws_bytes;
   return POLYQ_OK;
 }
 
@@ -845,9 +862,9 @@ extern "C" int polyq_linear_gemv_chain(const polyq_gemv_chain* ch, void* workspa
   const char* who = "polyq_linear_gemv_chain";
   if (!ch) return polyq_set_error(POLYQ_EINVAL, "%s: chain is NULL", who);
   if (!ch->plan_dev) return polyq_set_error(POLYQ_EINVAL, "%s: plan not uploaded", who);
-  if (!workspace || ws_bytes < POLYQ_CHAIN_WORKSPACE_BYTES)
-    return polyq_set_error(POLYQ_ENOMEM, "%s: workspace needs %u bytes", who,
-                           (unsigned)POLYQ_CHAIN_WORKSPACE_BYTES);
+  if (!workspace || ws_bytes < ch->ws_bytes)
+    return polyq_set_error(POLYQ_ENOMEM, "%s: workspace needs %zu bytes, got %zu", who,
+                           ch->ws_bytes, ws_bytes);
   if ((uintptr_t)workspace % 256)
     return polyq_set_error(POLYQ_EINVAL, "%s: workspace must be 256-byte aligned", who);
   int dev_sms = 0;

@@ -97,8 +97,6 @@ class GemvPhase(C.Structure):
                 ("ys", C.c_void_p * MAX_GROUP), ("residuals", C.c_void_p * MAX_GROUP)]
 
 
-CHAIN_WORKSPACE_BYTES = 256
-
 _P = C.c_void_p
 _SIGS = {
     "polyq_last_error": (C.c_char_p, []),
@@ -131,6 +129,7 @@ _SIGS = {
     "polyq_gemv_chain_create": (C.c_int, [C.POINTER(GemvPhase), C.c_int, C.c_int,
                                           C.POINTER(C.c_void_p)]),
     "polyq_gemv_chain_plan_bytes": (C.c_int, [_P, C.POINTER(C.c_size_t)]),
+    "polyq_gemv_chain_workspace_bytes": (C.c_int, [_P, C.POINTER(C.c_size_t)]),
     "polyq_gemv_chain_upload": (C.c_int, [_P, _P, C.c_size_t, _P]),
     "polyq_linear_gemv_chain": (C.c_int, [_P, _P, C.c_size_t, _P]),
     "polyq_gemv_chain_free": (None, [_P]),
@@ -601,7 +600,9 @@ class GemvChain:
         self.plan = torch.empty(max(1, nbytes.value), dtype=torch.uint8, device="cuda")
         _check(_lib.polyq_gemv_chain_upload(self._h, self.plan.data_ptr(), self.plan.numel(),
                                             _stream_ptr(stream)))
-        self.workspace = torch.zeros(CHAIN_WORKSPACE_BYTES, dtype=torch.uint8, device="cuda")
+        wsb = C.c_size_t()
+        _check(_lib.polyq_gemv_chain_workspace_bytes(self._h, C.byref(wsb)))
+        self.workspace = torch.zeros(wsb.value, dtype=torch.uint8, device="cuda")
         self.n_phases = len(phases)
 
     def run(self, stream=None, workspace=None):

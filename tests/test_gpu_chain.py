@@ -1,7 +1,7 @@
 """GPU parity of the chained persistent GEMV (polyq_linear_gemv_chain):
 decoder layers as dependent phases against the oracle and against the
 per-call path, independent phases against the oracle at every batch size,
-and a phase whose CTAs need several record rounds.  All calls go through the
+and a phase with more activation records than CTAs.  All calls go through the
 C ABI."""
 import numpy as np
 import pytest
@@ -156,10 +156,10 @@ def test_independent_phases_match_oracle(polyq_lib, batch):
             check_tolerance(ys[name].cpu().numpy(), ref, xs[name][1], K)
 
 
-def test_phase_with_record_rounds_and_single_tiles(polyq_lib):
+def test_phase_with_more_records_than_ctas(polyq_lib):
     # Four layers of 48 rows (one partial tile each) over K = 65536 channels
-    # of all five widths: 2048 items, so CTAs hold several steps of one tile
-    # (records built in rounds, rows summed across steps before adding).
+    # of all five widths at batch 4: 2048 records, so every CTA builds
+    # several, and each CTA's items are consecutive steps of one tile.
     K, N, batch = 65536, 48, 4
     bits = synth.random_codes_layer_bits(K, 91)
     dev, refs = [], []
