@@ -40,10 +40,10 @@ GROUPS = [(0, 1, 2), (3,), (4, 5), (6,)]
 # ncu launch list in profiles/gemv_decode_llama13b_b3_launches.md, with the
 # SHA-1 of the kernel sources it was taken on; reported as null once those
 # sources change.
-TRAFFIC = {"bytes_per_step": 143061000,
-           "sources_sha1": "a5a9b457de15b707d0b8a100b7ae04624e4d1f5c",
+TRAFFIC = {"bytes_per_step": 143070000,
+           "sources_sha1": "27aad085cb22f2e3dd33a88b8ddbe3b04974cc22",
            "profile": "profiles/gemv_decode_llama13b_b3_launches.md"}
-GEMV_SOURCES = ("polyq_gemv.cu", "polyq_gemv_layout.cuh", "polyq_dev.cuh")
+GEMV_SOURCES = ("polyq_gemv.cu", "polyq_gemv_dev.cuh", "polyq_gemv_layout.cuh", "polyq_dev.cuh")
 
 
 def _gemv_sources_sha1():
@@ -310,6 +310,10 @@ def run_polyq(args):
     if not args.no_decode:
         decode = bench_decode_step(polyq, synth, torch, device, stream, args, hbm)
 
+    qwen = None
+    if not args.no_qwen:
+        qwen = bench_qwen(polyq, synth, torch, device, stream, args, hbm)
+
     gemm = None
     if not args.no_gemm:
         gemm = bench_gemm(polyq, synth, torch, device, stream, args, tf_burst, tf_sus)
@@ -340,6 +344,7 @@ def run_polyq(args):
             "clocks": clk.summary(),
             "prefill_gemm": gemm,
             "decode_step": decode,
+            "qwen3_32b_gemv": qwen,
             "permutation_plan": plan_report(polyq),
             "quanta_matching": quanta_report(polyq, synth),
         }
@@ -570,6 +575,72 @@ def quanta_report(polyq, synth):
     return out
 
 
+QWEN = [("q", 8192, 5120), ("k", 1024, 5120), ("v", 1024, 5120), ("o", 5120, 8192),
+        ("gate", 25600, 5120), ("up", 25600, 5120), ("down", 5120, 25600)]
+
+
+def bench_qwen(polyq, synth, torch, device, stream, args, hbm):
+    """The Qwen3-32B-shaped decode linears (q 8192x5120, k/v 1024x5120,
+    o 5120x8192, gate/up 25600x5120, down 5120x25600) at the budget of the
+    run, batch 1 and 4: one step is the four grouped calls (q+k+v, o,
+    gate+up, down), timed as a CUDA graph of steps over two device copies of
+    the layer (372 MB at B = 3, larger than L2)."""
+    copies = 2
+    layers, xs_np, infos = [], [None] * len(QWEN), []
+    for i, (name, N, K) in enumerate(QWEN):
+        W, a = synth.layer_weights(N, K, synth.seed_for(3, i))
+        host = polyq.HostLayer.pack(W, a, args.budget)
+        dev = polyq.DeviceLayer(host, device)
+        infos.append(host.info())
+        layers.append([dev] + [dev.clone() for _ in range(copies - 1)])
+        xs_np[i] = a
+    out = {"workload": f"qwen3-32b decode linears, B={args.budget}, groups q+k+v, o, gate+up, "
+                       f"down, {copies} device copies"}
+    for batch in (1, 4):
+        xs = []
+        for grp in GROUPS:
+            xb, _ = synth.activations(xs_np[grp[0]], batch, 11 + grp[0])
+            t = torch.from_numpy(xb.view(np.int16)).to(device).view(torch.bfloat16)
+            xs += [t] * len(grp)
+        ys = [torch.empty((batch, N), dtype=torch.float32, device=device) for _, N, _ in QWEN]
+        wsz = max(polyq.gemv_group_workspace_bytes([layers[i][0] for i in grp], batch)
+                  for grp in GROUPS)
+        wbuf = torch.zeros(max(wsz, 256), dtype=torch.uint8, device=device)
+        step_bytes = sum(layer_bytes(inf, batch) for inf in infos)
+
+        def run_step(c):
+            for grp in GROUPS:
+                polyq.linear_gemv_group([layers[i][c] for i in grp], [xs[i] for i in grp],
+                                        ys=[ys[i] for i in grp], workspace=wbuf, stream=stream)
+
+        with torch.cuda.stream(stream):
+            run_step(0)
+        stream.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            for c in range(copies):
+                run_step(c)
+        reps = 50
+        with torch.cuda.stream(stream):
+            for _ in range(3):
+                g.replay()
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for _ in range(reps):
+                g.replay()
+            e1.record(stream)
+        stream.synchronize()
+        us = e0.elapsed_time(e1) * 1e3 / (reps * copies)
+        tbs = step_bytes / (us * 1e-6) / 1e12
+        out[f"batch{batch}"] = {"us_per_step": round(us, 2), "bytes_per_step": step_bytes,
+                                "TB/s": round(tbs, 4), "frac_of_hbm": round(tbs * 1e3 / hbm, 4)}
+    out["b_real"] = {n: round(inf["b_real"], 5) for (n, _, _), inf in zip(QWEN, infos)}
+    del layers
+    torch.cuda.empty_cache()
+    return out
+
+
 def bench_gemm(polyq, synth, torch, device, stream, args, tf_burst, tf_sus):
     """Prefill GEMM on the gate/up/down linears at M=2048 (TFLOP/s)."""
     res = {}
@@ -691,6 +762,7 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-gemm", action="store_true")
     ap.add_argument("--no-decode", action="store_true")
+    ap.add_argument("--no-qwen", action="store_true")
     ap.add_argument("--decode-layers", type=int, default=40)
     ap.add_argument("--decode-steps", type=int, default=20)
     args = ap.parse_args()

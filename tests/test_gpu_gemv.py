@@ -94,7 +94,10 @@ def test_gemv_merged_rows_match_unmerged(polyq_lib):
     ("llama-q", 5120, 5120, 3.0, 1),
     ("llama-gate", 13824, 5120, 3.0, 1),
     ("llama-down", 5120, 13824, 4.5, 1),
+    ("qwen-q", 8192, 5120, 5.0, 1),
     ("qwen-kv", 1024, 5120, 3.5, 4),
+    ("qwen-o", 5120, 8192, 4.0, 1),
+    ("qwen-gate", 25600, 5120, 3.0, 4),
     ("qwen-down", 5120, 25600, 6.0, 4),
 ])
 def test_gemv_full_size_sampled_rows(polyq_lib, name, N, K, B, batch):
