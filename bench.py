@@ -52,6 +52,8 @@ def _gemv_sources_sha1():
     for f in GEMV_SOURCES:
         with open(os.path.join(ROOT, "paper_2607_14618_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
+    with open(os.path.join(ROOT, "include", "polyq.h"), "rb") as fh:  # launch parameter layout
+        h.update(fh.read())
     return h.hexdigest()
 
 
@@ -213,6 +215,15 @@ def run_polyq(args):
                 rest[r] = step_graph(r)
             rest[r].replay()
 
+    # the same seven GEMVs (each on its own input) in one grouped launch per
+    # step: the streaming kernel's rate with one launch boundary per step
+    one_graph = torch.cuda.CUDAGraph()
+    wsz1 = polyq.gemv_group_workspace_bytes([layers[i][0] for i in range(n_lin)], batch)
+    wbuf1 = torch.zeros(max(wsz1, 256), dtype=torch.uint8, device=device)
+    with torch.cuda.graph(one_graph, stream=stream):
+        for c in range(args.copies):
+            polyq.linear_gemv_group([layers[i][c] for i in range(n_lin)], xs, ys=ys,
+                                    workspace=wbuf1, stream=stream)
     lin_graphs = []  # per linear: one graph of that linear on every copy
     for i in range(n_lin):
         g = torch.cuda.CUDAGraph()
@@ -251,6 +262,22 @@ def run_polyq(args):
     # launches (pre-pass + streaming kernel per linear), back to back, so its
     # duration per launch is the step time split over the launches.  A
     # per-linear breakdown comes from graphs of one linear on every copy.
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            one_graph.replay()
+        o0 = torch.cuda.Event(enable_timing=True)
+        o1 = torch.cuda.Event(enable_timing=True)
+        o0.record(stream)
+        for _ in range(50):
+            one_graph.replay()
+        o1.record(stream)
+    stream.synchronize()
+    one_us = o0.elapsed_time(o1) * 1e3 / (50 * args.copies)
+    one_tbs = step_bytes / (one_us * 1e-6) / 1e12
+    one_launch = {"us_per_step": round(one_us, 2), "TB/s": round(one_tbs, 4),
+                  "frac_of_hbm": round(one_tbs * 1e3 / hbm, 4),
+                  "what": "the seven GEMVs of a step, each on its own input, as one "
+                          "polyq_linear_gemv_group call (2 kernels) per step"}
     per_lin_us = {}
     reps = 8
     for i in range(n_lin):
@@ -343,6 +370,7 @@ def run_polyq(args):
             "gpu_launches": args.steps * len(GROUPS) * kernels_per_call,
             "clocks": clk.summary(),
             "prefill_gemm": gemm,
+            "one_launch_step": one_launch,
             "decode_step": decode,
             "qwen3_32b_gemv": qwen,
             "permutation_plan": plan_report(polyq),

@@ -60,7 +60,7 @@ extern "C" {
 
 #define POLYQ_MAX_BLOCKS 5
 #define POLYQ_GROUP 64
-#define POLYQ_MAX_GROUP 4 /* layers per polyq_linear_gemv_group call */
+#define POLYQ_MAX_GROUP 8 /* layers per GEMV group call or chain phase */
 
 #define POLYQ_ALLOC_WATERFILL 0 /* Section 3.2 max-heap waterfilling (default) */
 #define POLYQ_ALLOC_LADDER 1    /* descending saliency, each channel climbs */
@@ -404,7 +404,7 @@ int polyq_linear_gemv_input(const polyq_dev_layer* const* layers, int n,
 /* ---- chained decode GEMVs in one persistent launch ----
  * A decoder's decode step is a chain of dependent GEMV phases (q/k/v, o,
  * gate/up, down, then the next layer's q/k/v, ...), each the product of
- * Section 4.1 for one to four layers that share an input.  A chain runs all
+ * Section 4.1 for one to POLYQ_MAX_GROUP layers that share an input.  A chain runs all
  * of its phases in one launch: one CTA per resident slot (three per SM)
  * streams the packed weights of every phase through its TMA ring without
  * stopping at phase boundaries.  Between phases the consumer warps of all

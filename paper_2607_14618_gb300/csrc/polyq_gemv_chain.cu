@@ -1,5 +1,5 @@
 // Chained decode GEMVs: every phase of a decoder's decode step (each phase
-// the Section 4.1 product of one to four layers that read one input) in one
+// the Section 4.1 product of one to eight layers that read one input) in one
 // persistent launch.
 //
 // One CTA per resident slot (3 per SM, all co-resident: cooperative launch).

@@ -21,7 +21,7 @@ POLYQ_ECUDA = -3
 POLYQ_EUNSUPPORTED = -4
 POLYQ_ETIMEOUT = -5
 MAX_BLOCKS = 5
-MAX_GROUP = 4
+MAX_GROUP = 8
 GROUP = 64
 NOALLOC_SCRATCH_BYTES = 1 << 20  # scratch compiled in for linear_gemv_noalloc
 ALLOC_WATERFILL = 0
@@ -563,7 +563,7 @@ def decoder_plan_graph(n_layers, hidden, ffn, perm_of, kv=None, qdim=None):
 class GemvChain:
     """A chain of dependent GEMV phases run in one persistent launch
     (polyq_linear_gemv_chain).  Each phase is a dict with ``layers`` (one to
-    four DeviceLayer reading one input), ``kind`` (X_BF16, X_F32, X_RMSNORM,
+    eight DeviceLayer reading one input), ``kind`` (X_BF16, X_F32, X_RMSNORM,
     X_SILU_MUL), ``a`` (and ``b`` for X_SILU_MUL) CUDA tensors [batch][K],
     ``ys`` fp32 CUDA tensors [batch][N], optional ``residuals``, ``eps``,
     ``x_out`` and, for X_BF16, per-layer inputs ``xs``.  The tensors must

@@ -139,5 +139,26 @@ def test_gemv_group_matches_oracle(polyq_lib, batch):
         if res[i] is not None:
             yref = yref + res[i].cpu().numpy().astype(np.float64)
         check_tolerance(y.cpu().numpy(), yref, x, K)
-    with pytest.raises(polyq_lib.PolyqError):
-        polyq_lib.linear_gemv_group(layers + layers[:1], [xt] * 5)
+    with pytest.raises(polyq_lib.PolyqError):  # at most POLYQ_MAX_GROUP = 8 layers
+        polyq_lib.linear_gemv_group(layers * 2 + layers[:1], [xt] * 9)
+
+
+@pytest.mark.parametrize("batch", [1, 3])
+def test_gemv_group_of_seven_layers_with_own_inputs(polyq_lib, batch):
+    """The seven linears of a decoder layer (scaled down) in one launch, each
+    reading its own activation."""
+    hidden, ffn = 384, 1024
+    layers, refs, xs, xts = [], [], [], []
+    for i, (name, N, K) in enumerate(O.llama_layer_linears(hidden, ffn)):
+        W, a = synth.layer_weights(N, K, 400 + i)
+        bits = synth.random_codes_layer_bits(K, 400 + i) if i % 3 == 0 else None
+        host = polyq_lib.HostLayer.pack(W, a, 3.0, forced_bits=bits)
+        layers.append(polyq_lib.DeviceLayer(host, "cuda"))
+        refs.append(O.pack_layer(W, a, 3.0, bits=bits))
+        xb, x = synth.activations(a, batch, 410 + i)
+        xs.append(x)
+        xts.append(_x_dev(xb))
+    ys = polyq_lib.linear_gemv_group(layers, xts)
+    torch.cuda.synchronize()
+    for y, ref, x in zip(ys, refs, xs):
+        check_tolerance(y.cpu().numpy(), O.linear(ref, x), x, x.shape[1])
