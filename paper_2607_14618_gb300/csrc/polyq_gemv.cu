@@ -717,7 +717,7 @@ extern "C" int polyq_linear_gemv_group(const polyq_dev_layer* const* layers, int
 // Some callers cannot allocate device memory: a plugin inside a host program
 // whose own pool owns the device, or a latency-bound loop that cannot take the
 // device-wide synchronisation cudaMalloc/cudaFree may cause.  For them the
-// status word, tile counters and piece sums live in this fixed array, one copy
+// status word and the activation records live in this fixed array, one copy
 // per device that loads the library, kept until the process exits.  In host
 // code the name below stands for a host-side shadow, never the device address:
 // the address is looked up with cudaGetSymbolAddress, once per device.
