@@ -16,7 +16,7 @@
 //    64-row tile, step) work items of all layers of the call form one list;
 //    each CTA takes a contiguous range of it.  Warp 4 (one thread) streams
 //    each item's packed codes and scale/zero metadata with TMA through a
-//    3-stage shared-memory ring, the first stages before the grid-dependency
+//    3-stage shared-memory ring, the first stage before the grid-dependency
 //    wait (weights do not depend on earlier kernels), and adds the item's
 //    record once the pre-pass is done.  Warps 0-3 each own 16 rows: a code
 //    pair becomes two exact fp16 values 1024 + q*2^p with one LOP3 against the
@@ -246,6 +246,7 @@ __global__ void __launch_bounds__(kConsumers) gemv_prep(const __grid_constant__ 
   float fac[2][2];
   const XIn in = xin_of(P, l);
   rec_sources<NB>(in, S.blk[l][bi], j, warp, lane, s_p3, src, fac);  // static layer data
+  if (P.xkind == POLYQ_X_RMSNORM) rms_prefetch(P.xa, P.L[0].K, P.batch);
   pdl_wait();  // x comes from the previous kernel; the records and y may still be in use
   float ra[2][2], rb[2][2];
   rec_load<NB>(in, S.blk[l][bi], j, warp, lane, s_p3, src, ra, rb);
@@ -346,7 +347,9 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) gemv_main(const __grid_c
         tma_load_2d(dst + kCodesBytes, &P.L[q.l].tm_meta, x0, q.tile * kRows, bar);
       }
     };
-    const int pre = min(n_mine, kStages);
+    // One stage before the wait: more would compete for DRAM with the
+    // pre-pass's activation loads, which are on the critical path.
+    const int pre = min(n_mine, 1);
     if (lane == 0) {
       for (int l = 0; l < nl; ++l) {
         for (int b = 0; b < S.n_blocks[l]; ++b) prefetch_tmap(&P.L[l].tm_codes[b]);
@@ -364,14 +367,12 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) gemv_main(const __grid_c
     for (int k = 0; k < n_mine; ++k) {
       const int slot = k % kStages;
       if (s_abort) break;
-      if (k >= kStages) {
-        if (!mbar_wait(empty0 + 8 * slot, ((k / kStages) - 1) & 1)) {
-          atomicExch(P.status, kStatusTimeoutEmpty);
-          s_abort = 1;
-          break;
-        }
-        issue_weights(k, it);
+      if (k >= kStages && !mbar_wait(empty0 + 8 * slot, ((k / kStages) - 1) & 1)) {
+        atomicExch(P.status, kStatusTimeoutEmpty);
+        s_abort = 1;
+        break;
       }
+      if (k >= pre) issue_weights(k, it);
       const int r = S.rec0[it.l] + it.s;
       bulk_load(smem_u32(stages + slot * kStageBytes + kRecOff),
                 P.rec + (size_t)r * RB, RB, full0 + 8 * slot);

@@ -112,8 +112,15 @@ struct XIn {
   int kind, K, batch;
 };
 
+__device__ __forceinline__ void prefetch_l2(const void* p) {
+  asm volatile("prefetch.global.L2 [%0];" ::"l"(p));
+}
+
 // Pass 1 of a record: the gather indices and activation factors (static
-// layer data, so this may run before the grid-dependency wait).
+// layer data, so this may run before the grid-dependency wait), and an L2
+// prefetch of the activations the record will read.  L2 is where writes of
+// earlier kernels land, so prefetching before their completion is safe: the
+// loads after the wait still see the final values.
 template <int NB>
 __device__ __forceinline__ void rec_sources(const XIn& in, const GvBlock& B, int j, int warp,
                                             int lane, const uint32_t* p3, int (&src)[2][2],
@@ -131,6 +138,13 @@ __device__ __forceinline__ void rec_sources(const XIn& in, const GvBlock& B, int
           const int p = B.pos0 + g.ch[h];
           src[s][h] = gather ? __ldg(gather + p) : p;
           if (in.xscale) fac[s][h] = __ldg(in.xscale + p);
+          const size_t o = (size_t)g.bb * in.K + src[s][h];
+          if (in.kind == POLYQ_X_BF16) {
+            prefetch_l2(in.x + o);
+          } else {
+            prefetch_l2(in.xa + o);
+            if (in.kind == POLYQ_X_SILU_MUL) prefetch_l2(in.xb + o);
+          }
         }
     }
   }
@@ -140,6 +154,13 @@ __device__ __forceinline__ void rec_sources(const XIn& in, const GvBlock& B, int
 // a streaming kernel does not take part).
 __device__ __forceinline__ void consumer_sync() {
   asm volatile("bar.sync 1, %0;" ::"n"(kConsumers) : "memory");
+}
+
+// L2 prefetch of the batch rows the RMSNorm factor reads (before a wait).
+__device__ __forceinline__ void rms_prefetch(const float* xa, int K, int batch) {
+  for (int bb = 0; bb < batch; ++bb)
+    for (int i = 32 * threadIdx.x; i < K; i += 32 * kConsumers)  // one 128-byte line each
+      prefetch_l2(xa + (size_t)bb * K + i);
 }
 
 // s_rnorm[b] = 1 / sqrt(mean_k a[b][k]^2 + eps) for each batch row, computed
