@@ -54,6 +54,7 @@ constexpr int kMeta = BN * 16;                  // 4 KB
 constexpr int kStageG = MT * kATile + kBTile + kCodes + kMeta;  // 48 KB
 constexpr int kThreadsG = 320;
 constexpr int kDqWarps = 8;
+constexpr double kUnitCostTiles = 12.0;  // per-unit overhead, in K tiles, of the split model
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kIdesc = umma_idesc_f16(BM, BN);
 
@@ -582,13 +583,23 @@ extern "C" int polyq_linear_gemm(const polyq_dev_layer* L, const void* X, int64_
   int sms = 0;
   rc = polyq_sm_count(&sms);
   if (rc) return rc;
-  // Split K when there are too few (M, N) tiles to keep two waves of SMs busy;
-  // each split keeps at least 16 K tiles.
+  // Split K when the (M, N) tiles fill the SMs poorly: take the split with
+  // the least modelled time, whole waves of units times (K tiles per unit +
+  // a per-unit cost for filling the pipeline and adding the tile into Y).
+  // Each split keeps at least 16 K tiles; near ties go to fewer splits.
   {
     const int mn = P.units_m * P.units_n;
     int ks = 1;
-    if (mn < 2 * sms) ks = std::min((2 * sms + mn - 1) / mn, std::max(1, KT / 16));
-    if (ks > 1 && (P.N % 4) != 0) ks = 1;  // the zeroing pass writes float4
+    double best = 1e300;
+    const int kmax = (P.N % 4) != 0 ? 1 : std::max(1, std::min(64, KT / 16));  // zeroing writes float4
+    for (int k = 1; k <= kmax; ++k) {
+      const long long waves = ((long long)mn * k + sms - 1) / sms;
+      const double t = (double)waves * ((double)KT / k + kUnitCostTiles);
+      if (t < 0.98 * best) {
+        best = t;
+        ks = k;
+      }
+    }
     P.ksplit = ks;
     P.units = mn * ks;
   }
