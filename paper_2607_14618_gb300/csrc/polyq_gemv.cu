@@ -52,6 +52,8 @@ using namespace polyq::gv;
 
 constexpr int kCtasPerSm = 3;
 constexpr int kMaxGrid = 1024;  // persistent CTAs at most
+constexpr uint32_t kDescEnd = 0x200u;   // descriptor flag: no more items
+constexpr uint32_t kDescPair = 0x400u;  // descriptor flag: the stage holds two steps
 
 
 // One layer of a call.  Tensor maps first (64-byte aligned).
@@ -300,18 +302,23 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) gemv_main(const __grid_c
   const long long I = P.items, C = gridDim.x;
   const int lo = (int)((long long)blockIdx.x * I / C);
   const int hi = (int)((long long)(blockIdx.x + 1) * I / C);
-  const int n_mine = hi - lo;
 
   if (warp == kWarps) {
     // ---------------- producer ----------------
     // The packed weights do not depend on earlier kernels: request the first
-    // stages before the grid-dependency wait.  The activation records come
-    // from this call's builders and are loaded once they are flagged ready.
+    // stage before the grid-dependency wait (more would compete for DRAM with
+    // the pre-pass's activation loads, which are on the critical path).  The
+    // activation records come from this call's pre-pass and are loaded after
+    // it.
     ItemPos it;
-    it.init(S, nl, lo);
-    auto issue_weights = [&](int k, const ItemPos& q) {
+    int item = lo;
+    if (lo < hi) it.init(S, nl, lo);
+    int rec_a[kStages], rec_b[kStages];  // records of each stage's steps (-1: none)
+    // Weights of the next stage: one item, or at batch 2-4 two consecutive
+    // steps of one block and tile whose codes take one box each.
+    auto issue_stage = [&](int k) {
       const int slot = k % kStages;
-      const GvBlock& B = S.blk[q.l][q.bi];
+      const GvBlock& B = S.blk[it.l][it.bi];
       int sb, nbx, pitch;
       switch (B.bits) {
         case 2: sb = step_bytes(2, NB); nbx = nbox_of(2, NB); pitch = box_pitch(2, NB); break;
@@ -320,63 +327,95 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) gemv_main(const __grid_c
         case 8: sb = step_bytes(8, NB); nbx = nbox_of(8, NB); pitch = box_pitch(8, NB); break;
         default: sb = step_bytes(16, NB); nbx = nbox_of(16, NB); pitch = box_pitch(16, NB); break;
       }
+      const bool pair = NB > 1 && nbx == 1 && item + 1 < hi && it.j + 1 < B.n_steps;
+      const int j2 = it.j + 1;
       const uint32_t dst = smem_u32(stages + slot * kStageBytes);
       const uint32_t bar = full0 + 8 * slot;
       {
-        // what the consumers need of this item: width, whether the item ends
-        // a tile piece, layer, valid units, first meta entry, tile
-        const int uvalid = min(B.units, B.n_ch - q.j * B.units);
-        const int g0 = (B.grp_off + q.j * (B.units / 64)) & 3;
-        const bool flush = q.tile_end(S) || k == n_mine - 1;
+        // what the consumers need: width, whether the stage ends a tile
+        // piece, pairing, layer, valid units of each step, first meta entry,
+        // tile
+        const int uvalid = min(B.units, B.n_ch - it.j * B.units);
+        const int uvalid2 = pair ? min(B.units, B.n_ch - j2 * B.units) : 0;
+        const int g0 = (B.grp_off + it.j * (B.units / 64)) & 3;
+        const int last_s = it.s + (pair ? 1 : 0);
+        const bool flush = last_s == S.steps[it.l] - 1 || item + (pair ? 2 : 1) == hi;
         uint4 d;
-        d.x = (uint32_t)B.bits | ((uint32_t)flush << 8) | ((uint32_t)q.l << 16);
+        d.x = (uint32_t)B.bits | ((uint32_t)flush << 8) | ((uint32_t)pair << 10) |
+              ((uint32_t)it.l << 16);
         d.y = (uint32_t)uvalid | ((uint32_t)g0 << 16);
-        d.z = (uint32_t)q.tile;
-        d.w = 0u;
+        d.z = (uint32_t)it.tile;
+        d.w = (uint32_t)uvalid2;
         *reinterpret_cast<uint4*>(stages + slot * kStageBytes + kDescOff) = d;
       }
-      uint32_t bytes = nbx * pitch * kRows + RB;
+      uint32_t bytes = (pair ? 2 : 1) * (nbx * pitch * kRows + RB);
       if (B.bits < 16) bytes += kMetaBytes;
       mbar_expect_tx(bar, bytes);
-      const CUtensorMap* tm = &P.L[q.l].tm_codes[q.bi];
+      const CUtensorMap* tm = &P.L[it.l].tm_codes[it.bi];
       for (int h = 0; h < nbx; ++h)
-        tma_load_2d(dst + h * kRows * pitch, tm, B.seg_off + q.j * sb + h * (sb / nbx),
-                    q.tile * kRows, bar);
+        tma_load_2d(dst + h * kRows * pitch, tm, B.seg_off + it.j * sb + h * (sb / nbx),
+                    it.tile * kRows, bar);
+      if (pair) tma_load_2d(dst + kRows * pitch, tm, B.seg_off + j2 * sb, it.tile * kRows, bar);
       if (B.bits < 16) {
-        const int x0 = (B.grp_off + q.j * (B.units / 64)) & ~3;
-        tma_load_2d(dst + kCodesBytes, &P.L[q.l].tm_meta, x0, q.tile * kRows, bar);
+        // one box of kMetaBox groups covers both steps of a pair
+        const int x0 = (B.grp_off + it.j * (B.units / 64)) & ~3;
+        tma_load_2d(dst + kCodesBytes, &P.L[it.l].tm_meta, x0, it.tile * kRows, bar);
+      }
+      rec_a[slot] = S.rec0[it.l] + it.s;
+      rec_b[slot] = pair ? rec_a[slot] + 1 : -1;
+      it.next(S, nl);
+      ++item;
+      if (pair) {
+        it.next(S, nl);
+        ++item;
       }
     };
-    // One stage before the wait: more would compete for DRAM with the
-    // pre-pass's activation loads, which are on the critical path.
-    const int pre = min(n_mine, 1);
+    auto issue_records = [&](int k) {
+      const int slot = k % kStages;
+      const uint32_t dst = smem_u32(stages + slot * kStageBytes + kRecOff);
+      bulk_load(dst, P.rec + (size_t)rec_a[slot] * RB, RB, full0 + 8 * slot);
+      if (rec_b[slot] >= 0)
+        bulk_load(dst + RB, P.rec + (size_t)rec_b[slot] * RB, RB, full0 + 8 * slot);
+    };
+    int ks = 0;  // stages issued
     if (lane == 0) {
       for (int l = 0; l < nl; ++l) {
         for (int b = 0; b < S.n_blocks[l]; ++b) prefetch_tmap(&P.L[l].tm_codes[b]);
         prefetch_tmap(&P.L[l].tm_meta);
       }
-      ItemPos q = it;
-      for (int k = 0; k < pre; ++k) {
-        issue_weights(k, q);
-        q.next(S, nl);
-      }
+      if (item < hi) issue_stage(ks++);
     }
     pdl_wait();  // the records come from the pre-pass of this call
     fence_proxy_async_global();  // it wrote them through the generic proxy
     if (lane != 0) return;
-    for (int k = 0; k < n_mine; ++k) {
-      const int slot = k % kStages;
-      if (s_abort) break;
-      if (k >= kStages && !mbar_wait(empty0 + 8 * slot, ((k / kStages) - 1) & 1)) {
-        atomicExch(P.status, kStatusTimeoutEmpty);
+    if (ks > 0) issue_records(0);
+    bool ok = true;
+    while (item < hi) {
+      const int slot = ks % kStages;
+      if (s_abort || (ks >= kStages && !mbar_wait(empty0 + 8 * slot, ((ks / kStages) - 1) & 1))) {
+        if (!s_abort) atomicExch(P.status, kStatusTimeoutEmpty);
         s_abort = 1;
+        ok = false;
         break;
       }
-      if (k >= pre) issue_weights(k, it);
-      const int r = S.rec0[it.l] + it.s;
-      bulk_load(smem_u32(stages + slot * kStageBytes + kRecOff),
-                P.rec + (size_t)r * RB, RB, full0 + 8 * slot);
-      it.next(S, nl);
+      issue_stage(ks);
+      issue_records(ks);
+      ++ks;
+    }
+    // wait (bounded) for the copies still in flight, then mark the end of
+    // the items in the next stage
+    for (int k = max(0, ks - kStages); k < ks; ++k)
+      mbar_wait(full0 + 8 * (k % kStages), (k / kStages) & 1);
+    if (ok) {
+      const int slot = ks % kStages;
+      if (ks < kStages || mbar_wait(empty0 + 8 * slot, ((ks / kStages) - 1) & 1)) {
+        *reinterpret_cast<uint4*>(stages + slot * kStageBytes + kDescOff) =
+            make_uint4(kDescEnd, 0u, 0u, 0u);
+        mbar_arrive(full0 + 8 * slot);
+      } else {
+        atomicExch(P.status, kStatusTimeoutEmpty);
+        s_abort = 1;
+      }
     }
     return;
   }
@@ -391,7 +430,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) gemv_main(const __grid_c
     for (int b = 0; b < NB; ++b) acc[r][b] = 0.f;
   int slot = 0;
   uint32_t phase = 0;
-  for (int k = 0; k < n_mine; ++k) {
+  for (;;) {
     if (s_abort || !mbar_wait(full0 + 8 * slot, phase)) {
       if (lane == 0 && !s_abort) atomicExch(P.status, kStatusTimeoutFull);
       s_abort = 1;
@@ -400,14 +439,27 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) gemv_main(const __grid_c
     const uint8_t* stage = stages + slot * kStageBytes;
     const uint32_t* rec = reinterpret_cast<const uint32_t*>(stage + kRecOff);
     const uint4 desc = *reinterpret_cast<const uint4*>(stage + kDescOff);
+    if (desc.x & kDescEnd) break;
     const int bits = (int)(desc.x & 0xFFu);
     const int uvalid = (int)(desc.y & 0xFFFFu), g0 = (int)(desc.y >> 16);
     switch (bits) {
-      case 2: step_mma<NB, 2>(P.magic, P.batch, uvalid, g0, stage, rec, zeros, warp, lane, acc); break;
-      case 3: step_mma<NB, 3>(P.magic, P.batch, uvalid, g0, stage, rec, zeros, warp, lane, acc); break;
-      case 4: step_mma<NB, 4>(P.magic, P.batch, uvalid, g0, stage, rec, zeros, warp, lane, acc); break;
-      case 8: step_mma<NB, 8>(P.magic, P.batch, uvalid, g0, stage, rec, zeros, warp, lane, acc); break;
+      case 2: step_mma<NB, 2>(P.magic, P.batch, uvalid, g0, stage, stage, rec, zeros, warp, lane, acc); break;
+      case 3: step_mma<NB, 3>(P.magic, P.batch, uvalid, g0, stage, stage, rec, zeros, warp, lane, acc); break;
+      case 4: step_mma<NB, 4>(P.magic, P.batch, uvalid, g0, stage, stage, rec, zeros, warp, lane, acc); break;
+      case 8: step_mma<NB, 8>(P.magic, P.batch, uvalid, g0, stage, stage, rec, zeros, warp, lane, acc); break;
       default: step_16<NB>(P.batch, uvalid, stage, rec, zeros, warp, lane, acc); break;
+    }
+    if (NB > 1 && (desc.x & kDescPair)) {
+      // the second step of the pair: its box follows the first, its record
+      // follows the first record, its chunks follow in the meta box
+      const uint32_t* rec2 = rec + RB / 4;
+      const int uv2 = (int)desc.w;
+      switch (bits) {
+        case 2: step_mma<NB, 2>(P.magic, P.batch, uv2, g0 + step_chunks(2, NB), stage + kRows * box_pitch(2, NB), stage, rec2, zeros, warp, lane, acc); break;
+        case 3: step_mma<NB, 3>(P.magic, P.batch, uv2, g0 + step_chunks(3, NB), stage + kRows * box_pitch(3, NB), stage, rec2, zeros, warp, lane, acc); break;
+        case 4: step_mma<NB, 4>(P.magic, P.batch, uv2, g0 + step_chunks(4, NB), stage + kRows * box_pitch(4, NB), stage, rec2, zeros, warp, lane, acc); break;
+        default: step_mma<NB, 8>(P.magic, P.batch, uv2, g0 + step_chunks(8, NB), stage + kRows * box_pitch(8, NB), stage, rec2, zeros, warp, lane, acc); break;
+      }
     }
     __syncwarp();
     if (lane == 0) mbar_arrive(empty0 + 8 * slot);

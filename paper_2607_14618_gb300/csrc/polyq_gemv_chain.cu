@@ -468,10 +468,10 @@ __global__ void __launch_bounds__(kThreads, kChCtasPerSm) gemv_chain(const __gri
         const int bits = (int)(desc.x & 0xFFu);
         const int uvalid = (int)(desc.y & 0xFFFFu), g0 = (int)(desc.y >> 16);
         switch (bits) {
-          case 2: step_mma<NB, 2>(P.magic, P.batch, uvalid, g0, stage, rec, zeros, warp, lane, acc); break;
-          case 3: step_mma<NB, 3>(P.magic, P.batch, uvalid, g0, stage, rec, zeros, warp, lane, acc); break;
-          case 4: step_mma<NB, 4>(P.magic, P.batch, uvalid, g0, stage, rec, zeros, warp, lane, acc); break;
-          case 8: step_mma<NB, 8>(P.magic, P.batch, uvalid, g0, stage, rec, zeros, warp, lane, acc); break;
+          case 2: step_mma<NB, 2>(P.magic, P.batch, uvalid, g0, stage, stage, rec, zeros, warp, lane, acc); break;
+          case 3: step_mma<NB, 3>(P.magic, P.batch, uvalid, g0, stage, stage, rec, zeros, warp, lane, acc); break;
+          case 4: step_mma<NB, 4>(P.magic, P.batch, uvalid, g0, stage, stage, rec, zeros, warp, lane, acc); break;
+          case 8: step_mma<NB, 8>(P.magic, P.batch, uvalid, g0, stage, stage, rec, zeros, warp, lane, acc); break;
           default: step_16<NB>(P.batch, uvalid, stage, rec, zeros, warp, lane, acc); break;
         }
         __syncwarp();

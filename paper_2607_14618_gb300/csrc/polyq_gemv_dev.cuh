@@ -357,7 +357,8 @@ __device__ __forceinline__ void load_words(uint32_t* w, const uint8_t* codes, in
 // scaled, into acc[row][batch].
 template <int NB, int BITS>
 __device__ __forceinline__ void step_mma(uint32_t magic, int batch, int uvalid, int g0,
-                                         const uint8_t* stage, const uint32_t* rec,
+                                         const uint8_t* codes, const uint8_t* stage,
+                                         const uint32_t* rec,
                                          const uint32_t* zeros, int warp, int lane,
                                          float (&acc)[2][NB]) {
   constexpr int U = step_units(BITS, NB);
@@ -376,8 +377,8 @@ __device__ __forceinline__ void step_mma(uint32_t magic, int batch, int uvalid, 
   const uint32_t* meta_s = reinterpret_cast<const uint32_t*>(stage + kCodesBytes);
 
   uint32_t wa[NW], wb[NW];
-  load_words<BITS, NB>(wa, stage, rA, t);
-  load_words<BITS, NB>(wb, stage, rB, t);
+  load_words<BITS, NB>(wa, codes, rA, t);
+  load_words<BITS, NB>(wb, codes, rB, t);
 
   // Column g of the B fragment is (batch my_b, chunk my_c); lane t's codes in
   // box h belong to chunk c_t + h*CPB, so only a matching lane loads its

@@ -29,9 +29,13 @@ constexpr int kPitchSplit = 144;   // row pitch of 128-byte boxes (16 extra byte
 constexpr int kMetaBox = 12;       // meta entries per row loaded per step
 constexpr int kCodesBytes = 2 * kRows * kPitchSplit;  // largest codes area (2 boxes)
 constexpr int kMetaBytes = kRows * kMetaBox * 4;
-constexpr int kRecMax = 1344;      // largest activation record (NB = 4)
-// A stage holds an item's code boxes, its scale/zero box, its record and a
-// 16-byte descriptor written by the producer.
+constexpr int kRecOne = 1344;      // largest activation record (NB = 4)
+constexpr int kRecMax = 2 * kRecOne;  // a stage may hold two steps' records
+// A stage holds an item's code boxes, its scale/zero box, its record(s) and
+// a 16-byte descriptor written by the producer.  At batch 2-4 a step whose
+// codes take one box can share its stage with the next step of the same
+// block and tile (the second step's box follows the first, both records
+// follow each other).
 constexpr int kRecOff = kCodesBytes + kMetaBytes;
 constexpr int kDescOff = kRecOff + kRecMax;
 constexpr int kStageBytes = ((kDescOff + 16) + 127) / 128 * 128;
@@ -83,7 +87,7 @@ __host__ __device__ constexpr int rec_pair_words(int nb) { return nb * 4 * rec_l
 __host__ __device__ constexpr int rec_bytes(int nb) {
   return (rec_pair_words(nb) + 2 * nb * (8 / nb)) * 4;
 }
-static_assert(rec_bytes(1) <= kRecMax && rec_bytes(2) <= kRecMax && rec_bytes(4) <= kRecMax, "");
+static_assert(rec_bytes(1) <= kRecOne && rec_bytes(2) <= kRecOne && rec_bytes(4) <= kRecOne, "");
 static_assert(rec_bytes(1) % 16 == 0 && rec_bytes(2) % 16 == 0 && rec_bytes(4) % 16 == 0, "");
 static_assert(lane_pairs(2, 1) + 4 <= rec_lane_words(1) && lane_pairs(2, 4) + 4 <= rec_lane_words(4), "");
 
