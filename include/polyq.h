@@ -473,6 +473,18 @@ int polyq_linear_gemv_chain(const polyq_gemv_chain* chain, void* workspace,
 
 void polyq_gemv_chain_free(polyq_gemv_chain* chain);
 
+/* Read the status word of a GEMV, GEMM or chain workspace (its first 4 bytes)
+ * after the work queued on `stream`: a copy to the host and a wait for the
+ * stream.  *status = 0 and POLYQ_OK when no bounded device wait gave up;
+ * otherwise *status names the wait (1 a consumer's wait for a stage's data,
+ * 2 a producer's wait for a free stage, 3 a chained launch's grid barrier,
+ * 4 a chained launch's wait for a phase's records) and the call returns
+ * POLYQ_ETIMEOUT.  The kernels that gave up returned normally, so the
+ * context stays usable; zero the workspace before using it again.  The GEMM
+ * workspace keeps its status word in its last 256 bytes: pass that address
+ * (workspace + polyq_gemm_workspace_bytes() - 256). */
+int polyq_workspace_status(const void* workspace, int* status, void* stream);
+
 /* Device scratch bytes polyq_linear_gemm needs for this layer and M. */
 int polyq_gemm_workspace_bytes(const polyq_dev_layer* layer, int64_t M,
                                size_t* bytes);

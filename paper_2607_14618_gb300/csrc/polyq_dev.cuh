@@ -15,8 +15,10 @@ namespace polyq {
 constexpr uint32_t kWaitLimit = 1u << 24;
 
 // Status codes written by kernels into the workspace status word.
-constexpr int kStatusTimeoutFull = 1;
-constexpr int kStatusTimeoutEmpty = 2;
+constexpr int kStatusTimeoutFull = 1;     // a consumer's wait for a stage's data
+constexpr int kStatusTimeoutEmpty = 2;    // a producer's wait for a free stage
+constexpr int kStatusTimeoutGrid = 3;     // a chained launch's grid barrier
+constexpr int kStatusTimeoutRecords = 4;  // a chained launch's wait for a phase's records
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return (uint32_t)__cvta_generic_to_shared(p);

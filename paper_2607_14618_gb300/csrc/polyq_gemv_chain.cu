@@ -44,9 +44,10 @@ using namespace polyq::gv;
 
 constexpr int kChCtasPerSm = 3;
 constexpr int kChMaxGrid = 1024;
-constexpr uint32_t kGridWaitLimit = 1u << 23;  // barrier polls (each sleeps >= 256 ns)
-constexpr int kStatusTimeoutGrid = 3;
-constexpr int kStatusTimeoutRecords = 4;
+// Polls of a grid barrier or a record counter before giving up (each poll
+// sleeps at least 128-256 ns and reads L2): about a second, against waits of
+// microseconds in a working launch.
+constexpr uint32_t kGridWaitLimit = 1u << 21;
 constexpr int kItemFixedCost = 2048;  // per-item overhead in the cost model, bytes
 // workspace: status word at 0; barrier arrivals, CTAs done and the launch
 // count at 64; per-phase record-ready counters from 256; then the records
@@ -254,9 +255,11 @@ __global__ void __launch_bounds__(kThreads, kChCtasPerSm) gemv_chain(const __gri
     const uint8_t* rsrc[kStages]; // record source of each pending item, by slot
     int rphase[kStages];
     auto wait_ready = [&](int p) -> bool {
+      // the counter grows by recs per launch and wraps after 2^32 / recs
+      // launches: compare by signed difference
       const unsigned target = (epoch + 1u) * (unsigned)P.ph[p].recs;
       uint32_t it = 0;
-      while (ld_acquire_gpu(P.ready + p) < target) {
+      while ((int)(target - ld_acquire_gpu(P.ready + p)) > 0) {
         if (++it > kGridWaitLimit || s_abort) return false;
         __nanosleep(128);
       }

@@ -92,3 +92,23 @@ int polyq_tensor_map_2d(CUtensorMap* out, const void* base, int elem_bytes, uint
   *out = m;
   return POLYQ_OK;
 }
+
+extern "C" int polyq_workspace_status(const void* workspace, int* status, void* stream) {
+  polyq_clear_error();
+  if (!workspace || !status)
+    return polyq_set_error(POLYQ_EINVAL, "polyq_workspace_status: NULL argument");
+  cudaStream_t st = (cudaStream_t)stream;
+  int v = 0;
+  cudaError_t e = cudaMemcpyAsync(&v, workspace, sizeof v, cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  if (e != cudaSuccess)
+    return polyq_set_error(POLYQ_ECUDA, "polyq_workspace_status: %s", cudaGetErrorString(e));
+  *status = v;
+  if (v == 0) return POLYQ_OK;
+  static const char* what[] = {"?", "a consumer's wait for a stage's data",
+                               "a producer's wait for a free stage",
+                               "a chained launch's grid barrier",
+                               "a chained launch's wait for a phase's records"};
+  return polyq_set_error(POLYQ_ETIMEOUT, "a bounded device wait gave up: %s (status %d)",
+                         what[(v >= 1 && v <= 4) ? v : 0], v);
+}

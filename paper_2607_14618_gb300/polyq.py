@@ -133,6 +133,7 @@ _SIGS = {
     "polyq_gemv_chain_upload": (C.c_int, [_P, _P, C.c_size_t, _P]),
     "polyq_linear_gemv_chain": (C.c_int, [_P, _P, C.c_size_t, _P]),
     "polyq_gemv_chain_free": (None, [_P]),
+    "polyq_workspace_status": (C.c_int, [_P, C.POINTER(C.c_int), _P]),
     "polyq_gemm_workspace_bytes": (C.c_int, [C.POINTER(DevLayer), C.c_int64,
                                              C.POINTER(C.c_size_t)]),
     "polyq_linear_gemm": (C.c_int, [C.POINTER(DevLayer), _P, C.c_int64, _P, _P, C.c_size_t, _P]),
@@ -614,3 +615,11 @@ class GemvChain:
         if getattr(self, "_h", None) and self._h.value:
             _lib.polyq_gemv_chain_free(self._h)
             self._h = C.c_void_p()
+
+
+def workspace_status(workspace, stream=None):
+    """Status word of a workspace after the queued work (0: no device wait
+    gave up); raises PolyqError(POLYQ_ETIMEOUT) when one did."""
+    v = C.c_int()
+    _check(_lib.polyq_workspace_status(workspace.data_ptr(), C.byref(v), _stream_ptr(stream)))
+    return v.value

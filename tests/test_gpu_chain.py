@@ -176,3 +176,32 @@ def test_phase_with_more_records_than_ctas(polyq_lib):
     torch.cuda.synchronize()
     for y, ref in zip(ys, refs):
         check_tolerance(y.cpu().numpy(), O.linear(ref, x), x, K)
+
+
+def test_record_wait_gives_up_with_a_status(polyq_lib):
+    # Failure detection without a fault: the launch count in the workspace is
+    # raised so that the producers' target for the records of phase 0 is one
+    # nothing will reach.  Their bounded wait gives up after about a second,
+    # the launch returns with status 4, and after zeroing the workspace the
+    # same chain runs correctly again.
+    K, N = 512, 256
+    W, a = synth.layer_weights(N, K, 97)
+    dev = polyq_lib.DeviceLayer(polyq_lib.HostLayer.pack(W, a, 3.0), "cuda")
+    ref = O.pack_layer(W, a, 3.0)
+    xb, x = synth.activations(a, 1, 97)
+    y = torch.zeros((1, N), device="cuda")
+    chain = polyq_lib.GemvChain([dict(layers=[dev], kind=polyq_lib.X_BF16, a=_x_dev(xb),
+                                      ys=[y])], batch=1)
+    assert polyq_lib.workspace_status(chain.workspace) == 0
+    chain.workspace[72:76].view(torch.int32).fill_(1 << 20)  # launches completed
+    chain.run()
+    with pytest.raises(polyq_lib.PolyqError) as ei:
+        polyq_lib.workspace_status(chain.workspace)
+    assert ei.value.code == polyq_lib.POLYQ_ETIMEOUT
+    assert int(chain.workspace[:4].view(torch.int32).item()) == 4
+    # the context still works: clear the workspace and run again
+    chain.workspace.zero_()
+    chain.run()
+    torch.cuda.synchronize()
+    assert polyq_lib.workspace_status(chain.workspace) == 0
+    check_tolerance(y.cpu().numpy(), O.linear(ref, x), x, K)
