@@ -24,6 +24,13 @@ import subprocess
 import sys
 import time
 
+# The oracle's fp64 product goes through BLAS, which would use every host core
+# unless told otherwise: the reference arm and the one-thread CPU baseline pin
+# it to one thread before numpy loads (the driver's own setting wins).
+if "--cpu-baseline-child" in sys.argv or ("--impl" in sys.argv and "reference" in sys.argv):
+    for _v in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS"):
+        os.environ.setdefault(_v, "1")
+
 import numpy as np
 
 ROOT = os.path.dirname(os.path.abspath(__file__))
@@ -41,7 +48,7 @@ GROUPS = [(0, 1, 2), (3,), (4, 5), (6,)]
 # SHA-1 of the kernel sources it was taken on; reported as null once those
 # sources change.
 TRAFFIC = {"bytes_per_step": 143135000,
-           "sources_sha1": "d7dc2314be22b3e871a3ad0302a77b40147fffc0",
+           "sources_sha1": "4422acc0b771ada7a1c8c0d9dfb283b745f259d0",
            "profile": "profiles/gemv_decode_llama13b_b3_launches.md"}
 GEMV_SOURCES = ("polyq_gemv.cu", "polyq_gemv_dev.cuh", "polyq_gemv_layout.cuh", "polyq_dev.cuh")
 
@@ -302,6 +309,8 @@ def run_polyq(args):
             "launch_unit": "one step: 4 grouped GEMV calls (8 launches), "
                            f"{step_bytes} algorithmic bytes",
             "traffic_source": TRAFFIC["profile"] if traffic else None,
+            "codes_only_GBps": round(sum(inf["packed_bytes"] for _, inf in infos)
+                                     / (ms_step * 1e-3) / 1e9, 1),
             "per_linear": per_lin_us}
 
     # end to end through the public API: pinned host x -> device, GEMVs, y -> host
@@ -345,6 +354,15 @@ def run_polyq(args):
     if not args.no_gemm:
         gemm = bench_gemm(polyq, synth, torch, device, stream, args, tf_burst, tf_sus)
 
+    sweep = None
+    if not args.no_sweep and batch == 1:
+        sweep = bench_budgets(polyq, synth, torch, device, stream, hbm)
+
+    dense = None
+    if not args.no_dense and batch == 1:
+        dense = bench_dense(torch, device, stream, hbm)
+        dense["polyq_step_speedup"] = round(dense["us_per_step"] / (ms_step * 1e3), 3)
+
     if rank == 0:
         cpu = None if (args.no_cpu_baseline or ws > 1) else cpu_baseline(args.cpu_seconds)
         out = {
@@ -373,6 +391,8 @@ def run_polyq(args):
             "one_launch_step": one_launch,
             "decode_step": decode,
             "qwen3_32b_gemv": qwen,
+            "budget_sweep": sweep,
+            "dense_bf16_context": dense,
             "permutation_plan": plan_report(polyq),
             "quanta_matching": quanta_report(polyq, synth),
         }
@@ -607,34 +627,34 @@ QWEN = [("q", 8192, 5120), ("k", 1024, 5120), ("v", 1024, 5120), ("o", 5120, 819
         ("gate", 25600, 5120), ("up", 25600, 5120), ("down", 5120, 25600)]
 
 
-def bench_qwen(polyq, synth, torch, device, stream, args, hbm):
-    """The Qwen3-32B-shaped decode linears (q 8192x5120, k/v 1024x5120,
-    o 5120x8192, gate/up 25600x5120, down 5120x25600) at the budget of the
-    run, batch 1 and 4: one step is the four grouped calls (q+k+v, o,
-    gate+up, down), timed as a CUDA graph of steps over two device copies of
-    the layer (372 MB at B = 3, larger than L2)."""
-    copies = 2
-    layers, xs_np, infos = [], [None] * len(QWEN), []
-    for i, (name, N, K) in enumerate(QWEN):
-        W, a = synth.layer_weights(N, K, synth.seed_for(3, i))
-        host = polyq.HostLayer.pack(W, a, args.budget)
+def time_grouped_step(polyq, synth, torch, device, stream, shapes, config, budget, batches,
+                      copies, hbm):
+    """One decoder layer's seven linears of ``shapes`` (seeded from synthetic
+    config ``config``) packed at ``budget`` and run as the four grouped calls
+    (q+k+v, o, gate+up, down), timed as a CUDA graph of steps over ``copies``
+    device copies of the layer."""
+    layers, xs_np, infos = [], [None] * len(shapes), []
+    for i, (name, N, K) in enumerate(shapes):
+        W, a = synth.layer_weights(N, K, synth.seed_for(config, i))
+        host = polyq.HostLayer.pack(W, a, budget)
         dev = polyq.DeviceLayer(host, device)
         infos.append(host.info())
         layers.append([dev] + [dev.clone() for _ in range(copies - 1)])
         xs_np[i] = a
-    out = {"workload": f"qwen3-32b decode linears, B={args.budget}, groups q+k+v, o, gate+up, "
-                       f"down, {copies} device copies"}
-    for batch in (1, 4):
+        del W
+    out = {}
+    for batch in batches:
         xs = []
         for grp in GROUPS:
             xb, _ = synth.activations(xs_np[grp[0]], batch, 11 + grp[0])
             t = torch.from_numpy(xb.view(np.int16)).to(device).view(torch.bfloat16)
             xs += [t] * len(grp)
-        ys = [torch.empty((batch, N), dtype=torch.float32, device=device) for _, N, _ in QWEN]
+        ys = [torch.empty((batch, N), dtype=torch.float32, device=device) for _, N, _ in shapes]
         wsz = max(polyq.gemv_group_workspace_bytes([layers[i][0] for i in grp], batch)
                   for grp in GROUPS)
         wbuf = torch.zeros(max(wsz, 256), dtype=torch.uint8, device=device)
         step_bytes = sum(layer_bytes(inf, batch) for inf in infos)
+        codes = sum(inf["packed_bytes"] for inf in infos)
 
         def run_step(c):
             for grp in GROUPS:
@@ -662,11 +682,84 @@ def bench_qwen(polyq, synth, torch, device, stream, args, hbm):
         us = e0.elapsed_time(e1) * 1e3 / (reps * copies)
         tbs = step_bytes / (us * 1e-6) / 1e12
         out[f"batch{batch}"] = {"us_per_step": round(us, 2), "bytes_per_step": step_bytes,
-                                "TB/s": round(tbs, 4), "frac_of_hbm": round(tbs * 1e3 / hbm, 4)}
-    out["b_real"] = {n: round(inf["b_real"], 5) for (n, _, _), inf in zip(QWEN, infos)}
+                                "TB/s": round(tbs, 4), "frac_of_hbm": round(tbs * 1e3 / hbm, 4),
+                                "codes_only_TB/s": round(codes / (us * 1e-6) / 1e12, 4)}
+    out["b_real"] = {n: round(inf["b_real"], 5) for (n, _, _), inf in zip(shapes, infos)}
     del layers
     torch.cuda.empty_cache()
     return out
+
+
+def bench_qwen(polyq, synth, torch, device, stream, args, hbm):
+    """The Qwen3-32B-shaped decode linears (q 8192x5120, k/v 1024x5120,
+    o 5120x8192, gate/up 25600x5120, down 5120x25600) at the budget of the
+    run, batch 1 and 4: one step is the four grouped calls (q+k+v, o,
+    gate+up, down), timed as a CUDA graph of steps over two device copies of
+    the layer (372 MB at B = 3, larger than L2)."""
+    out = {"workload": f"qwen3-32b decode linears, B={args.budget}, groups q+k+v, o, gate+up, "
+                       "down, 2 device copies"}
+    out.update(time_grouped_step(polyq, synth, torch, device, stream, QWEN, 3, args.budget,
+                                 (1, 4), 2, hbm))
+    return out
+
+
+def bench_budgets(polyq, synth, torch, device, stream, hbm):
+    """The other budgets of the Llama2-13B (B = 4.5) and Qwen3-32B (B = 3.5,
+    4, 5, 6) decode linears, batch 1: the same four grouped calls per step,
+    timed over two device copies (every set is larger than L2)."""
+    out = {"what": "four grouped GEMV calls per step, batch 1, 2 device copies"}
+    for model, shapes, config, budgets in (("llama2_13b", LLAMA, 2, (4.5,)),
+                                           ("qwen3_32b", QWEN, 3, (3.5, 4.0, 5.0, 6.0))):
+        for B in budgets:
+            r = time_grouped_step(polyq, synth, torch, device, stream, shapes, config, B, (1,), 2,
+                                  hbm)
+            out[f"{model}_B{B}"] = dict(r["batch1"], b_real_min=min(r["b_real"].values()),
+                                        b_real_max=max(r["b_real"].values()))
+    return out
+
+
+def bench_dense(torch, device, stream, hbm, copies=2):
+    """Context, not the product: the same seven Llama2-13B decode linears as
+    dense bf16 matrix-vector products through torch (cuBLAS), batch 1, timed
+    as a CUDA graph over two copies of the weights (1.27 GB)."""
+    g = torch.Generator(device=device)
+    g.manual_seed(7)
+    Ws = [[(torch.randn((N, K), device=device, generator=g) * 0.02).to(torch.bfloat16)
+           for _, N, K in LLAMA] for _ in range(copies)]
+    xs = [torch.randn((1, K), device=device, generator=g).to(torch.bfloat16) for _, _, K in LLAMA]
+    ys = [None] * len(LLAMA)
+    step_bytes = sum(2 * N * K + 2 * K + 2 * N for _, N, K in LLAMA)
+
+    def run_step(c):
+        for i in range(len(LLAMA)):
+            ys[i] = torch.nn.functional.linear(xs[i], Ws[c][i])
+
+    with torch.cuda.stream(stream):
+        run_step(0)
+    stream.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        for c in range(copies):
+            run_step(c)
+    reps = 50
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            graph.replay()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(reps):
+            graph.replay()
+        e1.record(stream)
+    stream.synchronize()
+    us = e0.elapsed_time(e1) * 1e3 / (reps * copies)
+    tbs = step_bytes / (us * 1e-6) / 1e12
+    del Ws
+    torch.cuda.empty_cache()
+    return {"what": "context only: dense bf16 y = x W^T of the seven Llama2-13B linears, "
+                    "torch/cuBLAS, batch 1, 7 launches per step",
+            "us_per_step": round(us, 2), "bytes_per_step": step_bytes, "TB/s": round(tbs, 4),
+            "frac_of_hbm": round(tbs * 1e3 / hbm, 4)}
 
 
 def bench_gemm(polyq, synth, torch, device, stream, args, tf_burst, tf_sus):
@@ -704,7 +797,33 @@ def bench_gemm(polyq, synth, torch, device, stream, args, tf_burst, tf_sus):
     return res
 
 
+def _blas_threads():
+    v = os.environ.get("OPENBLAS_NUM_THREADS") or os.environ.get("OMP_NUM_THREADS")
+    return int(v) if v else os.cpu_count()
+
+
 def cpu_baseline(seconds):
+    """The oracle timed on the host cores in child processes (no CUDA state):
+    with BLAS pinned to one thread (the reported baseline) and with BLAS free
+    to use every core."""
+    runs = {}
+    for threads in (1, os.cpu_count() or 1):
+        env = dict(os.environ, OPENBLAS_NUM_THREADS=str(threads), OMP_NUM_THREADS=str(threads))
+        r = subprocess.run([sys.executable, os.path.abspath(__file__), "--cpu-baseline-child",
+                            "--cpu-seconds", str(seconds)], env=env, capture_output=True,
+                           text=True, timeout=600)
+        if r.returncode != 0:
+            return {"unavailable": f"oracle child exited {r.returncode}: {r.stderr[-300:]}"}
+        runs[threads] = json.loads(r.stdout.strip().splitlines()[-1])
+    one = runs[1]
+    many = runs[max(runs)]
+    one["all_cores"] = {"value": many["value"], "unit": many["unit"], "cores": many["cores"],
+                        "note": "BLAS free to use every host core; unpacking and dequantising "
+                                "stay single-threaded numpy"}
+    return one
+
+
+def cpu_baseline_child(seconds):
     """The oracle's linear (unpack + dequantise + fp64 dot from the packed
     bytes) on a bounded sample of the workload: row slices of the seven
     linears, repeated until about ``seconds`` of CPU time."""
@@ -726,9 +845,8 @@ def cpu_baseline(seconds):
             O.linear(L, x)
             nbytes += L["packed"].nbytes + L["meta"].nbytes + x.size * 2 + L["K"] * 4 + rows * 4
     dt = time.perf_counter() - t0
-    threads = os.environ.get("OMP_NUM_THREADS") or os.environ.get("OPENBLAS_NUM_THREADS")
     return {"value": round(nbytes / dt / 1e12, 8), "unit": "TB/s",
-            "cores": int(threads) if threads else 1, "host_cpus": os.cpu_count(),
+            "cores": _blas_threads(), "host_cpus": os.cpu_count(),
             "kind": "oracle",
             "sample": f"{rows} output rows of each of the 7 linears, oracle linear "
                       f"(unpack+dequant+fp64 dot) repeated for {dt:.1f} s"}
@@ -768,7 +886,7 @@ def run_reference(args):
            "ms_per_step": round(1e3 * dt / args.steps, 3), "higher_is_better": True,
            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
            "config": {"workload": WORKLOAD, "budget_bits": args.budget, "batch": 1},
-           "cpu_baseline": {"kind": "oracle", "cores": 1, "host_cpus": os.cpu_count(),
+           "cpu_baseline": {"kind": "oracle", "cores": _blas_threads(), "host_cpus": os.cpu_count(),
                             "value": round(v, 8), "unit": "TB/s",
                             "sample": f"{rows} output rows of each of the 7 linears per step"},
            "e2e": {"value": round(v, 8), "unit": "TB/s", "h2d_bytes_per_step": 0,
@@ -785,7 +903,7 @@ def main():
     ap.add_argument("--budget", type=float, default=3.0)
     ap.add_argument("--batch", type=int, default=1)
     ap.add_argument("--copies", type=int, default=6)
-    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-gemm", action="store_true")
@@ -793,7 +911,13 @@ def main():
     ap.add_argument("--no-qwen", action="store_true")
     ap.add_argument("--decode-layers", type=int, default=40)
     ap.add_argument("--decode-steps", type=int, default=20)
+    ap.add_argument("--no-sweep", action="store_true")
+    ap.add_argument("--no-dense", action="store_true")
+    ap.add_argument("--cpu-baseline-child", action="store_true", help=argparse.SUPPRESS)
     args = ap.parse_args()
+    if args.cpu_baseline_child:
+        print(json.dumps(cpu_baseline_child(args.cpu_seconds)), flush=True)
+        return
     if args.warmup < 3:
         args.warmup = 3
     if args.impl == "reference":
