@@ -16,10 +16,11 @@
 //       warp 1      allocates 512 TMEM columns and issues tcgen05.mma
 //                   (M=128, N=256, K=16, fp16 in, fp32 accumulate), two
 //                   M tiles per weight tile;
-//       warps 2..9  dequantise one weight row each: (q - z) * s in fp16 via
-//                   magic-number decode, written in the UMMA 64-byte-swizzle
-//                   K-major layout; afterwards they drain the accumulator with
-//                   tcgen05.ld and store fp32 Y.
+//       warps 2..9  dequantise: (q - z) * s in fp16 via magic-number decode,
+//                   written in the UMMA 64-byte-swizzle K-major layout.  Warps
+//                   2-5 take the even stages and 6-9 the odd ones, two weight
+//                   rows per thread; afterwards all eight drain the
+//                   accumulator with tcgen05.ld and store fp32 Y.
 //     Four pipeline stages.  When the (M, N) tiles cannot fill the GPU the K
 //     range is split and the pieces are added into a zeroed Y (so the order of
 //     those additions varies); otherwise Y is stored directly.  Every wait is
@@ -64,7 +65,7 @@ struct GmBlock {
 };
 
 struct GmParams {
-  CUtensorMap tm_x;      // Xg [M][KT*32] fp16, box {32, 128}, 64B swizzle
+  CUtensorMap tm_x;      // Xg [M][KT*32] fp16, box {32, 256} (both M tiles), 64B swizzle
   CUtensorMap tm_codes;  // packed [N][S] u8, box {48, 256}
   CUtensorMap tm_meta;   // meta [N][meta_stride] u32, box {4, 256}
   CUtensorMap tm_w16;    // packed [N][S/2] u16, box {32, 256}, 64B swizzle
@@ -80,6 +81,32 @@ struct GmParams {
   float* y;
   int* status;
 };
+
+// try_wait that lets the hardware suspend the thread for up to `hint_ns`
+// (it wakes when the phase completes) instead of returning at once.
+__device__ __forceinline__ bool mbar_try_wait_hint(uint32_t bar, uint32_t parity,
+                                                   uint32_t hint_ns) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity), "r"(hint_ns)
+      : "memory");
+  return ok != 0;
+}
+
+// Bounded wait for the lone producer and MMA threads: each poll may sleep up
+// to 1 us, so that their polling does not take issue slots from the
+// dequantisation warps that share their schedulers.  At most 2^22 polls, a
+// few seconds.
+constexpr uint32_t kWaitLimitSleep = 1u << 22;
+constexpr uint32_t kSuspendHintNs = 1000;
+__device__ __forceinline__ bool mbar_wait_sleep(uint32_t bar, uint32_t parity) {
+  for (uint32_t it = 0; it < kWaitLimitSleep; ++it)
+    if (mbar_try_wait_hint(bar, parity, kSuspendHintNs)) return true;
+  return false;
+}
 
 __device__ __forceinline__ int find_kblock(const GmBlock* blk, int nblk, int kt) {
   int b = 0;
@@ -262,7 +289,7 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
     s_abort = 0;
     for (int s = 0; s < kStagesG; ++s) {
       mbar_init(smem_u32(&bar_full[s]), 1);
-      mbar_init(smem_u32(&bar_bready[s]), kDqWarps);
+      mbar_init(smem_u32(&bar_bready[s]), kDqWarps / 2);  // one group of four warps per stage
       mbar_init(smem_u32(&bar_sfree[s]), 1);
     }
     mbar_init(smem_u32(&bar_accf), 1);
@@ -303,7 +330,7 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
         const int kt_hi = (int)((long long)(ks + 1) * KT / P.ksplit);
         for (int kt = kt_lo; kt < kt_hi && !s_abort; ++kt, ++kg) {
           const int s = kg % kStagesG, use = kg / kStagesG;
-          if (use > 0 && !mbar_wait(smem_u32(&bar_sfree[s]), (use - 1) & 1)) {
+          if (use > 0 && !mbar_wait_sleep(smem_u32(&bar_sfree[s]), (use - 1) & 1)) {
             fail(kStatusTimeoutEmpty);
             break;
           }
@@ -313,9 +340,8 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
           const uint32_t bar = smem_u32(&bar_full[s]);
           const bool w16 = B.bits == 16;
           mbar_expect_tx(bar, MT * kATile + (w16 ? kBTile : kCodes + kMeta));
-#pragma unroll
-          for (int t = 0; t < MT; ++t)
-            tma_load_2d(smem_u32(st + t * kATile), &P.tm_x, kt * BK, um * (MT * BM) + t * BM, bar);
+          // both M tiles in one box: 256 rows, the second at + kATile
+          tma_load_2d(smem_u32(st), &P.tm_x, kt * BK, um * (MT * BM), bar);
           if (w16) {
             tma_load_2d(smem_u32(st + MT * kATile), &P.tm_w16, (B.seg_off + 64 * hg) / 2, un * BN,
                         bar);
@@ -337,15 +363,15 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
         const int ks = u / (P.units_m * P.units_n);
         const int kt_lo = (int)((long long)ks * KT / P.ksplit);
         const int kt_hi = (int)((long long)(ks + 1) * KT / P.ksplit);
-        if (uc > 0 && !mbar_wait(smem_u32(&bar_acce), (uc - 1) & 1)) {
+        if (uc > 0 && !mbar_wait_sleep(smem_u32(&bar_acce), (uc - 1) & 1)) {
           fail(kStatusTimeoutEmpty);
           break;
         }
         tc_fence_after();
         for (int kt = kt_lo; kt < kt_hi && !s_abort; ++kt, ++kg) {
           const int s = kg % kStagesG, use = kg / kStagesG;
-          if (!mbar_wait(smem_u32(&bar_full[s]), use & 1) ||
-              !mbar_wait(smem_u32(&bar_bready[s]), use & 1)) {
+          if (!mbar_wait_sleep(smem_u32(&bar_full[s]), use & 1) ||
+              !mbar_wait_sleep(smem_u32(&bar_bready[s]), use & 1)) {
             fail(kStatusTimeoutFull);
             break;
           }
@@ -367,7 +393,13 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
     }
   } else {
     // ---------------- dequantisation + epilogue (8 warps) ----------------
-    const int r = threadIdx.x - 64;  // weight row of the tile, 0..255
+    // Two groups of four warps take alternate stages (group g the stages
+    // with kg % 2 == g); a thread dequantises rows r0 and r0 + 128 of its
+    // group's stages.  Each group so has two stage periods for its
+    // latency-bound work, and each thread two independent rows.
+    const int dq = threadIdx.x - 64;  // 0..255
+    const int grp = dq >> 7;
+    const int r0 = dq & 127;
     const int q = warp & 3;          // TMEM lane quarter this warp may access
     const int half = (warp - 2) >> 2;
     int kg = 0, uc = 0;
@@ -377,6 +409,7 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
       const int kt_lo = (int)((long long)ks * KT / P.ksplit);
       const int kt_hi = (int)((long long)(ks + 1) * KT / P.ksplit);
       for (int kt = kt_lo; kt < kt_hi && !s_abort; ++kt, ++kg) {
+        if ((kg & 1) != grp) continue;
         const int s = kg % kStagesG, use = kg / kStagesG;
         if (!mbar_wait(smem_u32(&bar_full[s]), use & 1) ||
             (use > 0 && !mbar_wait(smem_u32(&bar_sfree[s]), (use - 1) & 1))) {
@@ -388,36 +421,43 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
           const int hg = kt - B.kt0;
           uint8_t* st = stage_ptr(s);
           const int start = B.seg_off + 4 * B.bits * hg;
-          // the row's code bytes start at offset (start & 15) of a 16-byte
-          // aligned window; two conflict-free 16-byte reads cover them
-          const uint4* rp = reinterpret_cast<const uint4*>(st + MT * kATile + kBTile + r * kCodeBox);
-          const uint4 c0 = rp[0], c1 = rp[1];
-          const uint32_t cw[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
-          uint32_t w[8];
-          switch ((start & 15) >> 2) {  // uniform over the CTA
-            case 0:
+          const int mslot = (B.grp_off + hg / 2) & 3;
+          const int sh = (start & 15) >> 2;  // uniform over the CTA
 #pragma unroll
-              for (int k = 0; k < 8; ++k) w[k] = cw[k];
-              break;
-            case 1:
+          for (int h = 0; h < 2; ++h) {
+            const int r = r0 + 128 * h;
+            // the row's code bytes start at offset (start & 15) of a 16-byte
+            // aligned window; two conflict-free 16-byte reads cover them
+            const uint4* rp =
+                reinterpret_cast<const uint4*>(st + MT * kATile + kBTile + r * kCodeBox);
+            const uint4 c0 = rp[0], c1 = rp[1];
+            const uint32_t cw[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
+            uint32_t w[8];
+            switch (sh) {
+              case 0:
 #pragma unroll
-              for (int k = 0; k < 7; ++k) w[k] = cw[k + 1];
-              w[7] = 0;
-              break;
-            case 2:
+                for (int k = 0; k < 8; ++k) w[k] = cw[k];
+                break;
+              case 1:
 #pragma unroll
-              for (int k = 0; k < 6; ++k) w[k] = cw[k + 2];
-              w[6] = w[7] = 0;
-              break;
-            default:
+                for (int k = 0; k < 7; ++k) w[k] = cw[k + 1];
+                w[7] = 0;
+                break;
+              case 2:
 #pragma unroll
-              for (int k = 0; k < 5; ++k) w[k] = cw[k + 3];
-              w[5] = w[6] = w[7] = 0;
-              break;
+                for (int k = 0; k < 6; ++k) w[k] = cw[k + 2];
+                w[6] = w[7] = 0;
+                break;
+              default:
+#pragma unroll
+                for (int k = 0; k < 5; ++k) w[k] = cw[k + 3];
+                w[5] = w[6] = w[7] = 0;
+                break;
+            }
+            const uint32_t meta = reinterpret_cast<const uint32_t*>(
+                st + MT * kATile + kBTile + kCodes)[r * 4 + mslot];
+            dequant_row(B.bits, w, meta, st + MT * kATile, r);
           }
-          const uint32_t meta = reinterpret_cast<const uint32_t*>(
-              st + MT * kATile + kBTile + kCodes)[r * 4 + ((B.grp_off + hg / 2) & 3)];
-          dequant_row(B.bits, w, meta, st + MT * kATile, r);
           fence_proxy_async_smem();
         }
         __syncwarp();
@@ -564,7 +604,7 @@ extern "C" int polyq_linear_gemm(const polyq_dev_layer* L, const void* X, int64_
   P.y = Y;
   P.status = (int*)((uint8_t*)workspace + need - 256);
   rc = polyq_tensor_map_2d(&P.tm_x, P.xg, 2, (uint64_t)KT * BK, (uint64_t)M, (uint64_t)KT * BK * 2,
-                           BK, BM, 64);
+                           BK, MT * BM, 64);
   if (rc) return rc;
   rc = polyq_tensor_map_2d(&P.tm_codes, L->packed, 1, (uint64_t)L->row_stride, (uint64_t)L->N,
                            (uint64_t)L->row_stride, kCodeBox, BN);
