@@ -442,23 +442,30 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) gemv_main(const __grid_c
     if (desc.x & kDescEnd) break;
     const int bits = (int)(desc.x & 0xFFu);
     const int uvalid = (int)(desc.y & 0xFFFFu), g0 = (int)(desc.y >> 16);
-    switch (bits) {
-      case 2: step_mma<NB, 2>(P.magic, P.batch, uvalid, g0, stage, stage, rec, zeros, warp, lane, acc); break;
-      case 3: step_mma<NB, 3>(P.magic, P.batch, uvalid, g0, stage, stage, rec, zeros, warp, lane, acc); break;
-      case 4: step_mma<NB, 4>(P.magic, P.batch, uvalid, g0, stage, stage, rec, zeros, warp, lane, acc); break;
-      case 8: step_mma<NB, 8>(P.magic, P.batch, uvalid, g0, stage, stage, rec, zeros, warp, lane, acc); break;
-      default: step_16<NB>(P.batch, uvalid, stage, rec, zeros, warp, lane, acc); break;
-    }
     if (NB > 1 && (desc.x & kDescPair)) {
-      // the second step of the pair: its box follows the first, its record
-      // follows the first record, its chunks follow in the meta box
-      const uint32_t* rec2 = rec + RB / 4;
-      const int uv2 = (int)desc.w;
+      // two steps of one block and tile: the second one's box follows the
+      // first, its record follows the first record, its chunks follow in the
+      // meta box (the valid-unit counts are not needed: units past a block's
+      // end carry zero activations)
+      if constexpr (NB > 1) {
+        const uint32_t* rec2 = rec + RB / 4;
+        switch (bits) {
+          case 2: step_mma_pair<NB, 2>(P.magic, P.batch, g0, stage, stage + kRows * box_pitch(2, NB), stage, rec, rec2, zeros, warp, lane, acc); break;
+          case 3: step_mma_pair<NB, 3>(P.magic, P.batch, g0, stage, stage + kRows * box_pitch(3, NB), stage, rec, rec2, zeros, warp, lane, acc); break;
+          case 4: step_mma_pair<NB, 4>(P.magic, P.batch, g0, stage, stage + kRows * box_pitch(4, NB), stage, rec, rec2, zeros, warp, lane, acc); break;
+          default:  // 8-bit steps take one box, so pair, only at batch 4
+            if constexpr (nbox_of(8, NB) == 1)
+              step_mma_pair<NB, 8>(P.magic, P.batch, g0, stage, stage + kRows * box_pitch(8, NB), stage, rec, rec2, zeros, warp, lane, acc);
+            break;
+        }
+      }
+    } else {
       switch (bits) {
-        case 2: step_mma<NB, 2>(P.magic, P.batch, uv2, g0 + step_chunks(2, NB), stage + kRows * box_pitch(2, NB), stage, rec2, zeros, warp, lane, acc); break;
-        case 3: step_mma<NB, 3>(P.magic, P.batch, uv2, g0 + step_chunks(3, NB), stage + kRows * box_pitch(3, NB), stage, rec2, zeros, warp, lane, acc); break;
-        case 4: step_mma<NB, 4>(P.magic, P.batch, uv2, g0 + step_chunks(4, NB), stage + kRows * box_pitch(4, NB), stage, rec2, zeros, warp, lane, acc); break;
-        default: step_mma<NB, 8>(P.magic, P.batch, uv2, g0 + step_chunks(8, NB), stage + kRows * box_pitch(8, NB), stage, rec2, zeros, warp, lane, acc); break;
+        case 2: step_mma<NB, 2>(P.magic, P.batch, uvalid, g0, stage, stage, rec, zeros, warp, lane, acc); break;
+        case 3: step_mma<NB, 3>(P.magic, P.batch, uvalid, g0, stage, stage, rec, zeros, warp, lane, acc); break;
+        case 4: step_mma<NB, 4>(P.magic, P.batch, uvalid, g0, stage, stage, rec, zeros, warp, lane, acc); break;
+        case 8: step_mma<NB, 8>(P.magic, P.batch, uvalid, g0, stage, stage, rec, zeros, warp, lane, acc); break;
+        default: step_16<NB>(P.batch, uvalid, stage, rec, zeros, warp, lane, acc); break;
       }
     }
     __syncwarp();

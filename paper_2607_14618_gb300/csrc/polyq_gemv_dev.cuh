@@ -440,6 +440,93 @@ __device__ __forceinline__ void step_mma(uint32_t magic, int batch, int uvalid, 
   }
 }
 
+// Two consecutive one-box steps of a block and tile that share a stage (batch
+// 2-4): the same arithmetic as two step_mma calls, with both steps' loads and
+// MMAs interleaved so that each warp has two independent MMA chains in
+// flight.  The second step's box, record and meta chunks follow the first's.
+template <int NB, int BITS>
+__device__ __forceinline__ void step_mma_pair(uint32_t magic, int batch, int g0,
+                                              const uint8_t* codes0, const uint8_t* codes1,
+                                              const uint8_t* stage, const uint32_t* rec0,
+                                              const uint32_t* rec1, const uint32_t* zeros,
+                                              int warp, int lane, float (&acc)[2][NB]) {
+  constexpr int NGS = step_chunks(BITS, NB);
+  constexpr int NGM = 8 / NB;
+  constexpr int NW = lane_words(BITS, NB);
+  constexpr int LW = rec_lane_words(NB);
+  constexpr int PW = rec_pair_words(NB);
+  constexpr int GP = group_pairs(BITS), GW = group_words(BITS);
+  static_assert(nbox_of(BITS, NB) == 1 && GP % 4 == 0 && NW % GW == 0, "pair geometry");
+  constexpr int GPB = NW / GW;  // groups per step
+  const int g = lane >> 2, t = lane & 3;
+  const int rA = warp * 16 + g, rB = rA + 8;
+  const uint32_t* meta_s = reinterpret_cast<const uint32_t*>(stage + kCodesBytes);
+
+  uint32_t wa[2][NW], wb[2][NW];
+  load_words<BITS, NB>(wa[0], codes0, rA, t);
+  load_words<BITS, NB>(wb[0], codes0, rB, t);
+  load_words<BITS, NB>(wa[1], codes1, rA, t);
+  load_words<BITS, NB>(wb[1], codes1, rB, t);
+
+  const int my_b = g / NGS, my_c = g % NGS;
+  const int dc = my_b < batch ? my_c - lane_unit(BITS, NB, t, 0) / 64 : -1000;
+  const uint32_t* bs[2] = {dc == 0 ? rec0 + (my_b * 4 + t) * LW : zeros,
+                           dc == 0 ? rec1 + (my_b * 4 + t) * LW : zeros};
+
+  float d[2][4][4];
+#pragma unroll
+  for (int k = 0; k < 2; ++k)
+#pragma unroll
+    for (int q = 0; q < 4; ++q) d[k][q][0] = d[k][q][1] = d[k][q][2] = d[k][q][3] = 0.f;
+#pragma unroll
+  for (int qq = 0; qq < GPB; ++qq) {
+#pragma unroll
+    for (int m2 = 0; m2 < GP / 4; ++m2) {
+      const uint4 bv0 = *reinterpret_cast<const uint4*>(bs[0] + qq * GP + 4 * m2);
+      const uint4 bv1 = *reinterpret_cast<const uint4*>(bs[1] + qq * GP + 4 * m2);
+#pragma unroll
+      for (int hh = 0; hh < 2; ++hh) {
+        const int jp = qq * GP + 4 * m2 + 2 * hh;
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+          const uint32_t a0 = make_pair<BITS>(wa[k], jp, magic);
+          const uint32_t a1 = make_pair<BITS>(wb[k], jp, magic);
+          const uint32_t a2 = make_pair<BITS>(wa[k], jp + 1, magic);
+          const uint32_t a3 = make_pair<BITS>(wb[k], jp + 1, magic);
+          const uint4& bv = k ? bv1 : bv0;
+          mma_f16_16816(d[k][(jp / 2) & 3], a0, a1, a2, a3, hh ? bv.z : bv.x, hh ? bv.w : bv.y);
+        }
+      }
+    }
+  }
+#pragma unroll
+  for (int k = 0; k < 2; ++k) {
+    float D[4];
+#pragma unroll
+    for (int v = 0; v < 4; ++v) D[v] = (d[k][0][v] + d[k][1][v]) + (d[k][2][v] + d[k][3][v]);
+    const float* recf = reinterpret_cast<const float*>(k ? rec1 : rec0);
+#pragma unroll
+    for (int cc = 0; cc < 2; ++cc) {
+      const int col = 2 * t + cc;
+      const int be = col / NGS, c = col % NGS;
+      if (be < batch) {
+        const float C1 = recf[PW + be * NGM + c];
+        const float X = recf[PW + NB * NGM + be * NGM + c];
+#pragma unroll
+        for (int r = 0; r < 2; ++r) {
+          const uint32_t m = meta_s[(r ? rB : rA) * kMetaBox + g0 + k * NGS + c];
+          const float sc = __half2float(__ushort_as_half((uint16_t)(m & 0xFFFFu)));
+          const float ze = __half2float(__ushort_as_half((uint16_t)(m >> 16)));
+          const float v = sc * fmaf(-ze, X, D[2 * r + cc] - C1);
+#pragma unroll
+          for (int b = 0; b < NB; ++b)
+            if (b == be) acc[r][b] += v;
+        }
+      }
+    }
+  }
+}
+
 // One 16-bit step: the fp16 weights are the MMA's A operand as stored; column
 // n of B is batch row n.  Lane t holds weights [16t, 16t+16) of each of the
 // two 64-weight boxes.
