@@ -313,34 +313,79 @@ def run_polyq(args):
                                      / (ms_step * 1e-3) / 1e9, 1),
             "per_linear": per_lin_us}
 
-    # end to end through the public API: pinned host x -> device, GEMVs, y -> host
+    # end to end through the public API: pinned host x -> device, GEMVs,
+    # y -> host, the host waiting for every step's results
     e2e = None
     if not args.no_e2e:
-        hx = [torch.from_numpy(np.repeat(x, batch, 0).view(np.int16)).pin_memory() for x in xs_np]
-        hy = [torch.empty((batch, N), dtype=torch.float32).pin_memory() for _, N, _ in LLAMA]
-        dx = [torch.empty((batch, K), dtype=torch.int16, device=device) for _, _, K in LLAMA]
-        h2d = sum(hx[grp[0]].numel() * 2 for grp in GROUPS)
-        d2h = sum(t.numel() * 4 for t in hy)
+        # The step's inputs (one bf16 x per call) and outputs (one fp32 y per
+        # linear) each sit in one contiguous buffer, so that a step moves
+        # them with one host-to-device and one device-to-host copy.
+        in_off, o = {}, 0
+        for grp in GROUPS:
+            in_off[grp[0]] = o
+            o += batch * LLAMA[grp[0]][2]
+        hx_all = torch.empty(o, dtype=torch.int16).pin_memory()
+        for grp in GROUPS:
+            K0 = LLAMA[grp[0]][2]
+            hx_all[in_off[grp[0]]:in_off[grp[0]] + batch * K0] = torch.from_numpy(
+                np.repeat(xs_np[grp[0]], batch, 0).view(np.int16).reshape(-1))
+        dx_all = torch.empty(o, dtype=torch.int16, device=device)
+        dxs = {g0: dx_all[in_off[g0]:in_off[g0] + batch * LLAMA[g0][2]].view(batch, LLAMA[g0][2])
+               .view(torch.bfloat16) for g0 in in_off}
+        out_off, o = [], 0
+        for _, N, _ in LLAMA:
+            out_off.append(o)
+            o += batch * N
+        ys_all = torch.empty(o, dtype=torch.float32, device=device)
+        hy_all = torch.empty(o, dtype=torch.float32).pin_memory()
+        ye = [ys_all[out_off[i]:out_off[i] + batch * N].view(batch, N)
+              for i, (_, N, _) in enumerate(LLAMA)]
+        h2d = hx_all.numel() * 2
+        d2h = hy_all.numel() * 4
         e_steps = max(3, min(args.steps, 50))
+
+        def e2e_step(c):
+            dx_all.copy_(hx_all, non_blocking=True)
+            for grp in GROUPS:
+                polyq.linear_gemv_group([layers[i][c] for i in grp], [dxs[grp[0]]] * len(grp),
+                                        ys=[ye[i] for i in grp], workspace=wbuf, stream=stream)
+            hy_all.copy_(ys_all, non_blocking=True)
+
+        # (1) the calls made eagerly every step
         with torch.cuda.stream(stream):
             for s in range(args.warmup + e_steps):
                 if s == args.warmup:
                     stream.synchronize()
                     ta = time.perf_counter()
-                c = s % args.copies
-                for grp in GROUPS:
-                    dx[grp[0]].copy_(hx[grp[0]], non_blocking=True)
-                    polyq.linear_gemv_group([layers[i][c] for i in grp],
-                                            [dx[grp[0]].view(torch.bfloat16)] * len(grp),
-                                            ys=[ys[i] for i in grp], workspace=wbuf,
-                                            stream=stream)
-                    for i in grp:
-                        hy[i].copy_(ys[i], non_blocking=True)
+                e2e_step(s % args.copies)
+                stream.synchronize()
+            tb = time.perf_counter()
+        eager = {"value": round(step_bytes * e_steps / (tb - ta) / 1e12, 4), "unit": "TB/s",
+                 "ms_per_step": round(1e3 * (tb - ta) / e_steps, 4),
+                 "mode": "API calls and copies issued eagerly every step"}
+        # (2) each layer copy's step (copies and API calls) captured once as a
+        # CUDA graph, replayed every step, the host synchronising every step
+        e_graphs = []
+        for c in range(args.copies):
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                e2e_step(c)
+            e_graphs.append(g)
+        with torch.cuda.stream(stream):
+            for s in range(args.warmup + e_steps):
+                if s == args.warmup:
+                    stream.synchronize()
+                    ta = time.perf_counter()
+                e_graphs[s % args.copies].replay()
                 stream.synchronize()
             tb = time.perf_counter()
         e2e = {"value": round(step_bytes * e_steps / (tb - ta) / 1e12, 4), "unit": "TB/s",
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": e_steps,
-               "ms_per_step": round(1e3 * (tb - ta) / e_steps, 4)}
+               "ms_per_step": round(1e3 * (tb - ta) / e_steps, 4),
+               "mode": "each step's H2D copy of its inputs, 4 GEMV API calls and D2H copy of its "
+                       "7 outputs captured as a CUDA graph, replayed and synchronised every step",
+               "eager": eager}
+        del e_graphs
 
     decode = None
     if not args.no_decode:
