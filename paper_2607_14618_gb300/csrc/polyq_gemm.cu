@@ -22,9 +22,11 @@
 //                   rows per thread; afterwards all eight drain the
 //                   accumulator with tcgen05.ld and store fp32 Y.
 //     Four pipeline stages.  When the (M, N) tiles cannot fill the GPU the K
-//     range is split and the pieces are added into a zeroed Y (so the order of
-//     those additions varies); otherwise Y is stored directly.  Every wait is
-//     bounded and reports through the workspace status word.
+//     range is split, uniformly or stream-K (each CTA an equal contiguous
+//     share of all (tile, K tile) pairs), and the pieces are added into a
+//     zeroed Y (so the order of those additions varies); otherwise Y is
+//     stored directly.  Every wait is bounded and reports through the
+//     workspace status word.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
@@ -55,7 +57,9 @@ constexpr int kMeta = BN * 16;                  // 4 KB
 constexpr int kStageG = MT * kATile + kBTile + kCodes + kMeta;  // 48 KB
 constexpr int kThreadsG = 320;
 constexpr int kDqWarps = 8;
-constexpr double kUnitCostTiles = 12.0;  // per-unit overhead, in K tiles, of the split model
+constexpr double kUnitCostTiles = 12.0;  // per-piece overhead, in K-tile stages, of the split model
+constexpr double kStageSeconds = 0.6e-6;  // one K-tile stage of a CTA, measured
+constexpr double kZeroBytesPerS = 5e12;   // the pre-pass zeroing Y
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kIdesc = umma_idesc_f16(BM, BN);
 
@@ -73,6 +77,7 @@ struct GmParams {
   int n_blocks;
   int M, N, K, KT;
   int units_m, units_n, ksplit, units;  // work units: (M pair, N tile, K split)
+  int streamk;  // 1: each CTA takes an equal contiguous range of (unit, K tile) pairs
   int has_meta;
   const __nv_bfloat16* x;
   const int32_t* gather;
@@ -107,6 +112,47 @@ __device__ __forceinline__ bool mbar_wait_sleep(uint32_t bar, uint32_t parity) {
     if (mbar_try_wait_hint(bar, parity, kSuspendHintNs)) return true;
   return false;
 }
+
+// The pieces of work a CTA takes, in order: an output tile (um, un) and a
+// range [kt_lo, kt_hi) of its K tiles.  Units are strided over the grid, each
+// with its K split's range; with `streamk`, a CTA takes the K tiles
+// [T*b/C, T*(b+1)/C) of the T = units * KT (unit, K tile) pairs in unit-major
+// order, which cuts at most two units per CTA short.  Every role of a CTA
+// walks the same sequence.
+struct Pieces {
+  long long g, g_hi;
+  int u;
+  __device__ __forceinline__ void init(const GmParams& P) {
+    if (P.streamk) {
+      const long long T = (long long)P.units * P.KT;
+      g = T * blockIdx.x / gridDim.x;
+      g_hi = T * (blockIdx.x + 1) / gridDim.x;
+    } else {
+      u = blockIdx.x;
+    }
+  }
+  __device__ __forceinline__ bool next(const GmParams& P, int& um, int& un, int& kt_lo,
+                                       int& kt_hi) {
+    int uu;
+    if (P.streamk) {
+      if (g >= g_hi) return false;
+      uu = (int)(g / P.KT);
+      kt_lo = (int)(g - (long long)uu * P.KT);
+      kt_hi = (int)min((long long)P.KT, (long long)kt_lo + (g_hi - g));
+      g += kt_hi - kt_lo;
+    } else {
+      if (u >= P.units) return false;
+      uu = u;
+      u += gridDim.x;
+      const int ks = uu / (P.units_m * P.units_n);
+      kt_lo = (int)((long long)ks * P.KT / P.ksplit);
+      kt_hi = (int)((long long)(ks + 1) * P.KT / P.ksplit);
+    }
+    um = uu % P.units_m;
+    un = (uu / P.units_m) % P.units_n;
+    return true;
+  }
+};
 
 __device__ __forceinline__ int find_kblock(const GmBlock* blk, int nblk, int kt) {
   int b = 0;
@@ -147,7 +193,7 @@ __global__ void __launch_bounds__(256) gemm_prep(const __grid_constant__ GmParam
   }
   if (blockIdx.x == 0 && threadIdx.x == 0) *P.status = 0;
   __syncthreads();
-  if (P.ksplit > 1) {
+  if (P.ksplit > 1 || P.streamk) {
     const long long total4 = (long long)P.M * P.N / 4;
     for (long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x; e < total4;
          e += (long long)gridDim.x * blockDim.x)
@@ -306,7 +352,6 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
   const uint32_t tmem = tmem_base_slot;
   pdl_trigger();
 
-  const int KT = P.KT;
   const int nblk = P.n_blocks;
   auto stage_ptr = [&](int s) { return smem + s * kStageG; };
   auto fail = [&](int code) {
@@ -323,11 +368,10 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
       prefetch_tmap(&P.tm_w16);
       pdl_wait();  // Xg comes from the pre-pass
       int kg = 0;
-      for (int u = blockIdx.x; u < P.units && !s_abort; u += gridDim.x) {
-        const int um = u % P.units_m, un = (u / P.units_m) % P.units_n;
-        const int ks = u / (P.units_m * P.units_n);
-        const int kt_lo = (int)((long long)ks * KT / P.ksplit);
-        const int kt_hi = (int)((long long)(ks + 1) * KT / P.ksplit);
+      Pieces pc;
+      pc.init(P);
+      int um, un, kt_lo, kt_hi;
+      while (!s_abort && pc.next(P, um, un, kt_lo, kt_hi)) {
         for (int kt = kt_lo; kt < kt_hi && !s_abort; ++kt, ++kg) {
           const int s = kg % kStagesG, use = kg / kStagesG;
           if (use > 0 && !mbar_wait_sleep(smem_u32(&bar_sfree[s]), (use - 1) & 1)) {
@@ -359,10 +403,10 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
     // ---------------- MMA issuer ----------------
     if (lane == 0) {
       int kg = 0, uc = 0;
-      for (int u = blockIdx.x; u < P.units && !s_abort; u += gridDim.x, ++uc) {
-        const int ks = u / (P.units_m * P.units_n);
-        const int kt_lo = (int)((long long)ks * KT / P.ksplit);
-        const int kt_hi = (int)((long long)(ks + 1) * KT / P.ksplit);
+      Pieces pc;
+      pc.init(P);
+      int um, un, kt_lo, kt_hi;
+      for (; !s_abort && pc.next(P, um, un, kt_lo, kt_hi); ++uc) {
         if (uc > 0 && !mbar_wait_sleep(smem_u32(&bar_acce), (uc - 1) & 1)) {
           fail(kStatusTimeoutEmpty);
           break;
@@ -403,11 +447,10 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
     const int q = warp & 3;          // TMEM lane quarter this warp may access
     const int half = (warp - 2) >> 2;
     int kg = 0, uc = 0;
-    for (int u = blockIdx.x; u < P.units && !s_abort; u += gridDim.x, ++uc) {
-      const int um = u % P.units_m, un = (u / P.units_m) % P.units_n;
-      const int ks = u / (P.units_m * P.units_n);
-      const int kt_lo = (int)((long long)ks * KT / P.ksplit);
-      const int kt_hi = (int)((long long)(ks + 1) * KT / P.ksplit);
+    Pieces pc;
+    pc.init(P);
+    int um, un, kt_lo, kt_hi;
+    for (; !s_abort && pc.next(P, um, un, kt_lo, kt_hi); ++uc) {
       for (int kt = kt_lo; kt < kt_hi && !s_abort; ++kt, ++kg) {
         if ((kg & 1) != grp) continue;
         const int s = kg % kStagesG, use = kg / kStagesG;
@@ -483,7 +526,7 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
           if (m < P.M) {
             float* dst = P.y + (size_t)m * P.N + n0;
             const bool vec = n0 + 32 <= P.N && (P.N % 4) == 0;
-            if (P.ksplit > 1) {  // Y was zeroed by the pre-pass: add this K range
+            if (P.ksplit > 1 || P.streamk) {  // Y was zeroed by the pre-pass: add this K range
               if (vec) {
 #pragma unroll
                 for (int j = 0; j < 8; ++j)
@@ -521,7 +564,10 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
       // the last commit of this CTA went to bar_accf; its completion means all
       // MMAs have finished reading shared memory and writing TMEM
       int uc = 0;
-      for (int u = blockIdx.x; u < P.units; u += gridDim.x) ++uc;
+      Pieces pc;
+      pc.init(P);
+      int um, un, kt_lo, kt_hi;
+      while (pc.next(P, um, un, kt_lo, kt_hi)) ++uc;
       if (uc > 0) mbar_wait(smem_u32(&bar_accf), (uc - 1) & 1);
     }
     __syncwarp();
@@ -623,25 +669,38 @@ extern "C" int polyq_linear_gemm(const polyq_dev_layer* L, const void* X, int64_
   int sms = 0;
   rc = polyq_sm_count(&sms);
   if (rc) return rc;
-  // Split K when the (M, N) tiles fill the SMs poorly: take the split with
-  // the least modelled time, whole waves of units times (K tiles per unit +
-  // a per-unit cost for filling the pipeline and adding the tile into Y).
-  // Each split keeps at least 16 K tiles; near ties go to fewer splits.
+  // Split K when the (M, N) tiles fill the SMs poorly.  The modelled time, in
+  // K-tile stages of one CTA, is for a uniform split into k ranges: whole
+  // waves of units times (K tiles per unit + a per-piece cost for filling the
+  // pipeline and adding the tile into Y); for stream-K: the K tiles of one
+  // CTA's equal share plus the per-piece cost of the (at most three) pieces
+  // it touches.  Both add the zeroing of Y when they split.  Each uniform
+  // split keeps at least 16 K tiles; near ties go to the simpler choice.
   {
     const int mn = P.units_m * P.units_n;
+    const bool can_split = (P.N % 4) == 0;  // zeroing writes float4
+    const double zero = (double)M * P.N * 4.0 / kZeroBytesPerS / kStageSeconds;
     int ks = 1;
     double best = 1e300;
-    const int kmax = (P.N % 4) != 0 ? 1 : std::max(1, std::min(64, KT / 16));  // zeroing writes float4
+    const int kmax = can_split ? std::max(1, std::min(64, KT / 16)) : 1;
     for (int k = 1; k <= kmax; ++k) {
       const long long waves = ((long long)mn * k + sms - 1) / sms;
-      const double t = (double)waves * ((double)KT / k + kUnitCostTiles);
+      const double t = (double)waves * ((double)KT / k + kUnitCostTiles) + (k > 1 ? zero : 0.0);
       if (t < 0.98 * best) {
         best = t;
         ks = k;
       }
     }
-    P.ksplit = ks;
-    P.units = mn * ks;
+    const double share = std::ceil((double)mn * KT / sms);
+    const double t_sk = share + kUnitCostTiles * (std::ceil(share / KT) + 1.0) + zero;
+    if (can_split && (long long)mn * KT >= sms && t_sk < 0.98 * best) {
+      P.streamk = 1;
+      P.ksplit = 1;
+      P.units = mn;
+    } else {
+      P.ksplit = ks;
+      P.units = mn * ks;
+    }
   }
   static bool attr_done[8] = {false};
   int dev = 0;
@@ -670,7 +729,7 @@ extern "C" int polyq_linear_gemm(const polyq_dev_layer* L, const void* X, int64_
     return polyq_set_error(POLYQ_ECUDA, "polyq_linear_gemm: prep launch: %s", cudaGetErrorString(e));
   // no programmatic overlap for the main kernel: it owns all of TMEM on an SM
   cfg.numAttrs = 0;
-  cfg.gridDim = dim3((unsigned)std::min(P.units, sms));
+  cfg.gridDim = dim3((unsigned)(P.streamk ? sms : std::min(P.units, sms)));
   cfg.blockDim = dim3(kThreadsG);
   cfg.dynamicSmemBytes = smem;
   e = cudaLaunchKernelEx(&cfg, gemm_main, P);

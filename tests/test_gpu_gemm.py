@@ -22,6 +22,8 @@ def _x_dev(xb):
     (130, 257, 1536, 6.0, 55, False),    # B = 6: many 8-bit channels
     (64, 64, 320, 16.0, 56, False),      # all 16-bit
     (96, 96, 640, 2.0, 57, False),       # all 2-bit
+    (300, 520, 2100, 3.0, 60, True),     # stream-K: ~3 K tiles per CTA, cut across tiles
+    (64, 2000, 4000, 3.0, 61, False),    # uniform K split into 8 ranges
 ])
 def test_gemm_matches_oracle(polyq_lib, M, N, K, B, seed, forced):
     W, a = synth.layer_weights(N, K, seed)
