@@ -143,9 +143,6 @@ struct ItemPos {
     while (bi + 1 < S.n_blocks[l] && s >= S.blk[l][bi + 1].step0) ++bi;
     j = s - S.blk[l][bi].step0;
   }
-  __device__ __forceinline__ bool tile_end(const GvShared& S) const {
-    return s == S.steps[l] - 1;
-  }
   __device__ __forceinline__ void next(const GvShared& S, int nl) {
     ++s;
     ++j;
@@ -534,8 +531,8 @@ int steps_of(const polyq_dev_layer* L, int nb, GvBlock* blk) {
   return s;
 }
 
-// CTAs of one launch: all of them must be resident at once (an owner waits
-// for pieces of later CTAs), so never more than the device holds.
+// CTAs of one launch: persistent, one wave of them (never more than the
+// device holds at once) and no more than there are work items.
 int grid_for(int items, int* grid) {
   int sms = 0;
   int rc = polyq_sm_count(&sms);
