@@ -129,6 +129,25 @@ def _dist():
     return ws, rank, local
 
 
+def max_over_ranks(ms, ws, device=None):
+    """The job's time: the slowest replica's (one all-reduce over the ranks'
+    timings; ``device`` is where the process group's backend wants the
+    tensor, a GPU for NCCL, the CPU for gloo)."""
+    if ws <= 1:
+        return float(ms)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(ms)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_tbs(ws, step_bytes, steps, ms):
+    """Whole-job throughput: every replica streams ``step_bytes`` per step,
+    over the slowest replica's time."""
+    return ws * step_bytes * steps / (ms * 1e-3) / 1e12
+
+
 def build_layers(polyq, synth, budget, copies, device):
     """Pack the seven linears once (seeded), upload, and clone on device.
     Linears of one launch group share their input activation."""
@@ -257,13 +276,9 @@ def run_polyq(args):
         torch.cuda.synchronize()
     if ws > 1:
         dist.barrier()
-    ms = t0.elapsed_time(t1)
-    if ws > 1:
-        t = torch.tensor([ms], device=device)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(t0.elapsed_time(t1), ws, device)
     ms_step = ms / args.steps
-    value_tbs = ws * step_bytes * args.steps / (ms * 1e-3) / 1e12
+    value_tbs = job_tbs(ws, step_bytes, args.steps, ms)
 
     # Roofline of the dominant kernel.  The timed region holds only GEMV
     # launches (pre-pass + streaming kernel per linear), back to back, so its
