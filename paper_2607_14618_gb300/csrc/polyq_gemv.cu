@@ -418,13 +418,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) gemv_main(const __grid_c
   }
 
   // ---------------- consumers ----------------
-  const int g = lane >> 2, t = lane & 3;
   pdl_wait();  // y, the workspace and the records are this call's from here on
-  float acc[2][NB];
-#pragma unroll
-  for (int r = 0; r < 2; ++r)
-#pragma unroll
-    for (int b = 0; b < NB; ++b) acc[r][b] = 0.f;
+  float acc[2] = {0.f, 0.f};  // this lane's row sums (see lane_batch)
   int slot = 0;
   uint32_t phase = 0;
   for (;;) {
@@ -474,17 +469,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) gemv_main(const __grid_c
 
     if (desc.x & 0x100u) {
       // ---- add this warp's 16 rows of the tile piece into y ----
-      // Sum the four lanes of each row; lane t adds batch row t.  A tile
-      // whose steps are split over CTAs gets one addition per piece.
-#pragma unroll
-      for (int r = 0; r < 2; ++r)
-#pragma unroll
-        for (int b = 0; b < NB; ++b) {
-          float v = acc[r][b];
-          v += __shfl_xor_sync(0xffffffffu, v, 1);
-          v += __shfl_xor_sync(0xffffffffu, v, 2);
-          acc[r][b] = v;
-        }
+      // A tile whose steps are split over CTAs gets one addition per piece.
       const int l = (int)(desc.x >> 16);
       float* y = P.L[0].y;
       int N = P.L[0].N;
@@ -494,15 +479,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) gemv_main(const __grid_c
           y = P.L[q].y;
           N = P.L[q].N;
         }
-#pragma unroll
-      for (int r = 0; r < 2; ++r) {
-        const int n = (int)desc.z * kRows + warp * 16 + g + 8 * r;
-#pragma unroll
-        for (int b = 0; b < NB; ++b)
-          if (b == t && b < P.batch && n < N) atomicAdd(y + (size_t)b * N + n, acc[r][b]);
-#pragma unroll
-        for (int b = 0; b < NB; ++b) acc[r][b] = 0.f;
-      }
+      flush_rows<NB>(acc, y, N, P.batch, (int)desc.z * kRows + warp * 16, lane);
     }
   }
 }

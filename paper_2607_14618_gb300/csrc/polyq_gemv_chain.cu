@@ -391,12 +391,7 @@ __global__ void __launch_bounds__(kThreads, kChCtasPerSm) gemv_chain(const __gri
   }
 
   // ---------------- consumers ----------------
-  const int g = lane >> 2, t = lane & 3;
-  float acc[2][NB];
-#pragma unroll
-  for (int r = 0; r < 2; ++r)
-#pragma unroll
-    for (int b = 0; b < NB; ++b) acc[r][b] = 0.f;
+  float acc[2] = {0.f, 0.f};  // this lane's row sums (see lane_batch)
   int slot = 0;
   uint32_t phase = 0;
   unsigned gen = 0;
@@ -480,29 +475,9 @@ __global__ void __launch_bounds__(kThreads, kChCtasPerSm) gemv_chain(const __gri
         __syncwarp();
         if (lane == 0) mbar_arrive(empty0 + 8 * slot);
         if (desc.x & 0x100u) {
-          // add this warp's 16 rows of the tile piece into y; lane t adds
-          // batch row t
-#pragma unroll
-          for (int rr = 0; rr < 2; ++rr)
-#pragma unroll
-            for (int b = 0; b < NB; ++b) {
-              float v = acc[rr][b];
-              v += __shfl_xor_sync(0xffffffffu, v, 1);
-              v += __shfl_xor_sync(0xffffffffu, v, 2);
-              acc[rr][b] = v;
-            }
+          // add this warp's 16 rows of the tile piece into y
           const int l = (int)(desc.x >> 16);
-          float* y = S.y[l];
-          const int N = S.N[l];
-#pragma unroll
-          for (int rr = 0; rr < 2; ++rr) {
-            const int n = (int)desc.z * kRows + warp * 16 + g + 8 * rr;
-#pragma unroll
-            for (int b = 0; b < NB; ++b)
-              if (b == t && b < P.batch && n < N) atomicAdd(y + (size_t)b * N + n, acc[rr][b]);
-#pragma unroll
-            for (int b = 0; b < NB; ++b) acc[rr][b] = 0.f;
-          }
+          flush_rows<NB>(acc, S.y[l], S.N[l], P.batch, (int)desc.z * kRows + warp * 16, lane);
         }
       }
       if (++slot == kStages) {

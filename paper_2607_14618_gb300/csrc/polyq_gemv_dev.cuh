@@ -295,6 +295,42 @@ __device__ __forceinline__ void rec_store(const XIn& in, const GvBlock& B, int j
 }
 
 // ---------------------------------------------------------------------------
+// row sums of a tile piece
+// ---------------------------------------------------------------------------
+// Lane t of a quad keeps one partial sum per row for batch row t*NB/4: at
+// batch 1 every lane row 0, at batch 2 lanes 0-1 row 0 and lanes 2-3 row 1,
+// at batch 4 lane t row t.  For 2/3/4/8-bit steps that is the batch row of
+// both MMA columns the lane holds (columns of other rows are past the
+// batch); 16-bit steps hand their values to the first lane of the group.
+template <int NB>
+__device__ __forceinline__ int lane_batch(int t) {
+  return t * NB / 4;
+}
+template <int NB>
+__device__ __forceinline__ bool lane_first(int t) {
+  return t % (4 / NB) == 0;
+}
+
+// Add the warp's 16 rows (row0 + g, row0 + g + 8) of a finished tile piece
+// into y, summing first the lanes of a quad that hold the same batch row, and
+// clear the sums.
+template <int NB>
+__device__ __forceinline__ void flush_rows(float (&acc)[2], float* y, int N, int batch, int row0,
+                                           int lane) {
+  const int g = lane >> 2, t = lane & 3;
+  const int bl = lane_batch<NB>(t);
+#pragma unroll
+  for (int r = 0; r < 2; ++r) {
+    float v = acc[r];
+    if (NB <= 2) v += __shfl_xor_sync(0xffffffffu, v, 1);
+    if (NB == 1) v += __shfl_xor_sync(0xffffffffu, v, 2);
+    const int n = row0 + g + 8 * r;
+    if (lane_first<NB>(t) && bl < batch && n < N) atomicAdd(y + (size_t)bl * N + n, v);
+    acc[r] = 0.f;
+  }
+}
+
+// ---------------------------------------------------------------------------
 // MMA steps
 // ---------------------------------------------------------------------------
 template <int BITS>
@@ -360,7 +396,7 @@ __device__ __forceinline__ void step_mma(uint32_t magic, int batch, int uvalid, 
                                          const uint8_t* codes, const uint8_t* stage,
                                          const uint32_t* rec,
                                          const uint32_t* zeros, int warp, int lane,
-                                         float (&acc)[2][NB]) {
+                                         float (&acc)[2]) {
   constexpr int U = step_units(BITS, NB);
   constexpr int NGS = step_chunks(BITS, NB);
   constexpr int NGM = 8 / NB;
@@ -431,10 +467,7 @@ __device__ __forceinline__ void step_mma(uint32_t magic, int batch, int uvalid, 
         const uint32_t m = meta_s[(r ? rB : rA) * kMetaBox + g0 + c];
         const float sc = __half2float(__ushort_as_half((uint16_t)(m & 0xFFFFu)));
         const float ze = __half2float(__ushort_as_half((uint16_t)(m >> 16)));
-        const float v = sc * fmaf(-ze, X, D[2 * r + cc] - C1);
-#pragma unroll
-        for (int b = 0; b < NB; ++b)
-          if (b == be) acc[r][b] += v;
+        acc[r] += sc * fmaf(-ze, X, D[2 * r + cc] - C1);  // be is this lane's row
       }
     }
   }
@@ -449,7 +482,7 @@ __device__ __forceinline__ void step_mma_pair(uint32_t magic, int batch, int g0,
                                               const uint8_t* codes0, const uint8_t* codes1,
                                               const uint8_t* stage, const uint32_t* rec0,
                                               const uint32_t* rec1, const uint32_t* zeros,
-                                              int warp, int lane, float (&acc)[2][NB]) {
+                                              int warp, int lane, float (&acc)[2]) {
   constexpr int NGS = step_chunks(BITS, NB);
   constexpr int NGM = 8 / NB;
   constexpr int NW = lane_words(BITS, NB);
@@ -517,10 +550,7 @@ __device__ __forceinline__ void step_mma_pair(uint32_t magic, int batch, int g0,
           const uint32_t m = meta_s[(r ? rB : rA) * kMetaBox + g0 + k * NGS + c];
           const float sc = __half2float(__ushort_as_half((uint16_t)(m & 0xFFFFu)));
           const float ze = __half2float(__ushort_as_half((uint16_t)(m >> 16)));
-          const float v = sc * fmaf(-ze, X, D[2 * r + cc] - C1);
-#pragma unroll
-          for (int b = 0; b < NB; ++b)
-            if (b == be) acc[r][b] += v;
+          acc[r] += sc * fmaf(-ze, X, D[2 * r + cc] - C1);  // be is this lane's row
         }
       }
     }
@@ -534,7 +564,7 @@ template <int NB>
 __device__ __forceinline__ void step_16(int batch, int uvalid,
                                         const uint8_t* stage, const uint32_t* rec,
                                         const uint32_t* zeros, int warp, int lane,
-                                        float (&acc)[2][NB]) {
+                                        float (&acc)[2]) {
   constexpr int LW = rec_lane_words(NB);
   constexpr int PITCH = kPitchSplit;
   static_assert(box_pitch(16, NB) == PITCH && nbox_of(16, NB) == 2, "16-bit geometry");
@@ -563,15 +593,21 @@ __device__ __forceinline__ void step_16(int batch, int uvalid,
       }
     }
   }
+  // column c of D is batch row c: lane t holds rows 2t and 2t+1, and the
+  // first lane of each group takes its row's value from there
+  if constexpr (NB == 1) {
+    // row 0 is column 0, which lane 0 of the quad holds already
 #pragma unroll
-  for (int cc = 0; cc < 2; ++cc) {
-    const int be = 2 * t + cc;
+    for (int r = 0; r < 2; ++r)
+      if (t == 0) acc[r] += d[0][2 * r] + d[1][2 * r];
+  } else {
+    const int bl = lane_batch<NB>(t);
+    const int src = (lane & ~3) | (bl >> 1);
 #pragma unroll
     for (int r = 0; r < 2; ++r) {
-      const float v = d[0][2 * r + cc] + d[1][2 * r + cc];
-#pragma unroll
-      for (int b = 0; b < NB; ++b)
-        if (b == be) acc[r][b] += v;
+      const float v0 = __shfl_sync(0xffffffffu, d[0][2 * r] + d[1][2 * r], src);
+      const float v1 = __shfl_sync(0xffffffffu, d[0][2 * r + 1] + d[1][2 * r + 1], src);
+      if (lane_first<NB>(t)) acc[r] += (bl & 1) ? v1 : v0;
     }
   }
 }
