@@ -423,9 +423,12 @@ __device__ __forceinline__ void step_mma(uint32_t magic, int batch, int uvalid, 
   const int dc = my_b < batch ? my_c - lane_unit(BITS, NB, t, 0) / 64 : -1000;
   const uint32_t* brow = rec + (my_b * 4 + t) * LW;
 
-  float d[4][4];
+  // independent accumulator sets for the step's MMA chain: four for the 32
+  // MMAs of a batch-1 step, two for the 8-16 of a batch 2-4 step
+  constexpr int NACC = NB == 1 ? 4 : 2;
+  float d[NACC][4];
 #pragma unroll
-  for (int q = 0; q < 4; ++q) d[q][0] = d[q][1] = d[q][2] = d[q][3] = 0.f;
+  for (int q = 0; q < NACC; ++q) d[q][0] = d[q][1] = d[q][2] = d[q][3] = 0.f;
 #pragma unroll
   for (int h = 0; h < NBX; ++h) {
     if (h == 1 && uvalid <= U / 2) break;  // the second half of the step is empty
@@ -443,14 +446,17 @@ __device__ __forceinline__ void step_mma(uint32_t magic, int batch, int uvalid, 
           const uint32_t a1 = make_pair<BITS>(wb, jp, magic);
           const uint32_t a2 = make_pair<BITS>(wa, jp + 1, magic);
           const uint32_t a3 = make_pair<BITS>(wb, jp + 1, magic);
-          mma_f16_16816(d[(jp / 2) & 3], a0, a1, a2, a3, hh ? bv.z : bv.x, hh ? bv.w : bv.y);
+          mma_f16_16816(d[(jp / 2) % NACC], a0, a1, a2, a3, hh ? bv.z : bv.x, hh ? bv.w : bv.y);
         }
       }
     }
   }
   float D[4];
 #pragma unroll
-  for (int v = 0; v < 4; ++v) D[v] = (d[0][v] + d[1][v]) + (d[2][v] + d[3][v]);
+  for (int v = 0; v < 4; ++v) {
+    D[v] = d[0][v] + d[1][v];
+    if constexpr (NACC == 4) D[v] += d[2][v] + d[3][v];
+  }
 
   // epilogue: columns 2t, 2t+1 -> (batch, chunk) (col / NGS, col % NGS);
   // g0 is the step's first group in the meta box
@@ -506,11 +512,11 @@ __device__ __forceinline__ void step_mma_pair(uint32_t magic, int batch, int g0,
   const uint32_t* bs[2] = {dc == 0 ? rec0 + (my_b * 4 + t) * LW : zeros,
                            dc == 0 ? rec1 + (my_b * 4 + t) * LW : zeros};
 
-  float d[2][4][4];
+  float d[2][2][4];  // per step two accumulator sets: four independent chains
 #pragma unroll
   for (int k = 0; k < 2; ++k)
 #pragma unroll
-    for (int q = 0; q < 4; ++q) d[k][q][0] = d[k][q][1] = d[k][q][2] = d[k][q][3] = 0.f;
+    for (int q = 0; q < 2; ++q) d[k][q][0] = d[k][q][1] = d[k][q][2] = d[k][q][3] = 0.f;
 #pragma unroll
   for (int qq = 0; qq < GPB; ++qq) {
 #pragma unroll
@@ -527,7 +533,7 @@ __device__ __forceinline__ void step_mma_pair(uint32_t magic, int batch, int g0,
           const uint32_t a2 = make_pair<BITS>(wa[k], jp + 1, magic);
           const uint32_t a3 = make_pair<BITS>(wb[k], jp + 1, magic);
           const uint4& bv = k ? bv1 : bv0;
-          mma_f16_16816(d[k][(jp / 2) & 3], a0, a1, a2, a3, hh ? bv.z : bv.x, hh ? bv.w : bv.y);
+          mma_f16_16816(d[k][(jp / 2) & 1], a0, a1, a2, a3, hh ? bv.z : bv.x, hh ? bv.w : bv.y);
         }
       }
     }
@@ -536,7 +542,7 @@ __device__ __forceinline__ void step_mma_pair(uint32_t magic, int batch, int g0,
   for (int k = 0; k < 2; ++k) {
     float D[4];
 #pragma unroll
-    for (int v = 0; v < 4; ++v) D[v] = (d[k][0][v] + d[k][1][v]) + (d[k][2][v] + d[k][3][v]);
+    for (int v = 0; v < 4; ++v) D[v] = d[k][0][v] + d[k][1][v];
     const float* recf = reinterpret_cast<const float*>(k ? rec1 : rec0);
 #pragma unroll
     for (int cc = 0; cc < 2; ++cc) {
