@@ -51,6 +51,7 @@ TRAFFIC = {"bytes_per_step": 143138000,
            "sources_sha1": "73d670085494973fe8bca7cad4665ca617e383e4",
            "profile": "profiles/gemv_decode_llama13b_b3_launches.md"}
 GEMV_SOURCES = ("polyq_gemv.cu", "polyq_gemv_dev.cuh", "polyq_gemv_layout.cuh", "polyq_dev.cuh")
+REF_SECONDS = 120.0  # the reference arm's warm-up and timed steps together
 
 
 def _gemv_sources_sha1():
@@ -857,6 +858,16 @@ def bench_gemm(polyq, synth, torch, device, stream, args, tf_burst, tf_sus):
     return res
 
 
+def sample_bytes(L, x, N):
+    """Algorithmic bytes of an oracle run on a row sample of a linear with N
+    rows: the sample's packed codes and metadata, plus the layer's
+    activations, gather indices and outputs in proportion to the sample's
+    share of the rows (over the full layer they are spread over all N)."""
+    rows = L["N"]
+    return (L["packed"].nbytes + L["meta"].nbytes
+            + (x.size * 2 + L["K"] * 4 + x.shape[0] * N * 4) * rows / N)
+
+
 def _blas_threads():
     v = os.environ.get("OPENBLAS_NUM_THREADS") or os.environ.get("OMP_NUM_THREADS")
     return int(v) if v else os.cpu_count()
@@ -901,9 +912,9 @@ def cpu_baseline_child(seconds):
     nbytes = 0
     t0 = time.perf_counter()
     while time.perf_counter() - t0 < seconds:
-        for L, x in layers:
+        for (L, x), (_, N, _) in zip(layers, LLAMA):
             O.linear(L, x)
-            nbytes += L["packed"].nbytes + L["meta"].nbytes + x.size * 2 + L["K"] * 4 + rows * 4
+            nbytes += sample_bytes(L, x, N)
     dt = time.perf_counter() - t0
     return {"value": round(nbytes / dt / 1e12, 8), "unit": "TB/s",
             "cores": _blas_threads(), "host_cpus": os.cpu_count(),
@@ -913,32 +924,57 @@ def cpu_baseline_child(seconds):
 
 
 def run_reference(args):
+    """The reference arm: the oracle's linear on the host cores, on a row
+    sample of each of the seven linears per step.  The sample is sized so that
+    the warm-up and timed steps together take about ``REF_SECONDS`` whatever
+    --steps is (from 1 to 128 rows per linear; the metric is bytes per second,
+    so the sample size does not change what is measured)."""
     ws, rank, _ = _dist()
     if rank != 0:
         return
     from oracle import polyq_oracle as O
     from paper_2607_14618_gb300 import synth
-    rows = 128
-    layers = []
+    max_rows = 128
+    srcs = []  # (first max_rows rows of W, channel magnitudes, widths) per linear
     for i, (name, N, K) in enumerate(LLAMA):
         W, a = synth.layer_weights(N, K, synth.seed_for(2, i))
         bits = O.allocate_bits(O.saliency(W, a), args.budget)
-        L = O.pack_layer(W[:rows], a, args.budget, bits=bits)
-        _, x = synth.activations(a, 1, synth.seed_for(2, i))
-        layers.append((L, x))
+        srcs.append((W[:max_rows].copy(), a, bits))
         del W
 
-    def step():
+    def build(rows):
+        out = []
+        for i, (Wr, a, bits) in enumerate(srcs):
+            L = O.pack_layer(Wr[:rows], a, args.budget, bits=bits)
+            _, x = synth.activations(a, 1, synth.seed_for(2, i))
+            out.append((L, x))
+        return out
+
+    def step(layers):
         n = 0
-        for L, x in layers:
+        for (L, x), (_, N, _) in zip(layers, LLAMA):
             O.linear(L, x)
-            n += L["packed"].nbytes + L["meta"].nbytes + x.size * 2 + L["K"] * 4 + rows * 4
+            n += sample_bytes(L, x, N)
         return n
 
+    def step_seconds(rows):
+        layers = build(rows)
+        step(layers)
+        t0 = time.perf_counter()
+        for _ in range(3):
+            step(layers)
+        return (time.perf_counter() - t0) / 3
+
+    t1, t8 = step_seconds(1), step_seconds(8)
+    per_row = max((t8 - t1) / 7, 1e-6)
+    fixed = max(t1 - per_row, 0.0)
+    rows = int((REF_SECONDS / max(args.steps + args.warmup, 1) - fixed) / per_row)
+    rows = max(1, min(max_rows, rows))
+    layers = build(rows)
     for _ in range(args.warmup):
-        step()
+        step(layers)
     t0 = time.perf_counter()
-    nb = sum(step() for _ in range(args.steps))
+    nb = sum(step(layers) for _ in range(args.steps))
     dt = time.perf_counter() - t0
     v = nb / dt / 1e12
     out = {"impl": "reference", "metric": METRIC, "value": round(v, 8), "unit": "TB/s",
@@ -948,7 +984,8 @@ def run_reference(args):
            "config": {"workload": WORKLOAD, "budget_bits": args.budget, "batch": 1},
            "cpu_baseline": {"kind": "oracle", "cores": _blas_threads(), "host_cpus": os.cpu_count(),
                             "value": round(v, 8), "unit": "TB/s",
-                            "sample": f"{rows} output rows of each of the 7 linears per step"},
+                            "sample": f"{rows} output rows of each of the 7 linears per step "
+                                      f"(sized for about {REF_SECONDS:.0f} s of steps)"},
            "e2e": {"value": round(v, 8), "unit": "TB/s", "h2d_bytes_per_step": 0,
                    "d2h_bytes_per_step": 0}}
     print(json.dumps(out), flush=True)
