@@ -55,6 +55,7 @@ class Block(C.Structure):
                 ("n_grp", C.c_int32)]
 
     def as_dict(self):
+        """The block's fields as a dict."""
         return {f: getattr(self, f) for f, _ in self._fields_}
 
 
@@ -157,10 +158,12 @@ def _check(rc):
 
 
 def last_error():
+    """The calling thread's last error message from the library."""
     return _lib.polyq_last_error().decode()
 
 
 def f64_to_f16(v: float) -> int:
+    """The library's fp64 -> fp16 round-to-nearest-even, as raw bits (a test aid)."""
     return int(_lib.polyq_f64_to_f16(float(v)))
 
 
@@ -264,6 +267,7 @@ class HostLayer:
             self._h = C.c_void_p()
 
     def info(self) -> dict:
+        """Block table, realised budget, byte counts and Section 3.4 factors of the packed layer."""
         inf = Info()
         _check(_lib.polyq_layer_info(self._h, C.byref(inf)))
         d = {f: getattr(inf, f) for f, _ in Info._fields_ if f != "blocks"}
@@ -294,6 +298,7 @@ class HostLayer:
         return dict(info=inf, packed=packed, meta=meta, perm=perm, bits=bits, out_perm=out_perm)
 
     def permute_rows(self, row_perm):
+        """Reorder the output rows (Section 4.3 merge): row i becomes old row row_perm[i]."""
         rp = np.ascontiguousarray(row_perm, dtype=np.int32)
         _check(_lib.polyq_layer_permute_rows(self._h, rp.ctypes.data))
 
@@ -326,6 +331,7 @@ class DeviceLayer:
         self.K = self.info["K"]
 
     def packed_bytes(self):
+        """Device bytes of the packed codes and their scale/zero metadata."""
         return self.info["packed_bytes"] + self.info["meta_bytes"]
 
     def clone(self):
@@ -350,6 +356,7 @@ def _stream_ptr(stream):
 
 
 def gemv_workspace_bytes(layer: DeviceLayer, batch: int) -> int:
+    """Workspace bytes one GEMV call on `layer` at `batch` needs."""
     n = C.c_size_t()
     _check(_lib.polyq_gemv_workspace_bytes(C.byref(layer.desc), int(batch), C.byref(n)))
     return n.value
@@ -408,6 +415,7 @@ def _layer_array(layers):
 
 
 def gemv_group_workspace_bytes(layers, batch: int) -> int:
+    """Workspace bytes one grouped GEMV call on `layers` at `batch` needs."""
     n = C.c_size_t()
     _check(_lib.polyq_gemv_group_workspace_bytes(_layer_array(layers), len(layers), int(batch),
                                                  C.byref(n)))
@@ -476,6 +484,7 @@ def linear_gemv_input(layers, kind, a, b=None, eps=1e-6, ys=None, residuals=None
 
 
 def gemm_workspace_bytes(layer: DeviceLayer, M: int) -> int:
+    """Workspace bytes one GEMM call on `layer` with M tokens needs."""
     n = C.c_size_t()
     _check(_lib.polyq_gemm_workspace_bytes(C.byref(layer.desc), int(M), C.byref(n)))
     return n.value
@@ -607,6 +616,7 @@ class GemvChain:
         self.n_phases = len(phases)
 
     def run(self, stream=None, workspace=None):
+        """Launch every phase of the chain once on `stream` (one cooperative launch)."""
         ws = self.workspace if workspace is None else workspace
         _check(_lib.polyq_linear_gemv_chain(self._h, ws.data_ptr(), ws.numel(),
                                             _stream_ptr(stream)))
