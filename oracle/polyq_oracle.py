@@ -25,7 +25,7 @@ What is restated here (PolyQ, arXiv 2607.14618):
 * §5.3  the per-token reorder-traffic model (A16 read+write bytes of explicit
         activation shuffles).
 
-Readings taken where the paper is silent (the same list is in the design doc):
+Readings taken where the paper is silent:
 
 R1 quantiser: per (row n, block, 64-position group of the clustered order),
    lo=min w, hi=max w, qmax=2^b-1, s=fp16_rn((hi-lo)/qmax), if s==0 then
