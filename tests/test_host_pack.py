@@ -302,6 +302,26 @@ def test_scaled_pack_with_forced_widths_matches_oracle(polyq_lib):
     _compare_scaled(host, W, a, bits, _x2(a))
 
 
+def test_scaled_pack_finds_the_hand_worked_exponent(polyq_lib):
+    # The one-row 2-bit block of the Section 3.4 oracle pins: only alpha = 1/2
+    # puts every scaled weight on the 2-bit grid (worked by hand there), and
+    # then the packed layer reproduces W exactly.
+    m = np.array([4.0, 0.25, 0.25, 0.25, 0.25, 1.0], np.float32)
+    W = np.array([[3 / 16, 0.25, 0.5, 0.5, 0.25, 0.0]], np.float32)
+    host = polyq_lib.HostLayer.pack(W, m, 2.0, forced_bits=np.full(6, 2), act_scaling=True,
+                                    act_sqmean=np.ones(6, np.float32))
+    inf = host.info()
+    assert inf["alpha"][2] == 0.5
+    ex = host.export()
+    assert host.xscale().tolist() == [0.5, 2.0, 2.0, 2.0, 2.0, 1.0]  # perm is the identity
+    assert ex["perm"].tolist() == list(range(6))
+    ref = O.pack_layer_scaled(W, np.full(6, 2), np.array([0.5, 2, 2, 2, 2, 1.0]))
+    assert np.array_equal(ex["packed"], ref["packed"])
+    meta_ref = ref["meta"][:, :, 0].astype(np.uint32) | (ref["meta"][:, :, 1].astype(np.uint32) << 16)
+    assert np.array_equal(ex["meta"], meta_ref)
+    assert np.array_equal(O.dequant(ref) * ref["xscale"][None, :], W.astype(np.float64))
+
+
 def test_unscaled_layer_reports_no_factors(polyq_lib):
     W, a = synth.layer_weights(8, 300, 14)
     host = polyq_lib.HostLayer.pack(W, a, 3.0)

@@ -227,6 +227,65 @@ def test_scaled_layer_computes_x_times_dequantised_scaled_weights():
     assert np.allclose(O.linear_scaled(lay, x), ref, rtol=1e-12, atol=1e-12)
 
 
+def test_activation_factor_direction_on_hand_values():
+    # Section 3.4 defines s_j = m_j^alpha and Section 3.1 packs diag(s) W and
+    # multiplies the activation by 1/s.  The layer carries t = 1/s = m^-alpha:
+    # m = (4, 1/4) at alpha = 1/2 gives t = (1/2, 2), so the salient channel
+    # (m = 4) has its weights scaled up by 2 before quantisation.
+    t = O.act_factor(np.array([4.0, 0.25]), 0.5)
+    assert t.tolist() == [0.5, 2.0]
+    assert O.act_factor(np.array([4.0, 0.25]), 0.0).tolist() == [1.0, 1.0]
+    assert O.act_factor(np.array([16.0, 1.0]), 1.0).tolist() == [0.0625, 1.0]
+    # m_k = a_k / mean(a): hand values
+    assert O.act_metric(np.array([4.0, 0.25, 0.25, 0.25, 0.25, 1.0], np.float32)).tolist() == \
+        [4.0, 0.25, 0.25, 0.25, 0.25, 1.0]
+    assert O.act_metric(np.array([1.0, 3.0], np.float32)).tolist() == [0.5, 1.5]
+
+
+# A one-row 2-bit block of six channels, built so that its scaled weights
+# u_j = w_j * m_j^alpha land exactly on the 2-bit grid {0, 1, 2, 3}/8 at
+# alpha = 1/2 and at no other alpha (worked by hand):
+#   m = (4, 1/4, 1/4, 1/4, 1/4, 1), w = (3/16, 1/4, 1/2, 1/2, 1/4, 0).
+#   u = (3/16 * 4^a, 1/4 * 4^-a, 1/2 * 4^-a, 1/2 * 4^-a, 1/4 * 4^-a, 0).
+#   lo = 0, hi = max(u_0, u_2), scale = hi / 3.  Channels 1 and 2 have the
+#   ratio 1/2 at every alpha, so both sit on the grid only as hi/3 and 2hi/3,
+#   i.e. hi = 3 u_1 = (3/4) 4^-a; hi must also be u_0, so 4^(2a) = 4: a = 1/2.
+# At alpha = 1/2 the quantised layer reproduces w exactly; at every other
+# grid alpha some channel is off the grid and its error is positive.
+_E8_M = np.array([4.0, 0.25, 0.25, 0.25, 0.25, 1.0], np.float32)
+_E8_W = np.array([[3 / 16, 0.25, 0.5, 0.5, 0.25, 0.0]], np.float32)
+
+
+def test_alpha_search_finds_the_only_exact_exponent():
+    bits = np.full(6, 2)
+    x2 = np.ones(6)
+    alphas, t = O.choose_alphas(_E8_W, bits, _E8_M, x2)
+    assert alphas == {2: 0.5}
+    assert t.tolist() == [0.5, 2.0, 2.0, 2.0, 2.0, 1.0]  # original channel order
+    # the packed scaled layer reproduces W exactly (dequant(Q(W/t)) * t = W)
+    lay = O.pack_layer_scaled(_E8_W, bits, t)
+    assert np.array_equal(O.dequant(lay) * lay["xscale"][None, :],
+                          _E8_W.astype(np.float64)[:, lay["perm"]])
+    # hand check of the unscaled layer (alpha = 0): lo = 0, hi = 1/2, scale =
+    # fp16(1/6) = 1365/8192, zero 0; codes rint(w/scale) = (1, 2, 3, 3, 2, 0)
+    # (1/4 is 1.5004 steps), so in units of 1/8192 the errors are
+    # (171, 682, 1, 1, 682, 0) and the block mean is 959491 / (6 * 8192^2)
+    e0 = O.block_scaled_error(_E8_W.astype(np.float64), x2, np.ones(6), 2)
+    assert e0 == pytest.approx(959491.0 / (6 * 8192.0 ** 2), rel=1e-12)
+    assert O.block_scaled_error(_E8_W.astype(np.float64), x2, t, 2) == 0.0
+
+
+def test_alpha_search_would_fail_with_the_exponent_sign_flipped():
+    # With t = m^+alpha (the flipped reading) the exact point would need
+    # 4^(-2a) = 4, i.e. a = -1/2, which is off the grid: no grid alpha then
+    # reproduces W.  Evaluated through the block error with t built by hand.
+    x2 = np.ones(6)
+    for j in range(11):
+        a = j / 10
+        t_flip = (_E8_M.astype(np.float64) ** a).astype(np.float32).astype(np.float64)
+        assert O.block_scaled_error(_E8_W.astype(np.float64), x2, t_flip, 2) > 0.0
+
+
 def test_scaling_never_raises_the_block_error():
     W, a = synth.layer_weights(48, 512, 10)
     x2 = a.astype(np.float64) ** 2
