@@ -143,6 +143,18 @@ def max_over_ranks(ms, ws, device=None):
     return float(t.item())
 
 
+def window_max_over_ranks(win_ms, ws, device=None):
+    """Per window, the slowest rank's duration (all ranks time the same
+    number of windows)."""
+    if ws == 1:
+        return list(win_ms)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor(win_ms, dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return t.cpu().tolist()
+
+
 def job_tbs(ws, step_bytes, steps, ms):
     """Whole-job throughput: every replica streams ``step_bytes`` per step,
     over the slowest replica's time."""
@@ -265,21 +277,45 @@ def run_polyq(args):
         run_steps(args.warmup)
         run_steps(args.steps % args.copies)  # captures the remainder graph outside the timing
     torch.cuda.synchronize()
-    t0 = torch.cuda.Event(enable_timing=True)
-    t1 = torch.cuda.Event(enable_timing=True)
+    # The timed unit is a window of exactly `steps` steps between two events
+    # on the launching stream, synchronised on both sides.  A window of the
+    # default 20 steps lasts about a millisecond, far below the clock
+    # sampler's period, so the window is repeated back to back for about
+    # 1.5 s; the reported time is the median window (max over ranks).
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(2)]
+    with torch.cuda.stream(stream):
+        ev[0][0].record(stream)
+        run_steps(args.steps)
+        ev[0][1].record(stream)
+    torch.cuda.synchronize()
+    probe_ms = ev[0][0].elapsed_time(ev[0][1])
+    n_win = int(min(args.max_windows, max(1, np.ceil(args.timed_seconds * 1e3 / (probe_ms + 0.05)))))
     if ws > 1:
+        n_win = int(max_over_ranks(float(n_win), ws, device))
         dist.barrier()
     torch.cuda.synchronize()
+    win_ms = []
     with ClockSampler(local) as clk, torch.cuda.stream(stream):
-        t0.record(stream)
-        run_steps(args.steps)
-        t1.record(stream)
-        torch.cuda.synchronize()
+        for w in range(n_win):
+            t0, t1 = ev[w % 2]
+            t0.record(stream)
+            run_steps(args.steps)
+            t1.record(stream)
+            t1.synchronize()
+            win_ms.append(t0.elapsed_time(t1))
+    torch.cuda.synchronize()
     if ws > 1:
         dist.barrier()
-    ms = max_over_ranks(t0.elapsed_time(t1), ws, device)
+    win_ms = window_max_over_ranks(win_ms, ws, device)
+    ms = statistics.median(win_ms)
     ms_step = ms / args.steps
     value_tbs = job_tbs(ws, step_bytes, args.steps, ms)
+    timing = {"windows": n_win, "steps_per_window": args.steps,
+              "window_ms_median": round(ms, 5), "window_ms_min": round(min(win_ms), 5),
+              "window_ms_max": round(max(win_ms), 5), "first_window_ms": round(win_ms[0], 5),
+              "what": "each window: exactly `steps` steps between CUDA events on the launching "
+                      "stream, synchronised on both sides; value from the median window"}
 
     # Roofline of the dominant kernel.  The timed region holds only GEMV
     # launches (pre-pass + streaming kernel per linear), back to back, so its
@@ -426,6 +462,8 @@ def run_polyq(args):
 
     if rank == 0:
         cpu = None if (args.no_cpu_baseline or ws > 1) else cpu_baseline(args.cpu_seconds)
+        plan = plan_report(polyq)
+        quanta = quanta_report(polyq, synth)
         out = {
             "metric": METRIC, "value": round(value_tbs, 4), "unit": "TB/s", "n_gpus": ws,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_step, 5),
@@ -441,25 +479,58 @@ def run_polyq(args):
                        "b_real": {n: round(inf["b_real"], 5) for n, inf in infos},
                        "launch_groups": "q+k+v, o, gate+up, down (4 calls of 2 kernels)",
                        "graph": f"one CUDA graph of {args.copies} steps (one per layer "
-                                "copy), replayed"},
+                                "copy), replayed",
+                       "timing": f"median of {n_win} windows of {args.steps} steps"},
             "pct_of_peak": round(100 * value_tbs * 1e3 / (hbm * ws), 2),
             "roofline": roof,
             "cpu_baseline": cpu,
             "e2e": e2e,
             "gpu_launches": args.steps * len(GROUPS) * kernels_per_call,
             "clocks": clk.summary(),
-            "prefill_gemm": gemm,
-            "one_launch_step": one_launch,
-            "decode_step": decode,
-            "qwen3_32b_gemv": qwen,
+            "timing": timing,
+            # the long reports first, the measured paths after them and a
+            # compact summary last, where a tail of the output keeps them
+            "permutation_plan": plan,
+            "quanta_matching": quanta,
             "budget_sweep": sweep,
             "dense_bf16_context": dense,
-            "permutation_plan": plan_report(polyq),
-            "quanta_matching": quanta_report(polyq, synth),
+            "one_launch_step": one_launch,
+            "qwen3_32b_gemv": qwen,
+            "decode_step": decode,
+            "prefill_gemm": gemm,
         }
+        out["summary"] = summary(out)
         print(json.dumps(out), flush=True)
     if ws > 1:
         dist.destroy_process_group()
+
+
+def summary(out):
+    """The headline figures of every measured path, compact."""
+    sm = {"step_TBps": out["value"], "frac": out["roofline"]["frac"],
+          "e2e_TBps": (out.get("e2e") or {}).get("value"),
+          "one_launch_TBps": (out.get("one_launch_step") or {}).get("TB/s"),
+          "sm_mhz": out["clocks"].get("sm_mhz"), "reasons": out["clocks"].get("reasons")}
+    g = out.get("prefill_gemm")
+    if g:
+        sm["gemm_TFLOPs"] = {k: v["tflops"] for k, v in g.items() if isinstance(v, dict)
+                             and "tflops" in v}
+    d = out.get("decode_step")
+    if d:
+        sm["decode_40L_ms_per_token"] = {k: v.get("ms_per_token") for k, v in d.items()
+                                         if isinstance(v, dict) and "ms_per_token" in v}
+        ch = (d.get("grouped") or {}).get("chained")
+        if ch:
+            sm["decode_40L_chained_ms"] = ch.get("ms_per_token")
+    q = out.get("qwen3_32b_gemv")
+    if q:
+        sm["qwen3_32b_TBps"] = {k: v.get("TB/s") for k, v in q.items() if isinstance(v, dict)
+                                and "TB/s" in v}
+    bs = out.get("budget_sweep")
+    if bs:
+        sm["budget_sweep_TBps"] = {k: v.get("TB/s") for k, v in bs.items() if isinstance(v, dict)
+                                   and "TB/s" in v}
+    return sm
 
 
 def bench_decode_step(polyq, synth, torch, device, stream, args, hbm):
@@ -1010,6 +1081,9 @@ def main():
     ap.add_argument("--decode-steps", type=int, default=20)
     ap.add_argument("--no-sweep", action="store_true")
     ap.add_argument("--no-dense", action="store_true")
+    ap.add_argument("--timed-seconds", type=float, default=1.5,
+                    help="repeat the timed window of --steps steps for about this long")
+    ap.add_argument("--max-windows", type=int, default=2000)
     ap.add_argument("--cpu-baseline-child", action="store_true", help=argparse.SUPPRESS)
     args = ap.parse_args()
     if args.cpu_baseline_child:

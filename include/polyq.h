@@ -301,10 +301,15 @@ int polyq_gemv_workspace_bytes(const polyq_dev_layer* layer, int batch,
 
 /* Decode GEMV (Section 4.1 factorisation; Section 4.2 blocks in one launch):
  *   y[b][n] = residual[b][n] + sum_p x[b][gather[p]] * W'[n][p]
- * x: device bf16 [batch][K] (the activation in its producer's basis), every
- * value within the fp16 range (|x| <= 65504): the kernel multiplies fp16
- * copies of x (exact for values in the fp16 normal range) with the decoded
- * codes and accumulates in fp32.  batch in 1..4; y: device fp32 [batch][N];
+ * x: device bf16 [batch][K] (the activation in its producer's basis), any
+ * finite values.  The kernel multiplies fp16 copies of the gathered x with the
+ * decoded codes and accumulates in fp32.  Before the fp16 rounding each
+ * 64-channel group of a 2/3/4/8-bit block (each step of 128 channels of a
+ * 16-bit block) and batch row is scaled by the power of two that brings its
+ * largest |x| into [2^14, 2^15); its result is scaled back in fp32.  So the
+ * copies are exact whatever the activations' absolute scale, except for
+ * values more than about 2^20 below their group's largest, which lose low
+ * bits as fp16 subnormals (each by at most 2^-31 of that largest value).  batch in 1..4; y: device fp32 [batch][N];
  * residual: device fp32 [batch][N] or NULL (y may alias residual).  y is
  * first set to the residual (or zero), then each of the few pieces a row's
  * sum is split into is added with an fp32 atomic addition, so the last bits
@@ -320,7 +325,7 @@ int polyq_linear_gemv(const polyq_dev_layer* layer, const void* x, int batch,
 
 /* Scratch, in bytes, compiled into the library for polyq_linear_gemv_noalloc
  * (1 MiB).  A call needs 256 bytes plus one activation record per step of K
- * (1152 bytes per 512 channels at batch 1, 1344 bytes per 128 channels at
+ * (1184 bytes per 512 channels at batch 1, 1376 bytes per 128 channels at
  * batch 4), so every layer with K <= 65536 fits at any batch and any mix of
  * widths; N does not matter (see polyq_gemv_workspace_bytes). */
 #define POLYQ_NOALLOC_SCRATCH_BYTES (1u << 20)
@@ -339,16 +344,26 @@ int polyq_linear_gemv(const polyq_dev_layer* layer, const void* x, int batch,
  * call before any stream capture on that device.  Every call on a device uses
  * the same array, so calls whose kernels may overlap on the GPU (different
  * streams, or different host threads without ordering) race and corrupt each
- * other's results; serialise them, e.g. on one stream.  Each call clears the
- * scratch's status word (cudaMemsetAsync of 256 bytes on `stream`, no
- * allocation) before its kernels run, and the pre-pass writes every record
- * before the main kernel reads it, so nothing left by an earlier call leaks
- * into a later one.
+ * other's results; serialise them, e.g. on one stream.  The call's first
+ * kernel zeroes the scratch's status word once the previous kernel on the
+ * stream has finished, and writes every record before the second kernel reads
+ * it, so nothing left by an earlier call leaks into a later one.  A bounded
+ * device wait that gives up sets the status word and leaves y incomplete:
+ * read it with polyq_noalloc_status after the call and before the next
+ * no-allocation call on the same device.
  * Arguments and results are those of polyq_linear_gemv.  Returns
  * POLYQ_ENOMEM, touching nothing, when the layer and batch need more than
  * POLYQ_NOALLOC_SCRATCH_BYTES (see polyq_gemv_workspace_bytes). */
 int polyq_linear_gemv_noalloc(const polyq_dev_layer* layer, const void* x, int batch,
                               float* y, const float* residual, void* stream);
+
+/* Status word of the current device's no-allocation scratch after the work
+ * queued on `stream` (a 4-byte copy to the host and a wait for the stream; no
+ * allocation): the status of the last polyq_linear_gemv_noalloc call on this
+ * device, decoded as polyq_workspace_status does (POLYQ_ETIMEOUT when a
+ * bounded device wait gave up, with *status naming the wait).  The paper has
+ * no counterpart. */
+int polyq_noalloc_status(int* status, void* stream);
 
 /* Device scratch bytes polyq_linear_gemv_group needs for these layers
  * (same rules as polyq_gemv_workspace_bytes). */
@@ -491,11 +506,15 @@ int polyq_gemm_workspace_bytes(const polyq_dev_layer* layer, int64_t M,
 
 /* Prefill GEMM (the same product for M tokens, Section 5.4 prefill):
  *   Y[m][n] = sum_p X[m][gather[p]] * W'[n][p]
- * X: device bf16 [M][K]; Y: device fp32 [M][N]; workspace as for the GEMV.
- * Weights are dequantised to fp16 tiles in shared memory and multiplied on
- * the tcgen05 tensor cores with fp32 accumulation in tensor memory.  X is
- * gathered and converted to fp16 first, so |X| must stay within the fp16
- * range (65504); the product is then within fp16 rounding of each weight. */
+ * X: device bf16 [M][K], any finite values; Y: device fp32 [M][N], 16-byte
+ * aligned (else POLYQ_EINVAL); workspace as for the GEMV (its status word in
+ * its last 256 bytes).  Weights are dequantised to fp16 tiles in shared
+ * memory and multiplied on the tcgen05 tensor cores with fp32 accumulation in
+ * tensor memory.  X is gathered and converted to fp16 first, each row scaled
+ * by the power of two that brings its largest |x| into [2^14, 2^15) (scaled
+ * back in the epilogue), so the conversion is exact at any absolute scale
+ * except for values more than about 2^28 below their row's largest; the
+ * product is then within fp16 rounding of each weight. */
 int polyq_linear_gemm(const polyq_dev_layer* layer, const void* X, int64_t M,
                       float* Y, void* workspace, size_t workspace_bytes,
                       void* stream);

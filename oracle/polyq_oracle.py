@@ -392,16 +392,35 @@ def gather_index(layer, producer_basis=None):
     return permute_merge(producer_basis, perm)
 
 
+def dense_layer(W, bits):
+    """The clustered dequantised weights of a layer with width map ``bits``,
+    computed straight from W with the R1 quantiser, block by block, without
+    the bitstream (§4.1, §4.2): the same W' as ``dequant(pack_layer(W,
+    bits=bits))``, for layers too large to pack here in reasonable time.
+    Returns a layer dict with N, K, bits, perm, out_perm and Wd [N][K]."""
+    W = _check_weights(W)
+    N, K = W.shape
+    bits = np.asarray(bits, dtype=np.int64)
+    perm = cluster_perm(bits)
+    Wd = np.zeros((N, K), dtype=np.float64)
+    for blk in make_blocks(bits)[0]:
+        b, kb, p0 = blk["bits"], blk["n_ch"], blk["pos0"]
+        Wd[:, p0:p0 + kb] = dequant_rows(W[:, perm[p0:p0 + kb]].astype(np.float64), b)
+    return dict(N=N, K=K, bits=bits, perm=perm, out_perm=np.arange(N, dtype=np.int64), Wd=Wd)
+
+
 def linear(layer, x, gather=None):
     """y[b][n'] = sum_p x[b][r[p]] * W'[row(n')][p] in fp64 (§4.1, R6).
 
     ``x`` is [batch][K] (the activation in its producer's basis, values exact
     in fp64), ``gather`` is r (default: ``perm``, natural producer basis).
-    Rows come out in the layer's current output basis (``out_perm``)."""
+    Rows come out in the layer's current output basis (``out_perm``).  W'
+    comes from the packed bytes, or from ``Wd`` for a ``dense_layer``."""
     x = np.atleast_2d(np.asarray(x, dtype=np.float64))
     r = layer["perm"] if gather is None else np.asarray(gather)
     xs = x[:, r]
-    return xs @ dequant(layer).T
+    Wd = layer["Wd"] if "Wd" in layer else dequant(layer)
+    return xs @ Wd.T
 
 
 def linear_natural(layer, x):
@@ -440,8 +459,9 @@ def permute_rows(layer, row_perm):
     the producer's output channels)."""
     rp = _check_perm(row_perm, layer["N"])
     out = dict(layer)
-    out["packed"] = layer["packed"][rp].copy()
-    out["meta"] = layer["meta"][rp].copy()
+    for key in ("packed", "meta", "Wd"):
+        if key in layer:
+            out[key] = layer[key][rp].copy()
     out["out_perm"] = layer["out_perm"][rp].copy()
     return out
 
@@ -493,8 +513,9 @@ def row_slice(layer, r0, r1):
     """Rows [r0, r1) of a packed layer as a layer of their own (same channel
     permutation and blocks): a jointly allocated stack of linears, split."""
     out = dict(layer)
-    out["packed"] = layer["packed"][r0:r1].copy()
-    out["meta"] = layer["meta"][r0:r1].copy()
+    for key in ("packed", "meta", "Wd"):
+        if key in layer:
+            out[key] = layer[key][r0:r1].copy()
     out["out_perm"] = np.arange(r1 - r0, dtype=np.int64)
     out["N"] = r1 - r0
     return out

@@ -9,6 +9,10 @@
 //  1. gemm_prep gathers X through `gather` into a clustered fp16 matrix
 //     Xg[M][KT*32] (workspace), zero-padded at block ends, with the K order
 //     inside each tile permuted the same way the dequantiser emits codes.
+//     Each row m is scaled by the power of two 2^-e_m that brings its largest
+//     |x * t| into [2^14, 2^15), so that any finite bf16 row rounds to fp16
+//     without overflow and without dropping small values into subnormals;
+//     the epilogue multiplies row m of Y by 2^e_m.
 //  2. gemm_main: one persistent CTA per SM, 10 warps.
 //       warp 0      TMA producer: Xg tiles (64-byte swizzle), packed code
 //                   bytes and meta of 256 weight rows, or for 16-bit blocks the
@@ -83,6 +87,7 @@ struct GmParams {
   const int32_t* gather;
   const float* xscale;  // Section 3.4 activation factors (clustered order) or NULL
   __half* xg;
+  float* rowscale;      // [M]: 2^e_m, the power of two row m of Xg was divided by
   float* y;
   int* status;
 };
@@ -173,15 +178,33 @@ __host__ __device__ inline int slot_code(int bits, int s) {
 }
 
 // ---------------------------------------------------------------------------
-// pre-pass: Xg[m][kt*32 + s] = fp16(X[m][gather[p]] * xscale[p]) with
+// pre-pass: Xg[m][kt*32 + s] = fp16(X[m][gather[p]] * xscale[p] * 2^-e_m) with
 // p = pos0 + 32 h + slot_code(s)
-// for the h-th 32-code half group of the block (tile kt); Y is zeroed when the
-// K range is split over CTAs
+// for the h-th 32-code half group of the block (tile kt), one CTA per row at a
+// time; Y is zeroed when the K range is split over CTAs
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(256) gemm_prep(const __grid_constant__ GmParams P) {
+constexpr int kRowExp = 14;       // a row's largest magnitude becomes [2^14, 2^15)
+constexpr int kRowExpMin = -126;  // 2^e stays a normal float
+constexpr int kPrepThreads = 256;
+
+// The value that lands at clustered K slot k of row m (0 past a block's end).
+__device__ __forceinline__ float prep_value(const GmParams& P, const GmBlock* sblk, int m, int k) {
+  const int kt = k / BK, s = k % BK;
+  const GmBlock& B = sblk[find_kblock(sblk, P.n_blocks, kt)];
+  const int w = 32 * (kt - B.kt0) + slot_code(B.bits, s);
+  if (w >= B.n_ch) return 0.f;
+  const int p = B.pos0 + w;
+  const int src = P.gather ? P.gather[p] : p;
+  float xv = __bfloat162float(P.x[(size_t)m * P.K + src]);
+  if (P.xscale) xv *= P.xscale[p];
+  return xv;
+}
+
+__global__ void __launch_bounds__(kPrepThreads) gemm_prep(const __grid_constant__ GmParams P) {
   pdl_trigger();
   pdl_wait();
   __shared__ GmBlock sblk[POLYQ_MAX_BLOCKS];
+  __shared__ uint32_t s_wmax[kPrepThreads / 32];
   if (threadIdx.x < POLYQ_MAX_BLOCKS) {
     switch (threadIdx.x) {
       case 0: sblk[0] = P.blk[0]; break;
@@ -199,29 +222,45 @@ __global__ void __launch_bounds__(256) gemm_prep(const __grid_constant__ GmParam
          e += (long long)gridDim.x * blockDim.x)
       reinterpret_cast<float4*>(P.y)[e] = make_float4(0.f, 0.f, 0.f, 0.f);
   }
-  const int Kp = P.KT * BK;
-  const long long pairs = (long long)P.M * (Kp / 2);
-  for (long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x; e < pairs;
-       e += (long long)gridDim.x * blockDim.x) {
-    const int m = (int)(e / (Kp / 2));
-    const int k = 2 * (int)(e - (long long)m * (Kp / 2));
-    const int kt = k / BK, s = k % BK;
-    const GmBlock& B = sblk[find_kblock(sblk, P.n_blocks, kt)];
-    const int hg = kt - B.kt0;  // half group index inside the block
-    __half v[2];
+  const int half = P.KT * BK / 2;  // fp16 pairs per row of Xg
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int m = blockIdx.x; m < P.M; m += gridDim.x) {
+    // largest magnitude of the row's values (bit patterns of non-negative
+    // floats order as integers); without activation factors that is the
+    // largest |X[m][k]| over the raw row, since the gather is a permutation
+    uint32_t mx = 0;
+    if (!P.xscale) {
+      const uint16_t* row = reinterpret_cast<const uint16_t*>(P.x) + (size_t)m * P.K;
+      if ((P.K & 7) == 0 && (reinterpret_cast<uintptr_t>(row) & 15) == 0) {
+        for (int i = threadIdx.x; i < P.K / 8; i += kPrepThreads) {
+          const uint4 v = reinterpret_cast<const uint4*>(row)[i];
+          const uint32_t w[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      const int w = 32 * hg + slot_code(B.bits, s + h);
-      float xv = 0.f;
-      if (w < B.n_ch) {
-        const int p = B.pos0 + w;
-        const int src = P.gather ? P.gather[p] : p;
-        xv = __bfloat162float(P.x[(size_t)m * P.K + src]);
-        if (P.xscale) xv *= P.xscale[p];
+          for (int q = 0; q < 4; ++q)
+            mx = max(mx, max(w[q] & 0x7FFFu, (w[q] >> 16) & 0x7FFFu));
+        }
+      } else {
+        for (int i = threadIdx.x; i < P.K; i += kPrepThreads) mx = max(mx, row[i] & 0x7FFFu);
       }
-      v[h] = __float2half_rn(xv);
+      mx <<= 16;  // bf16 magnitude bits -> fp32 bits
+    } else {
+      for (int e = threadIdx.x; e < half; e += kPrepThreads)
+        mx = max(mx, max(__float_as_uint(fabsf(prep_value(P, sblk, m, 2 * e))),
+                         __float_as_uint(fabsf(prep_value(P, sblk, m, 2 * e + 1)))));
     }
-    reinterpret_cast<__half2*>(P.xg)[e] = __halves2half2(v[0], v[1]);
+    mx = __reduce_max_sync(0xffffffffu, mx);
+    if (lane == 0) s_wmax[warp] = mx;
+    __syncthreads();
+#pragma unroll
+    for (int w = 0; w < kPrepThreads / 32; ++w) mx = max(mx, s_wmax[w]);
+    // e_m = floor(log2(max)) - kRowExp (an fp32 subnormal maximum counts as 2^-127)
+    const int e = mx ? max((int)(mx >> 23) - 127 - kRowExp, kRowExpMin) : 0;
+    if (threadIdx.x == 0) P.rowscale[m] = ldexpf(1.f, e);
+    __half2* dst = reinterpret_cast<__half2*>(P.xg) + (size_t)m * half;
+    for (int i = threadIdx.x; i < half; i += kPrepThreads)
+      dst[i] = __halves2half2(__float2half_rn(ldexpf(prep_value(P, sblk, m, 2 * i), -e)),
+                              __float2half_rn(ldexpf(prep_value(P, sblk, m, 2 * i + 1), -e)));
+    __syncthreads();  // s_wmax is reused by the next row
   }
 }
 
@@ -516,12 +555,16 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
 #pragma unroll
       for (int t = 0; t < MT; ++t) {
         const int m = um * (MT * BM) + t * BM + 32 * q + lane;
+        const float rs = m < P.M ? P.rowscale[m] : 0.f;  // 2^e_m of the pre-pass
 #pragma unroll
         for (int c4 = 0; c4 < 4; ++c4) {
           const int col = 128 * half + 32 * c4;
           uint32_t v[32];
           tc_ld_32x32b_x32(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(t * BN + col), v);
           tc_wait_ld();
+          float f[32];
+#pragma unroll
+          for (int j = 0; j < 32; ++j) f[j] = __uint_as_float(v[j]) * rs;
           const int n0 = un * BN + col;
           if (m < P.M) {
             float* dst = P.y + (size_t)m * P.N + n0;
@@ -530,23 +573,21 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
               if (vec) {
 #pragma unroll
                 for (int j = 0; j < 8; ++j)
-                  red_add_v4(dst + 4 * j, __uint_as_float(v[4 * j]), __uint_as_float(v[4 * j + 1]),
-                             __uint_as_float(v[4 * j + 2]), __uint_as_float(v[4 * j + 3]));
+                  red_add_v4(dst + 4 * j, f[4 * j], f[4 * j + 1], f[4 * j + 2], f[4 * j + 3]);
               } else {
 #pragma unroll
                 for (int j = 0; j < 32; ++j)
-                  if (n0 + j < P.N) atomicAdd(dst + j, __uint_as_float(v[j]));
+                  if (n0 + j < P.N) atomicAdd(dst + j, f[j]);
               }
             } else if (vec) {
 #pragma unroll
               for (int j = 0; j < 8; ++j)
                 reinterpret_cast<float4*>(dst)[j] =
-                    make_float4(__uint_as_float(v[4 * j]), __uint_as_float(v[4 * j + 1]),
-                                __uint_as_float(v[4 * j + 2]), __uint_as_float(v[4 * j + 3]));
+                    make_float4(f[4 * j], f[4 * j + 1], f[4 * j + 2], f[4 * j + 3]);
             } else {
 #pragma unroll
               for (int j = 0; j < 32; ++j)
-                if (n0 + j < P.N) dst[j] = __uint_as_float(v[j]);
+                if (n0 + j < P.N) dst[j] = f[j];
             }
           }
         }
@@ -598,9 +639,13 @@ int k_tiles(const polyq_dev_layer* L, GmBlock* blk) {
   return kt;
 }
 
+// Workspace: Xg [M][KT*32] fp16, the row scales [M] fp32, then 256 bytes
+// holding the status word; each part starts on a 256-byte boundary.
+size_t gemm_xg_bytes(const polyq_dev_layer* L, int64_t M) {
+  return ((size_t)M * k_tiles(L, nullptr) * BK * 2 + 255) / 256 * 256;
+}
 size_t gemm_workspace(const polyq_dev_layer* L, int64_t M) {
-  const size_t xg = (size_t)M * k_tiles(L, nullptr) * BK * 2;
-  return (xg + 255) / 256 * 256 + 256;
+  return gemm_xg_bytes(L, M) + ((size_t)M * 4 + 255) / 256 * 256 + 256;
 }
 
 }  // namespace
@@ -622,6 +667,8 @@ extern "C" int polyq_linear_gemm(const polyq_dev_layer* L, const void* X, int64_
   int rc = polyq_check_dev_layer(L, "polyq_linear_gemm");
   if (rc) return rc;
   if (!X || !Y) return polyq_set_error(POLYQ_EINVAL, "polyq_linear_gemm: X or Y is NULL");
+  if ((uintptr_t)Y % 16)  // Y is written (and zeroed for split K) with 16-byte stores
+    return polyq_set_error(POLYQ_EINVAL, "polyq_linear_gemm: Y must be 16-byte aligned");
   if (M < 1 || M > (1 << 24))
     return polyq_set_error(POLYQ_EINVAL, "polyq_linear_gemm: M=%lld", (long long)M);
   const size_t need = gemm_workspace(L, M);
@@ -647,6 +694,7 @@ extern "C" int polyq_linear_gemm(const polyq_dev_layer* L, const void* X, int64_
   P.gather = L->gather;
   P.xscale = L->xscale;
   P.xg = (__half*)workspace;
+  P.rowscale = (float*)((uint8_t*)workspace + gemm_xg_bytes(L, M));
   P.y = Y;
   P.status = (int*)((uint8_t*)workspace + need - 256);
   rc = polyq_tensor_map_2d(&P.tm_x, P.xg, 2, (uint64_t)KT * BK, (uint64_t)M, (uint64_t)KT * BK * 2,
@@ -721,9 +769,8 @@ extern "C" int polyq_linear_gemm(const polyq_dev_layer* L, const void* X, int64_
   cfg.stream = st;
   cfg.attrs = at;
   cfg.numAttrs = 1;
-  const long long pairs = M * (long long)(KT * BK / 2);
-  cfg.gridDim = dim3((unsigned)std::min<long long>((pairs + 255) / 256, (long long)sms * 16));
-  cfg.blockDim = dim3(256);
+  cfg.gridDim = dim3((unsigned)std::min<long long>(M, (long long)sms * 16));
+  cfg.blockDim = dim3(kPrepThreads);
   cudaError_t e = cudaLaunchKernelEx(&cfg, gemm_prep, P);
   if (e != cudaSuccess)
     return polyq_set_error(POLYQ_ECUDA, "polyq_linear_gemm: prep launch: %s", cudaGetErrorString(e));

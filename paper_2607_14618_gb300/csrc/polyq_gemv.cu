@@ -83,6 +83,7 @@ struct GvParams {
   uint32_t magic;  // 0x64006400 (two fp16 1024.0), kept in a register
   // workspace
   int* status;     // sticky error word
+  int clear_status;  // 1: the pre-pass zeroes the status word first
   uint8_t* rec;    // [recs][rec_bytes(NB)] activation records
   // input transform shared by all layers (POLYQ_X_*); with POLYQ_X_BF16 each
   // layer reads its own L[l].x
@@ -247,6 +248,9 @@ __global__ void __launch_bounds__(kConsumers) gemv_prep(const __grid_constant__ 
   rec_sources<NB>(in, S.blk[l][bi], j, warp, lane, s_p3, src, fac);  // static layer data
   if (P.xkind == POLYQ_X_RMSNORM) rms_prefetch(P.xa, P.L[0].K, P.batch);
   pdl_wait();  // x comes from the previous kernel; the records and y may still be in use
+  // The streaming kernel writes the status only after its own wait for this
+  // grid, so clearing it here cannot lose one of its reports.
+  if (P.clear_status && blockIdx.x == 0 && threadIdx.x == 0) *P.status = 0;
   float ra[2][2], rb[2][2];
   rec_load<NB>(in, S.blk[l][bi], j, warp, lane, s_p3, src, ra, rb);
   __shared__ float s_rnorm[4];
@@ -600,7 +604,8 @@ int launch(const GvParams& P, int grid, cudaStream_t st) {
 
 int gemv_group(const char* who, const polyq_dev_layer* const* L, int n, const void* const* xs,
                int batch, float* const* ys, const float* const* res, void* workspace,
-               size_t ws_bytes, cudaStream_t st, const polyq_gemv_input* in = nullptr) {
+               size_t ws_bytes, cudaStream_t st, const polyq_gemv_input* in = nullptr,
+               bool clear_status = false) {
   int rc = check_group(who, L, n, batch);
   if (rc) return rc;
   const void* shared_x[POLYQ_MAX_GROUP];
@@ -672,6 +677,7 @@ int gemv_group(const char* who, const polyq_dev_layer* const* L, int n, const vo
   P.magic = kMagic;
   uint8_t* ws = (uint8_t*)workspace;
   P.status = (int*)ws;
+  P.clear_status = clear_status ? 1 : 0;
   P.rec = ws + w.rec_off;
   P.xkind = in ? in->kind : POLYQ_X_BF16;
   P.eps = in ? in->eps : 0.f;
@@ -808,16 +814,21 @@ extern "C" int polyq_linear_gemv_noalloc(const polyq_dev_layer* L, const void* x
   void* scratch = nullptr;
   rc = noalloc_scratch(&scratch);
   if (rc) return rc;
-  // The status word must start at zero.  A call that gave up on a wait
-  // leaves it set, and this caller cannot reset the library's array itself:
-  // clear it on every call.
-  cudaError_t e = cudaMemsetAsync(scratch, 0, 256, (cudaStream_t)stream);
-  if (e != cudaSuccess)
-    return polyq_set_error(POLYQ_ECUDA, "%s: clearing the scratch counters: %s", who,
-                           cudaGetErrorString(e));
   const void* xs[1] = {x};
   float* ys[1] = {y};
   const float* rs[1] = {residual};
+  // The status word must start at zero, and this caller cannot reset the
+  // library's array: the call's pre-pass clears it (after its wait for the
+  // previous kernel, so the previous call's status is readable until then).
   return gemv_group(who, one, 1, xs, batch, ys, rs, scratch, POLYQ_NOALLOC_SCRATCH_BYTES,
-                    (cudaStream_t)stream);
+                    (cudaStream_t)stream, nullptr, /*clear_status=*/true);
+}
+
+extern "C" int polyq_noalloc_status(int* status, void* stream) {
+  polyq_clear_error();
+  if (!status) return polyq_set_error(POLYQ_EINVAL, "polyq_noalloc_status: status is NULL");
+  void* scratch = nullptr;
+  int rc = noalloc_scratch(&scratch);
+  if (rc) return rc;
+  return polyq_workspace_status(scratch, status, stream);
 }

@@ -267,13 +267,36 @@ __device__ __forceinline__ void rec_store(const XIn& in, const GvBlock& B, int j
       xv[s][h] = v * fac[s][h];  // Section 3.4 factor (1 if none)
     }
   }
+  // Largest magnitude of each slot's values over the warp (the bit patterns of
+  // non-negative floats order as integers).  For b < 16 a slot's warp holds
+  // exactly one chunk; a 16-bit batch row spans warps w and w ^ 1, which
+  // exchange their maxima through shared memory (the width is uniform over
+  // the record, so every consumer thread takes the same branch).
+  uint32_t mx[2];
+#pragma unroll
+  for (int s = 0; s < 2; ++s)
+    mx[s] = __reduce_max_sync(0xffffffffu, max(__float_as_uint(fabsf(xv[s][0])),
+                                               __float_as_uint(fabsf(xv[s][1]))));
+  if (B.bits == 16) {
+    __shared__ uint32_t s_wmax[kWarps][2];
+    consumer_sync();  // an earlier record's readers are done with s_wmax
+    if (lane == 0) {
+      s_wmax[warp][0] = mx[0];
+      s_wmax[warp][1] = mx[1];
+    }
+    consumer_sync();
+    mx[0] = max(mx[0], s_wmax[warp ^ 1][0]);
+    mx[1] = max(mx[1], s_wmax[warp ^ 1][1]);
+  }
   float* recf = reinterpret_cast<float*>(rec);
 #pragma unroll
   for (int s = 0; s < 2; ++s) {
     const SlotGeom g = slot_geom<NB>(B.bits, warp, lane, threadIdx.x, s, j, p3);
-    if (!g.valid) continue;  // uniform over the warp for b < 16
-    const __half hlo = __float2half_rn(ldexpf(xv[s][0], -g.p[0]));
-    const __half hhi = __float2half_rn(ldexpf(xv[s][1], -g.p[1]));
+    if (!g.valid) continue;  // uniform over the warp
+    // e: floor(log2(max)) - kRecExp (an fp32 subnormal maximum counts as 2^-127)
+    const int e = mx[s] ? max((int)(mx[s] >> 23) - 127 - kRecExp, kRecExpMin) : 0;
+    const __half hlo = __float2half_rn(ldexpf(xv[s][0], -g.p[0] - e));
+    const __half hhi = __float2half_rn(ldexpf(xv[s][1], -g.p[1] - e));
     rec[(g.bb * 4 + g.t) * LW + g.jp] = pack_half2(hlo, hhi);
     if (B.bits != 16) {
       // X sums the values the MMA multiplies (fp16 times 2^p), so that the
@@ -289,7 +312,10 @@ __device__ __forceinline__ void rec_store(const XIn& in, const GvBlock& B, int j
       if (lane == 0) {
         recf[PW + g.bb * NGM + g.c] = kMagicF * s1;
         recf[PW + NB * NGM + g.bb * NGM + g.c] = s2;
+        recf[PW + 2 * NB * NGM + g.bb * NGM + g.c] = ldexpf(1.f, e);
       }
+    } else if (g.jp == 0 && g.t == 0) {
+      recf[PW + 2 * NB * NGM + g.bb * NGM] = ldexpf(1.f, e);
     }
   }
 }
@@ -468,12 +494,13 @@ __device__ __forceinline__ void step_mma(uint32_t magic, int batch, int uvalid, 
     if (be < batch) {
       const float C1 = recf[PW + be * NGM + c];
       const float X = recf[PW + NB * NGM + be * NGM + c];
+      const float E = recf[PW + 2 * NB * NGM + be * NGM + c];
 #pragma unroll
       for (int r = 0; r < 2; ++r) {
         const uint32_t m = meta_s[(r ? rB : rA) * kMetaBox + g0 + c];
         const float sc = __half2float(__ushort_as_half((uint16_t)(m & 0xFFFFu)));
         const float ze = __half2float(__ushort_as_half((uint16_t)(m >> 16)));
-        acc[r] += sc * fmaf(-ze, X, D[2 * r + cc] - C1);  // be is this lane's row
+        acc[r] += (sc * E) * fmaf(-ze, X, D[2 * r + cc] - C1);  // be is this lane's row
       }
     }
   }
@@ -551,12 +578,13 @@ __device__ __forceinline__ void step_mma_pair(uint32_t magic, int batch, int g0,
       if (be < batch) {
         const float C1 = recf[PW + be * NGM + c];
         const float X = recf[PW + NB * NGM + be * NGM + c];
+        const float E = recf[PW + 2 * NB * NGM + be * NGM + c];
 #pragma unroll
         for (int r = 0; r < 2; ++r) {
           const uint32_t m = meta_s[(r ? rB : rA) * kMetaBox + g0 + k * NGS + c];
           const float sc = __half2float(__ushort_as_half((uint16_t)(m & 0xFFFFu)));
           const float ze = __half2float(__ushort_as_half((uint16_t)(m >> 16)));
-          acc[r] += sc * fmaf(-ze, X, D[2 * r + cc] - C1);  // be is this lane's row
+          acc[r] += (sc * E) * fmaf(-ze, X, D[2 * r + cc] - C1);  // be is this lane's row
         }
       }
     }
@@ -600,20 +628,26 @@ __device__ __forceinline__ void step_16(int batch, int uvalid,
     }
   }
   // column c of D is batch row c: lane t holds rows 2t and 2t+1, and the
-  // first lane of each group takes its row's value from there
+  // first lane of each group takes its row's value from there, times the
+  // row's 2^e
+  constexpr int PW = rec_pair_words(NB);
+  constexpr int NGM = 8 / NB;
+  const float* Erow = reinterpret_cast<const float*>(rec) + PW + 2 * NB * NGM;
   if constexpr (NB == 1) {
     // row 0 is column 0, which lane 0 of the quad holds already
+    const float E = Erow[0];
 #pragma unroll
     for (int r = 0; r < 2; ++r)
-      if (t == 0) acc[r] += d[0][2 * r] + d[1][2 * r];
+      if (t == 0) acc[r] += E * (d[0][2 * r] + d[1][2 * r]);
   } else {
     const int bl = lane_batch<NB>(t);
     const int src = (lane & ~3) | (bl >> 1);
+    const float E = bl < batch ? Erow[bl * NGM] : 0.f;
 #pragma unroll
     for (int r = 0; r < 2; ++r) {
       const float v0 = __shfl_sync(0xffffffffu, d[0][2 * r] + d[1][2 * r], src);
       const float v1 = __shfl_sync(0xffffffffu, d[0][2 * r + 1] + d[1][2 * r + 1], src);
-      if (lane_first<NB>(t)) acc[r] += (bl & 1) ? v1 : v0;
+      if (lane_first<NB>(t)) acc[r] += E * ((bl & 1) ? v1 : v0);
     }
   }
 }

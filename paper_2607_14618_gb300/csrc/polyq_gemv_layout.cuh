@@ -29,7 +29,7 @@ constexpr int kPitchSplit = 144;   // row pitch of 128-byte boxes (16 extra byte
 constexpr int kMetaBox = 12;       // meta entries per row loaded per step
 constexpr int kCodesBytes = 2 * kRows * kPitchSplit;  // largest codes area (2 boxes)
 constexpr int kMetaBytes = kRows * kMetaBox * 4;
-constexpr int kRecOne = 1344;      // largest activation record (NB = 4)
+constexpr int kRecOne = 1376;      // largest activation record (NB = 4)
 constexpr int kRecMax = 2 * kRecOne;  // a stage may hold two steps' records
 // A stage holds an item's code boxes, its scale/zero box, its record(s) and
 // a 16-byte descriptor written by the producer.  At batch 2-4 a step whose
@@ -80,13 +80,23 @@ __host__ __device__ constexpr int lane_pairs(int bits, int nb) {
 }
 
 // Record: for each batch row b and lane t, LW words of fp16 pairs (the lane's
-// pairs in order, then 16 bytes of padding); then C1[b][8/NB] and X[b][8/NB]
-// (fp32): C1 = 1024 * sum x' and X = sum x over the chunk.
+// pairs in order, then 16 bytes of padding); then C1[b][8/NB], X[b][8/NB] and
+// E[b][8/NB] (fp32).  The record holds each activation as x * 2^-(e+p): e is
+// the chunk's exponent (kRecExp below), p the one its code carries.
+// C1 = 1024 * sum x' and X = sum x' * 2^p over the chunk, in those scaled
+// units, and E = 2^e multiplies the chunk's result back.  A 16-bit step has
+// one exponent per batch row, in E[b][0].
 __host__ __device__ constexpr int rec_lane_words(int nb) { return 64 / nb + 4; }
 __host__ __device__ constexpr int rec_pair_words(int nb) { return nb * 4 * rec_lane_words(nb); }
 __host__ __device__ constexpr int rec_bytes(int nb) {
-  return (rec_pair_words(nb) + 2 * nb * (8 / nb)) * 4;
+  return (rec_pair_words(nb) + 3 * nb * (8 / nb)) * 4;
 }
+// Each chunk is scaled by the power of two 2^-e that brings its largest
+// magnitude into [2^kRecExp, 2^(kRecExp+1)): every value then rounds to fp16
+// without overflow, and values down to 2^-(kRecExp+14-8) of the chunk's
+// largest stay fp16 normals even after the decoder's 2^-p (p <= 8).
+constexpr int kRecExp = 14;
+constexpr int kRecExpMin = -126;  // 2^e stays a normal float
 static_assert(rec_bytes(1) <= kRecOne && rec_bytes(2) <= kRecOne && rec_bytes(4) <= kRecOne, "");
 static_assert(rec_bytes(1) % 16 == 0 && rec_bytes(2) % 16 == 0 && rec_bytes(4) % 16 == 0, "");
 static_assert(lane_pairs(2, 1) + 4 <= rec_lane_words(1) && lane_pairs(2, 4) + 4 <= rec_lane_words(4), "");

@@ -117,6 +117,7 @@ _SIGS = {
     "polyq_gemv_workspace_bytes": (C.c_int, [C.POINTER(DevLayer), C.c_int, C.POINTER(C.c_size_t)]),
     "polyq_linear_gemv": (C.c_int, [C.POINTER(DevLayer), _P, C.c_int, _P, _P, _P, C.c_size_t, _P]),
     "polyq_linear_gemv_noalloc": (C.c_int, [C.POINTER(DevLayer), _P, C.c_int, _P, _P, _P]),
+    "polyq_noalloc_status": (C.c_int, [C.POINTER(C.c_int), _P]),
     "polyq_gemv_group_workspace_bytes": (C.c_int, [C.POINTER(C.POINTER(DevLayer)), C.c_int,
                                                    C.c_int, C.POINTER(C.c_size_t)]),
     "polyq_linear_gemv_group": (C.c_int, [C.POINTER(C.POINTER(DevLayer)), C.c_int,
@@ -349,6 +350,30 @@ class DeviceLayer:
         return c
 
 
+def _require(t, name, dtype, shape, device):
+    """ValueError unless `t` is a contiguous tensor of `dtype` and `shape` on
+    `device`: the library reads and writes through raw pointers, so a wrong
+    buffer would otherwise reach the GPU."""
+    import torch
+    if (not isinstance(t, torch.Tensor) or t.dtype != dtype or tuple(t.shape) != tuple(shape)
+            or t.device != device or not t.is_contiguous()):
+        raise ValueError(f"{name} must be a contiguous {dtype} tensor {list(shape)} on {device}")
+
+
+def _cuda_input(x, name, dtype, K):
+    """Checks a [rows][K] CUDA input of `dtype` and returns its device, which
+    must be the current device: the stream and the library's per-device state
+    are looked up for the current device."""
+    import torch
+    if (not isinstance(x, torch.Tensor) or x.dtype != dtype or not x.is_cuda or x.dim() != 2
+            or x.shape[1] != K):
+        raise ValueError(f"{name} must be a CUDA {dtype} tensor [rows][{K}]")
+    if x.device.index != torch.cuda.current_device():
+        raise ValueError(f"{name} is on {x.device}, not on the current device "
+                         f"cuda:{torch.cuda.current_device()}")
+    return x.device
+
+
 def _stream_ptr(stream):
     import torch
     s = torch.cuda.current_stream() if stream is None else stream
@@ -365,16 +390,20 @@ def gemv_workspace_bytes(layer: DeviceLayer, batch: int) -> int:
 def linear_gemv(layer: DeviceLayer, x, y=None, residual=None, workspace=None, stream=None):
     """y[b][n] = residual[b][n] + sum_p x[b][gather[p]] W'[n][p] (device tensors)."""
     import torch
-    if x.dtype != torch.bfloat16 or not x.is_cuda or x.dim() != 2 or x.shape[1] != layer.K:
-        raise ValueError("x must be a CUDA bf16 tensor [batch][K]")
+    dev = _cuda_input(x, "x", torch.bfloat16, layer.K)
     x = x.contiguous()
     batch = x.shape[0]
     if y is None:
-        y = torch.empty((batch, layer.N), dtype=torch.float32, device=x.device)
+        y = torch.empty((batch, layer.N), dtype=torch.float32, device=dev)
+    _require(y, "y", torch.float32, (batch, layer.N), dev)
+    if residual is not None:
+        _require(residual, "residual", torch.float32, (batch, layer.N), dev)
     ws_need = gemv_workspace_bytes(layer, batch)
     if workspace is None and ws_need:
-        # the tile counters in the workspace start at zero; calls keep them so
-        workspace = torch.zeros(ws_need, dtype=torch.uint8, device=x.device)
+        # the status word must start at zero; every call rewrites the records
+        workspace = torch.zeros(ws_need, dtype=torch.uint8, device=dev)
+    if workspace is not None:
+        _require(workspace, "workspace", torch.uint8, (workspace.numel(),), dev)
     ws_ptr = workspace.data_ptr() if workspace is not None else None
     ws_len = workspace.numel() if workspace is not None else 0
     _check(_lib.polyq_linear_gemv(C.byref(layer.desc), x.data_ptr(), batch, y.data_ptr(),
@@ -390,21 +419,31 @@ def linear_gemv_noalloc(layer: DeviceLayer, x, y, residual=None, stream=None):
 
     `y` must be passed: nothing is allocated here.  Calls that may overlap on
     the GPU share the scratch and race; the first call on a device looks up the
-    scratch address and should come before any stream capture there.
+    scratch address and should come before any stream capture there.  Read
+    noalloc_status() after a call to learn whether a bounded device wait gave
+    up.
     """
     import torch
-    if x.dtype != torch.bfloat16 or not x.is_cuda or x.dim() != 2 or x.shape[1] != layer.K:
-        raise ValueError("x must be a CUDA bf16 tensor [batch][K]")
+    dev = _cuda_input(x, "x", torch.bfloat16, layer.K)
     if not x.is_contiguous():
         raise ValueError("x must be contiguous (no copy is made here)")
     batch = x.shape[0]
-    if (y is None or y.dtype != torch.float32 or not y.is_contiguous()
-            or tuple(y.shape) != (batch, layer.N)):
-        raise ValueError("y must be a contiguous CUDA fp32 tensor [batch][N]")
+    _require(y, "y", torch.float32, (batch, layer.N), dev)
+    if residual is not None:
+        _require(residual, "residual", torch.float32, (batch, layer.N), dev)
     _check(_lib.polyq_linear_gemv_noalloc(C.byref(layer.desc), x.data_ptr(), batch, y.data_ptr(),
                                           residual.data_ptr() if residual is not None else None,
                                           _stream_ptr(stream)))
     return y
+
+
+def noalloc_status(stream=None):
+    """Status word of the current device's no-allocation scratch after the
+    queued work: 0 when the last linear_gemv_noalloc call's waits all
+    completed; raises PolyqError(POLYQ_ETIMEOUT) when one gave up."""
+    v = C.c_int()
+    _check(_lib.polyq_noalloc_status(C.byref(v), _stream_ptr(stream)))
+    return v.value
 
 
 def _layer_array(layers):
@@ -422,6 +461,16 @@ def gemv_group_workspace_bytes(layers, batch: int) -> int:
     return n.value
 
 
+def _check_outputs(layers, batch, ys, residuals, dev):
+    import torch
+    if len(ys) != len(layers) or (residuals is not None and len(residuals) != len(layers)):
+        raise ValueError("one y (and one residual, or None) per layer")
+    for i, l in enumerate(layers):
+        _require(ys[i], f"ys[{i}]", torch.float32, (batch, l.N), dev)
+        if residuals is not None and residuals[i] is not None:
+            _require(residuals[i], f"residuals[{i}]", torch.float32, (batch, l.N), dev)
+
+
 def linear_gemv_group(layers, xs, ys=None, residuals=None, workspace=None, stream=None):
     """Independent GEMVs in one launch: ys[i] = residuals[i] + xs[i] W_i'^T."""
     import torch
@@ -429,15 +478,20 @@ def linear_gemv_group(layers, xs, ys=None, residuals=None, workspace=None, strea
     if len(xs) != n:
         raise ValueError("one x per layer")
     batch = xs[0].shape[0]
+    dev = None
     for l, x in zip(layers, xs):
-        if x.dtype != torch.bfloat16 or not x.is_cuda or x.dim() != 2 or x.shape != (batch, l.K):
-            raise ValueError("each x must be a CUDA bf16 tensor [batch][K]")
+        d = _cuda_input(x, "each x", torch.bfloat16, l.K)
+        if x.shape[0] != batch or (dev is not None and d != dev):
+            raise ValueError("every x must have the same batch and device")
+        dev = d
     xs = [x.contiguous() for x in xs]
     if ys is None:
-        ys = [torch.empty((batch, l.N), dtype=torch.float32, device=xs[0].device) for l in layers]
+        ys = [torch.empty((batch, l.N), dtype=torch.float32, device=dev) for l in layers]
+    _check_outputs(layers, batch, ys, residuals, dev)
     need = gemv_group_workspace_bytes(layers, batch)
     if workspace is None:
-        workspace = torch.zeros(need, dtype=torch.uint8, device=xs[0].device)
+        workspace = torch.zeros(need, dtype=torch.uint8, device=dev)
+    _require(workspace, "workspace", torch.uint8, (workspace.numel(),), dev)
     xa = (C.c_void_p * n)(*[x.data_ptr() for x in xs])
     ya = (C.c_void_p * n)(*[y.data_ptr() for y in ys])
     ra = None
@@ -457,20 +511,23 @@ def linear_gemv_input(layers, kind, a, b=None, eps=1e-6, ys=None, residuals=None
     n = len(layers)
     K = layers[0].K
     want = torch.bfloat16 if kind == X_BF16 else torch.float32
-    if a.dtype != want or not a.is_cuda or a.dim() != 2 or a.shape[1] != K or not a.is_contiguous():
-        raise ValueError(f"a must be a contiguous CUDA {want} tensor [batch][K]")
+    dev = _cuda_input(a, "a", want, K)
+    if not a.is_contiguous():
+        raise ValueError("a must be contiguous")
     batch = a.shape[0]
     if (kind == X_SILU_MUL) != (b is not None):
         raise ValueError("b is the second input of X_SILU_MUL only")
-    if b is not None and (b.dtype != torch.float32 or b.shape != a.shape or not b.is_contiguous()):
-        raise ValueError("b must be a contiguous fp32 tensor shaped like a")
-    if x_out is not None and (x_out.dtype != torch.bfloat16 or x_out.shape != a.shape):
-        raise ValueError("x_out must be a bf16 tensor shaped like a")
+    if b is not None:
+        _require(b, "b", torch.float32, tuple(a.shape), dev)
+    if x_out is not None:
+        _require(x_out, "x_out", torch.bfloat16, tuple(a.shape), dev)
     if ys is None:
-        ys = [torch.empty((batch, l.N), dtype=torch.float32, device=a.device) for l in layers]
+        ys = [torch.empty((batch, l.N), dtype=torch.float32, device=dev) for l in layers]
+    _check_outputs(layers, batch, ys, residuals, dev)
     need = gemv_group_workspace_bytes(layers, batch)
     if workspace is None:
-        workspace = torch.zeros(need, dtype=torch.uint8, device=a.device)
+        workspace = torch.zeros(need, dtype=torch.uint8, device=dev)
+    _require(workspace, "workspace", torch.uint8, (workspace.numel(),), dev)
     inp = GemvInput(kind, eps, a.data_ptr(), b.data_ptr() if b is not None else None,
                     x_out.data_ptr() if x_out is not None else None)
     ya = (C.c_void_p * n)(*[y.data_ptr() for y in ys])
@@ -493,15 +550,17 @@ def gemm_workspace_bytes(layer: DeviceLayer, M: int) -> int:
 def linear_gemm(layer: DeviceLayer, X, Y=None, workspace=None, stream=None):
     """Y[m][n] = sum_p X[m][gather[p]] W'[n][p] (device tensors)."""
     import torch
-    if X.dtype != torch.bfloat16 or not X.is_cuda or X.dim() != 2 or X.shape[1] != layer.K:
-        raise ValueError("X must be a CUDA bf16 tensor [M][K]")
+    dev = _cuda_input(X, "X", torch.bfloat16, layer.K)
     X = X.contiguous()
     M = X.shape[0]
     if Y is None:
-        Y = torch.empty((M, layer.N), dtype=torch.float32, device=X.device)
+        Y = torch.empty((M, layer.N), dtype=torch.float32, device=dev)
+    _require(Y, "Y", torch.float32, (M, layer.N), dev)
     ws_need = gemm_workspace_bytes(layer, M)
     if workspace is None and ws_need:
-        workspace = torch.empty(ws_need, dtype=torch.uint8, device=X.device)
+        workspace = torch.empty(ws_need, dtype=torch.uint8, device=dev)
+    if workspace is not None:
+        _require(workspace, "workspace", torch.uint8, (workspace.numel(),), dev)
     ws_ptr = workspace.data_ptr() if workspace is not None else None
     ws_len = workspace.numel() if workspace is not None else 0
     _check(_lib.polyq_linear_gemm(C.byref(layer.desc), X.data_ptr(), M, Y.data_ptr(),

@@ -72,3 +72,35 @@ def test_gemm_full_size_sampled(polyq_lib, name, N, K, M):
     ref, _ = oracle_rows(W, a, 3.0, rows)
     yref = O.linear(ref, X[ms])
     check_tolerance(Y.cpu().numpy()[np.ix_(ms, rows)], yref, X[ms], K)
+
+
+@pytest.mark.parametrize("scale_exp", [-40, -12, -8, 4, 10, 40])
+def test_gemm_meets_tolerance_at_any_activation_scale(polyq_lib, scale_exp):
+    """Each row of X is scaled by a power of two before its fp16 conversion,
+    so the relative tolerance holds at any scale.  Rows here also differ from
+    each other by up to 2^6, and all five widths are present."""
+    M, N, K, seed = 300, 300, 1100, 59
+    W, a = synth.layer_weights(N, K, seed)
+    bits = synth.random_codes_layer_bits(K, seed)
+    _, X = synth.activations(a, M, seed)
+    f = 2.0 ** (scale_exp + (np.arange(M) % 7) - 3)
+    Xs = X * f[:, None]
+    Xb = synth.bf16_bits(Xs.astype(np.float32))
+    assert np.array_equal(synth.bf16_to_f64(Xb), Xs)
+    host = polyq_lib.HostLayer.pack(W, a, 3.0, forced_bits=bits)
+    dev = polyq_lib.DeviceLayer(host, "cuda")
+    ref = O.pack_layer(W, a, 3.0, bits=bits)
+    Y = polyq_lib.linear_gemm(dev, _x_dev(Xb))
+    torch.cuda.synchronize()
+    check_tolerance(Y.cpu().numpy(), O.linear(ref, Xs), Xs, K)
+
+
+def test_gemm_rejects_unaligned_output(polyq_lib):
+    W, a = synth.layer_weights(64, 256, 62)
+    host = polyq_lib.HostLayer.pack(W, a, 3.0)
+    dev = polyq_lib.DeviceLayer(host, "cuda")
+    Xb, _ = synth.activations(a, 4, 62)
+    Ybuf = torch.zeros(4 * 64 + 1, dtype=torch.float32, device="cuda")
+    with pytest.raises(polyq_lib.PolyqError) as ei:
+        polyq_lib.linear_gemm(dev, _x_dev(Xb), Y=Ybuf[1:].view(4, 64))
+    assert ei.value.code == polyq_lib.POLYQ_EINVAL

@@ -162,3 +162,40 @@ def test_gemv_group_of_seven_layers_with_own_inputs(polyq_lib, batch):
     torch.cuda.synchronize()
     for y, ref, x in zip(ys, refs, xs):
         check_tolerance(y.cpu().numpy(), O.linear(ref, x), x, x.shape[1])
+
+
+def _scaled_bf16(x, f):
+    """bf16 bits of x * f for a power of two f (exact for bf16 x in range)."""
+    xs = x * f
+    bits = synth.bf16_bits(xs.astype(np.float32))
+    assert np.array_equal(synth.bf16_to_f64(bits), xs)
+    return bits, xs
+
+
+@pytest.mark.parametrize("batch", [1, 4])
+@pytest.mark.parametrize("scale_exp", [-40, -12, -8, 4, 10, 40])
+def test_gemv_meets_tolerance_at_any_activation_scale(polyq_lib, batch, scale_exp):
+    """The tolerance is relative, so it must hold whatever the activations'
+    absolute scale: the record builder scales each chunk by a power of two
+    before rounding to fp16.  All five widths, ragged blocks."""
+    W, a, bits, xb, x = make_case(200, 3001, 3.0, 17, True, batch)
+    xsb, xs = _scaled_bf16(x, 2.0 ** scale_exp)
+    host, dev = _dev(polyq_lib, W, a, 3.0, bits)
+    ref = oracle_layer(W, a, 3.0, bits)
+    y = polyq_lib.linear_gemv(dev, _x_dev(xsb))
+    torch.cuda.synchronize()
+    check_tolerance(y.cpu().numpy(), O.linear(ref, xs), xs, 3001)
+
+
+@pytest.mark.parametrize("batch", [1, 3])
+def test_gemv_chunks_of_very_different_magnitude(polyq_lib, batch):
+    """Channels whose magnitudes differ by 2^24 inside one layer: each
+    64-channel chunk (and each 16-bit step) gets its own exponent."""
+    W, a, bits, xb, x = make_case(130, 2500, 3.0, 18, True, batch)
+    f = np.where(np.arange(2500) % 3 == 0, 2.0 ** 12, 2.0 ** -12)
+    xsb, xs = _scaled_bf16(x, f[None, :])
+    host, dev = _dev(polyq_lib, W, a, 3.0, bits)
+    ref = oracle_layer(W, a, 3.0, bits)
+    y = polyq_lib.linear_gemv(dev, _x_dev(xsb))
+    torch.cuda.synchronize()
+    check_tolerance(y.cpu().numpy(), O.linear(ref, xs), xs, 2500)

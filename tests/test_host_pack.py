@@ -399,3 +399,33 @@ def test_chain_overlap_rules_checked_before_any_device_work(polyq_lib):
     # first device query fails instead.
     rc = create(phase(x0, y0), phase(y0, x0, x0), phase(y0, y1))
     assert rc in (0, polyq_lib.POLYQ_ECUDA)
+
+
+def test_binding_rejects_wrong_buffers_before_the_library(polyq_lib):
+    """The binding checks every buffer it hands to the library as a raw
+    pointer: dtype, shape, device and contiguity (CPU tensors here; on a GPU
+    the same checks compare against the input's CUDA device)."""
+    import torch
+    cpu = torch.device("cpu")
+    ok = torch.zeros(2, 8)
+    polyq_lib._require(ok, "y", torch.float32, (2, 8), cpu)
+    bad = [torch.zeros(2, 8, dtype=torch.float16), torch.zeros(8, 2), torch.zeros(2, 9),
+           torch.zeros(8, 2).t(), torch.zeros(2, 16)[:, ::2], np.zeros((2, 8), np.float32)]
+    for t in bad:
+        with pytest.raises(ValueError):
+            polyq_lib._require(t, "y", torch.float32, (2, 8), cpu)
+    # inputs must be CUDA tensors of the right dtype and width
+    for x in (torch.zeros(1, 16, dtype=torch.bfloat16), torch.zeros(1, 16)):
+        with pytest.raises(ValueError):
+            polyq_lib._cuda_input(x, "x", torch.bfloat16, 16)
+
+
+def test_gemm_rejects_unaligned_output_on_the_host(polyq_lib):
+    W, a = synth.layer_weights(64, 256, 62)
+    host = polyq_lib.HostLayer.pack(W, a, 3.0)
+    d = _desc_from(polyq_lib, host)
+    L = polyq_lib._lib
+    rc = L.polyq_linear_gemm(C.byref(d), C.c_void_p(0x300000), 4, C.c_void_p(0x400004),
+                             C.c_void_p(0x500000), 1 << 24, None)
+    assert rc == polyq_lib.POLYQ_EINVAL
+    assert "16-byte" in polyq_lib.last_error()

@@ -503,3 +503,55 @@ def test_row_slice_of_stacked_layer():
     y = O.linear(Ls, x)
     assert np.array_equal(O.linear(O.row_slice(Ls, 0, 40), x), y[:, :40])
     assert np.array_equal(O.linear(O.row_slice(Ls, 40, 64), x), y[:, 40:])
+
+
+@pytest.mark.parametrize("N,K,seed", [(9, 333, 21), (3, 1, 22), (17, 700, 23)])
+def test_dense_layer_equals_the_packed_route(N, K, seed):
+    # the direct quantise-dequantise route and the bitstream round trip give
+    # the same W' bit for bit (all five widths, ragged blocks)
+    W, a = synth.layer_weights(N, K, seed)
+    bits = synth.random_codes_layer_bits(K, seed, widths=(2, 3, 4, 8, 16)[: min(5, K)])
+    L = O.pack_layer(W, a, 3.0, bits=bits)
+    D = O.dense_layer(W, bits)
+    assert np.array_equal(D["perm"], L["perm"])
+    assert np.array_equal(D["Wd"], O.dequant(L))
+    _, x = synth.activations(a, 2, seed)
+    assert np.array_equal(O.linear(D, x), O.linear(L, x))
+    rp = np.random.default_rng(seed).permutation(N)
+    assert np.array_equal(O.permute_rows(D, rp)["Wd"], O.dequant(O.permute_rows(L, rp)))
+    assert np.array_equal(O.row_slice(D, 1, N)["Wd"], O.dequant(O.row_slice(L, 1, N)))
+
+
+@pytest.mark.parametrize("seed", range(3))
+def test_dense_layer_brute_force_small(seed):
+    # K <= 16: one group per width, quantised straight from W in original
+    # channel order, then placed at each channel's clustered position
+    rng = np.random.default_rng(100 + seed)
+    K = int(rng.integers(2, 17))
+    N = int(rng.integers(1, 5))
+    W = rng.normal(0, 0.3, size=(N, K)).astype(np.float32)
+    bits = rng.choice([2, 3, 4, 8, 16], size=K)
+    D = O.dense_layer(W, bits)
+    pos = np.empty(K, np.int64)
+    pos[D["perm"]] = np.arange(K)
+    for n in range(N):
+        for b in set(bits.tolist()):
+            ks = [k for k in range(K) if bits[k] == b]
+            if b == 16:
+                want = [float(np.float16(W[n, k])) for k in ks]
+            else:
+                s, z, q = O.quantize_group(W[n, ks].astype(np.float64), b)
+                want = [(qi - z) * s for qi in q]
+            assert [D["Wd"][n, pos[k]] for k in ks] == want
+
+
+def test_decode_layer_on_dense_layers_equals_packed():
+    lin = _small_layer_set(64, 160, 330)
+    dense = {}
+    for i, (name, N, K) in enumerate(O.llama_layer_linears(64, 160)):
+        W, _ = synth.layer_weights(N, K, 330 + i)
+        dense[name] = O.dense_layer(W, lin[name]["bits"])
+    s = np.random.default_rng(4).standard_normal((1, 64))
+    s_p, _ = O.decode_layer(s, O.merge_decoder_layer(lin))
+    s_d, _ = O.decode_layer(s, O.merge_decoder_layer(dense))
+    assert np.array_equal(s_p, s_d)

@@ -61,6 +61,8 @@ def test_noalloc_matches_workspace_entry_on_two_calls(polyq_lib):
     torch.cuda.synchronize()
     _same(y1b, ref1)
     _same(y2b, ref2)
+    # no bounded wait gave up: the scratch's status word reads zero
+    assert polyq_lib.noalloc_status() == 0
 
 
 def _wide_layer(polyq_lib, K):
@@ -74,7 +76,7 @@ def _wide_layer(polyq_lib, K):
 
 def test_noalloc_rejects_layers_beyond_the_scratch(polyq_lib):
     # At batch 4 a step covers 128 channels, so K = 131072 has 1024 steps whose
-    # activation records (1344 bytes each) do not fit the fixed 1 MiB.
+    # activation records (1376 bytes each) do not fit the fixed 1 MiB.
     dev, a = _wide_layer(polyq_lib, 131072)
     assert polyq_lib.gemv_workspace_bytes(dev, 4) > polyq_lib.NOALLOC_SCRATCH_BYTES
     xb, _ = synth.activations(a, 4, 74)
