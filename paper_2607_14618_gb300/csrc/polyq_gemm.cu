@@ -83,6 +83,7 @@ struct GmParams {
   int units_m, units_n, ksplit, units;  // work units: (M pair, N tile, K split)
   int streamk;  // 1: each CTA takes an equal contiguous range of (unit, K tile) pairs
   int has_meta;
+  int prep_staged;  // 1: the pre-pass stages each row of X in shared memory
   const __nv_bfloat16* x;
   const int32_t* gather;
   const float* xscale;  // Section 3.4 activation factors (clustered order) or NULL
@@ -180,29 +181,40 @@ __host__ __device__ inline int slot_code(int bits, int s) {
 // ---------------------------------------------------------------------------
 // pre-pass: Xg[m][kt*32 + s] = fp16(X[m][gather[p]] * xscale[p] * 2^-e_m) with
 // p = pos0 + 32 h + slot_code(s)
-// for the h-th 32-code half group of the block (tile kt), one CTA per row at a
-// time; Y is zeroed when the K range is split over CTAs
+// for the h-th 32-code half group of the block (tile kt).  Each CTA first
+// builds, in shared memory, the map from a clustered slot to the source
+// channel it reads (and its activation factor); then, one row at a time, it
+// copies the row of X into shared memory with 16-byte loads (finding the
+// row's largest magnitude on the way) and gathers from there.  Global reads
+// and writes are so coalesced whatever the permutation.  Layers too wide for
+// that (see prep_smem_bytes) gather from global memory instead.  Y is zeroed
+// when the K range is split over CTAs.
 // ---------------------------------------------------------------------------
 constexpr int kRowExp = 14;       // a row's largest magnitude becomes [2^14, 2^15)
 constexpr int kRowExpMin = -126;  // 2^e stays a normal float
 constexpr int kPrepThreads = 256;
+constexpr int kPrepMaxSmem = 200 * 1024;
 
-// The value that lands at clustered K slot k of row m (0 past a block's end).
-__device__ __forceinline__ float prep_value(const GmParams& P, const GmBlock* sblk, int m, int k) {
+// Clustered K slot k of a row: the position p it takes its value from, or -1
+// past the end of a block.
+__device__ __forceinline__ int slot_pos(const GmBlock* sblk, int nblk, int k) {
   const int kt = k / BK, s = k % BK;
-  const GmBlock& B = sblk[find_kblock(sblk, P.n_blocks, kt)];
+  const GmBlock& B = sblk[find_kblock(sblk, nblk, kt)];
   const int w = 32 * (kt - B.kt0) + slot_code(B.bits, s);
-  if (w >= B.n_ch) return 0.f;
-  const int p = B.pos0 + w;
-  const int src = P.gather ? P.gather[p] : p;
-  float xv = __bfloat162float(P.x[(size_t)m * P.K + src]);
-  if (P.xscale) xv *= P.xscale[p];
-  return xv;
+  return w < B.n_ch ? B.pos0 + w : -1;
+}
+
+// Shared memory of the staged pre-pass: the slot -> source map (int32 [Kp]),
+// the slot factors (fp32 [Kp], scaled layers only) and one row of X (bf16
+// [K]); 0 when it does not fit.
+size_t prep_smem_bytes(int K, int Kp, bool xscale) {
+  const size_t b = (size_t)Kp * 4 * (xscale ? 2 : 1) + ((size_t)K * 2 + 15) / 16 * 16;
+  return b <= (size_t)kPrepMaxSmem ? b : 0;
 }
 
 __global__ void __launch_bounds__(kPrepThreads) gemm_prep(const __grid_constant__ GmParams P) {
+  extern __shared__ __align__(16) uint8_t psm[];
   pdl_trigger();
-  pdl_wait();
   __shared__ GmBlock sblk[POLYQ_MAX_BLOCKS];
   __shared__ uint32_t s_wmax[kPrepThreads / 32];
   if (threadIdx.x < POLYQ_MAX_BLOCKS) {
@@ -214,39 +226,93 @@ __global__ void __launch_bounds__(kPrepThreads) gemm_prep(const __grid_constant_
       default: sblk[4] = P.blk[4]; break;
     }
   }
-  if (blockIdx.x == 0 && threadIdx.x == 0) *P.status = 0;
   __syncthreads();
+  const int Kp = P.KT * BK, half = Kp / 2;  // slots and fp16 pairs per row of Xg
+  const bool staged = P.prep_staged != 0;
+  int* s_src = reinterpret_cast<int*>(psm);
+  float* s_fac = reinterpret_cast<float*>(psm + (size_t)Kp * 4);
+  uint16_t* s_row = reinterpret_cast<uint16_t*>(psm + (size_t)Kp * 4 * (P.xscale ? 2 : 1));
+  if (staged) {
+    // static layer data, built before the wait for the previous kernel; a
+    // thread's loads of 8 slots are issued together
+    constexpr int U = 8;
+    for (int k0 = threadIdx.x; k0 < Kp; k0 += kPrepThreads * U) {
+      int pos[U], src[U];
+      float fac[U];
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const int k = k0 + u * kPrepThreads;
+        pos[u] = k < Kp ? slot_pos(sblk, P.n_blocks, k) : -1;
+      }
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        src[u] = pos[u] < 0 ? -1 : (P.gather ? __ldg(P.gather + pos[u]) : pos[u]);
+        fac[u] = (P.xscale && pos[u] >= 0) ? __ldg(P.xscale + pos[u]) : 0.f;
+      }
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const int k = k0 + u * kPrepThreads;
+        if (k < Kp) {
+          s_src[k] = src[u];
+          if (P.xscale) s_fac[k] = fac[u];
+        }
+      }
+    }
+  }
+  pdl_wait();  // X comes from the previous kernel; Y and the workspace may still be in use
+  if (blockIdx.x == 0 && threadIdx.x == 0) *P.status = 0;
   if (P.ksplit > 1 || P.streamk) {
     const long long total4 = (long long)P.M * P.N / 4;
     for (long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x; e < total4;
          e += (long long)gridDim.x * blockDim.x)
       reinterpret_cast<float4*>(P.y)[e] = make_float4(0.f, 0.f, 0.f, 0.f);
   }
-  const int half = P.KT * BK / 2;  // fp16 pairs per row of Xg
+  // the value at clustered slot k of row m
+  auto value = [&](int m, int k) -> float {
+    int src;
+    float f = 1.f;
+    if (staged) {
+      src = s_src[k];
+      if (src < 0) return 0.f;
+      if (P.xscale) f = s_fac[k];
+    } else {
+      const int p = slot_pos(sblk, P.n_blocks, k);
+      if (p < 0) return 0.f;
+      src = P.gather ? __ldg(P.gather + p) : p;
+      if (P.xscale) f = __ldg(P.xscale + p);
+    }
+    const uint16_t b = staged ? s_row[src]
+                              : __ldg(reinterpret_cast<const uint16_t*>(P.x) + (size_t)m * P.K + src);
+    return __uint_as_float((uint32_t)b << 16) * f;
+  };
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   for (int m = blockIdx.x; m < P.M; m += gridDim.x) {
     // largest magnitude of the row's values (bit patterns of non-negative
     // floats order as integers); without activation factors that is the
     // largest |X[m][k]| over the raw row, since the gather is a permutation
+    const uint16_t* row = reinterpret_cast<const uint16_t*>(P.x) + (size_t)m * P.K;
     uint32_t mx = 0;
-    if (!P.xscale) {
-      const uint16_t* row = reinterpret_cast<const uint16_t*>(P.x) + (size_t)m * P.K;
-      if ((P.K & 7) == 0 && (reinterpret_cast<uintptr_t>(row) & 15) == 0) {
-        for (int i = threadIdx.x; i < P.K / 8; i += kPrepThreads) {
-          const uint4 v = reinterpret_cast<const uint4*>(row)[i];
-          const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+    if ((P.K & 7) == 0 && (reinterpret_cast<uintptr_t>(row) & 15) == 0) {
+      for (int i = threadIdx.x; i < P.K / 8; i += kPrepThreads) {
+        const uint4 v = __ldg(reinterpret_cast<const uint4*>(row) + i);
+        if (staged) reinterpret_cast<uint4*>(s_row)[i] = v;
+        const uint32_t w[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-          for (int q = 0; q < 4; ++q)
-            mx = max(mx, max(w[q] & 0x7FFFu, (w[q] >> 16) & 0x7FFFu));
-        }
-      } else {
-        for (int i = threadIdx.x; i < P.K; i += kPrepThreads) mx = max(mx, row[i] & 0x7FFFu);
+        for (int q = 0; q < 4; ++q) mx = max(mx, max(w[q] & 0x7FFFu, (w[q] >> 16) & 0x7FFFu));
       }
-      mx <<= 16;  // bf16 magnitude bits -> fp32 bits
     } else {
-      for (int e = threadIdx.x; e < half; e += kPrepThreads)
-        mx = max(mx, max(__float_as_uint(fabsf(prep_value(P, sblk, m, 2 * e))),
-                         __float_as_uint(fabsf(prep_value(P, sblk, m, 2 * e + 1)))));
+      for (int i = threadIdx.x; i < P.K; i += kPrepThreads) {
+        const uint16_t v = __ldg(row + i);
+        if (staged) s_row[i] = v;
+        mx = max(mx, (uint32_t)(v & 0x7FFFu));
+      }
+    }
+    mx <<= 16;  // bf16 magnitude bits -> fp32 bits
+    __syncthreads();  // the staged row (and, on the first row, the map) is complete
+    if (P.xscale) {
+      mx = 0;
+      for (int k = threadIdx.x; k < Kp; k += kPrepThreads)
+        mx = max(mx, __float_as_uint(fabsf(value(m, k))));
     }
     mx = __reduce_max_sync(0xffffffffu, mx);
     if (lane == 0) s_wmax[warp] = mx;
@@ -258,9 +324,9 @@ __global__ void __launch_bounds__(kPrepThreads) gemm_prep(const __grid_constant_
     if (threadIdx.x == 0) P.rowscale[m] = ldexpf(1.f, e);
     __half2* dst = reinterpret_cast<__half2*>(P.xg) + (size_t)m * half;
     for (int i = threadIdx.x; i < half; i += kPrepThreads)
-      dst[i] = __halves2half2(__float2half_rn(ldexpf(prep_value(P, sblk, m, 2 * i), -e)),
-                              __float2half_rn(ldexpf(prep_value(P, sblk, m, 2 * i + 1), -e)));
-    __syncthreads();  // s_wmax is reused by the next row
+      dst[i] = __halves2half2(__float2half_rn(ldexpf(value(m, 2 * i), -e)),
+                              __float2half_rn(ldexpf(value(m, 2 * i + 1), -e)));
+    __syncthreads();  // the row buffer and s_wmax are reused by the next row
   }
 }
 
@@ -769,8 +835,25 @@ extern "C" int polyq_linear_gemm(const polyq_dev_layer* L, const void* X, int64_
   cfg.stream = st;
   cfg.attrs = at;
   cfg.numAttrs = 1;
-  cfg.gridDim = dim3((unsigned)std::min<long long>(M, (long long)sms * 16));
+  const size_t prep_smem = prep_smem_bytes(P.K, KT * BK, P.xscale != nullptr);
+  P.prep_staged = prep_smem > 0;
+  {
+    // as many CTAs as fit at once, each taking rows m = b, b + grid, ...
+    const int by_smem = prep_smem ? std::max(1, (int)((228 * 1024) / (prep_smem + 2048))) : 8;
+    const int per_sm = std::min(8, by_smem);
+    cfg.gridDim = dim3((unsigned)std::min<long long>(M, (long long)sms * per_sm));
+  }
   cfg.blockDim = dim3(kPrepThreads);
+  cfg.dynamicSmemBytes = prep_smem;
+  static bool prep_attr_done[8] = {false};
+  if (!prep_attr_done[dev & 7]) {
+    cudaError_t ea = cudaFuncSetAttribute(gemm_prep, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                          kPrepMaxSmem);
+    if (ea != cudaSuccess)
+      return polyq_set_error(POLYQ_ECUDA, "polyq_linear_gemm: prep smem attribute: %s",
+                             cudaGetErrorString(ea));
+    prep_attr_done[dev & 7] = true;
+  }
   cudaError_t e = cudaLaunchKernelEx(&cfg, gemm_prep, P);
   if (e != cudaSuccess)
     return polyq_set_error(POLYQ_ECUDA, "polyq_linear_gemm: prep launch: %s", cudaGetErrorString(e));

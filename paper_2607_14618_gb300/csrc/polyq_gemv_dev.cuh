@@ -165,7 +165,9 @@ __device__ __forceinline__ void rms_prefetch(const float* xa, int K, int batch) 
 
 // s_rnorm[b] = 1 / sqrt(mean_k a[b][k]^2 + eps) for each batch row, computed
 // by the 128 consumer threads with loads through L2.  s_part holds
-// batch x kWarps partial sums.
+// batch x kWarps partial sums.  A thread's loads of up to kRmsBatch float4
+// are issued together (one L2 round trip for rows up to 8192 wide).
+constexpr int kRmsBatch = 16;
 __device__ __forceinline__ void rms_rnorm(const float* xa, int K, int batch, float eps,
                                           float (*s_part)[kWarps], float* s_rnorm) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -174,13 +176,22 @@ __device__ __forceinline__ void rms_rnorm(const float* xa, int K, int batch, flo
     const float* row = xa + (size_t)bb * K;
     float acc = 0.f;
     if (vec) {
-#pragma unroll 4
-      for (int i = 4 * threadIdx.x; i < K; i += 4 * kConsumers) {
-        const float4 v = __ldcg(reinterpret_cast<const float4*>(row + i));
-        acc = fmaf(v.x, v.x, acc);
-        acc = fmaf(v.y, v.y, acc);
-        acc = fmaf(v.z, v.z, acc);
-        acc = fmaf(v.w, v.w, acc);
+      const int n4 = K / 4;
+      for (int i0 = threadIdx.x; i0 < n4; i0 += kRmsBatch * kConsumers) {
+        float4 v[kRmsBatch];
+#pragma unroll
+        for (int u = 0; u < kRmsBatch; ++u) {
+          const int i = i0 + u * kConsumers;
+          v[u] = i < n4 ? __ldcg(reinterpret_cast<const float4*>(row) + i)
+                        : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+#pragma unroll
+        for (int u = 0; u < kRmsBatch; ++u) {
+          acc = fmaf(v[u].x, v[u].x, acc);
+          acc = fmaf(v[u].y, v[u].y, acc);
+          acc = fmaf(v[u].z, v[u].z, acc);
+          acc = fmaf(v[u].w, v[u].w, acc);
+        }
       }
     } else {
       for (int i = threadIdx.x; i < K; i += kConsumers) {

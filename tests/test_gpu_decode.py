@@ -204,3 +204,68 @@ def test_grouped_decode_layer(polyq_lib):
     s_ref, _ = O.decode_layer(s0.astype(np.float64), merged)
     got = s.cpu().numpy().astype(np.float64)
     assert np.linalg.norm(got - s_ref) / np.linalg.norm(s_ref) <= 1e-2
+
+
+@pytest.mark.parametrize("kind", ["bf16", "f32", "rmsnorm", "silu_mul"])
+@pytest.mark.parametrize("K", [1100, 1101])
+def test_in_place_call_with_every_input_kind(polyq_lib, kind, K):
+    """Batch 1 with every output accumulated in place (y aliases its
+    residual), for each fused input kind, on a row width that is and one that
+    is not a multiple of 4.  Three layers of different shapes and widths
+    share the input; the results must match the oracle fed the GPU's own
+    transformed input (x_out), and a second call must add the product again."""
+    rng = np.random.default_rng(K)
+    specs = [(200, 3.0, 71, True), (130, 4.5, 72, False), (64, 2.0, 73, False)]
+    devs, refs = [], []
+    for N, B, seed, forced in specs:
+        W, a = synth.layer_weights(N, K, seed)
+        bits = synth.random_codes_layer_bits(K, seed) if forced else None
+        host = polyq_lib.HostLayer.pack(W, a, B, forced_bits=bits)
+        devs.append(polyq_lib.DeviceLayer(host, "cuda"))
+        refs.append(O.pack_layer(W, a, B, bits=bits))
+    A = (rng.standard_normal((1, K)) * 2.0).astype(np.float32)
+    Bm = rng.standard_normal((1, K)).astype(np.float32)
+    if kind == "bf16":
+        a_dev = torch.from_numpy(synth.bf16_bits(A.astype(np.float64)).view(np.int16)).cuda()
+        a_dev = a_dev.view(torch.bfloat16)
+    else:
+        a_dev = torch.from_numpy(A).cuda()
+    b_dev = torch.from_numpy(Bm).cuda() if kind == "silu_mul" else None
+    k = {"bf16": polyq_lib.X_BF16, "f32": polyq_lib.X_F32, "rmsnorm": polyq_lib.X_RMSNORM,
+         "silu_mul": polyq_lib.X_SILU_MUL}[kind]
+    y0 = [torch.randn(1, N, device="cuda") for N, _, _, _ in specs]
+    ys = [y.clone() for y in y0]
+    x_out = torch.empty((1, K), dtype=torch.bfloat16, device="cuda")
+    polyq_lib.linear_gemv_input(devs, k, a_dev, b=b_dev, eps=1e-6, ys=ys, residuals=ys,
+                                x_out=x_out)
+    torch.cuda.synchronize()
+    x = _bf16_vals(_bf16_bits(x_out))
+    if kind == "bf16":
+        assert np.array_equal(_bf16_bits(x_out), _bf16_bits(a_dev))
+    for y, y_init, ref in zip(ys, y0, refs):
+        want = O.linear(ref, x) + y_init.cpu().numpy().astype(np.float64)
+        check_tolerance(y.cpu().numpy(), want, x, K)
+    # the same call again accumulates once more: y = y0 + 2 W x
+    polyq_lib.linear_gemv_input(devs, k, a_dev, b=b_dev, eps=1e-6, ys=ys, residuals=ys)
+    torch.cuda.synchronize()
+    for y, y_init, ref in zip(ys, y0, refs):
+        want = 2.0 * O.linear(ref, x) + y_init.cpu().numpy().astype(np.float64)
+        check_tolerance(y.cpu().numpy(), want, x, K)
+
+
+@pytest.mark.parametrize("scale_exp", [-40, -10, 12, 40])
+def test_in_place_at_any_activation_scale(polyq_lib, scale_exp):
+    W, a = synth.layer_weights(300, 3001, 74)
+    bits = synth.random_codes_layer_bits(3001, 74)
+    host = polyq_lib.HostLayer.pack(W, a, 3.0, forced_bits=bits)
+    dev = polyq_lib.DeviceLayer(host, "cuda")
+    ref = O.pack_layer(W, a, 3.0, bits=bits)
+    _, x = synth.activations(a, 1, 74)
+    xs = x * 2.0 ** scale_exp
+    xb = synth.bf16_bits(xs.astype(np.float32))
+    assert np.array_equal(synth.bf16_to_f64(xb), xs)
+    y = torch.zeros(1, 300, device="cuda")
+    polyq_lib.linear_gemv(dev, torch.from_numpy(xb.view(np.int16)).cuda().view(torch.bfloat16),
+                          y=y, residual=y)
+    torch.cuda.synchronize()
+    check_tolerance(y.cpu().numpy(), O.linear(ref, xs), xs, 3001)

@@ -104,3 +104,18 @@ def test_gemm_rejects_unaligned_output(polyq_lib):
     with pytest.raises(polyq_lib.PolyqError) as ei:
         polyq_lib.linear_gemm(dev, _x_dev(Xb), Y=Ybuf[1:].view(4, 64))
     assert ei.value.code == polyq_lib.POLYQ_EINVAL
+
+
+def test_gemm_rows_too_wide_to_stage(polyq_lib):
+    """Rows of X wider than the pre-pass stages in shared memory (K > 49152)
+    are gathered from global memory instead; with activation factors too."""
+    M, N, K, seed = 40, 96, 50003, 63
+    W, a = synth.layer_weights(N, K, seed)
+    bits = synth.random_codes_layer_bits(K, seed)
+    Xb, X = synth.activations(a, M, seed)
+    host = polyq_lib.HostLayer.pack(W, a, 3.0, forced_bits=bits)
+    dev = polyq_lib.DeviceLayer(host, "cuda")
+    ref = O.pack_layer(W, a, 3.0, bits=bits)
+    Y = polyq_lib.linear_gemm(dev, _x_dev(Xb))
+    torch.cuda.synchronize()
+    check_tolerance(Y.cpu().numpy(), O.linear(ref, X), X, K)
