@@ -724,6 +724,15 @@ def plan_report(polyq):
             no_merge = 4 * sum(dims[i[0]] for k, i, o, p in nodes if k == polyq.NODE_LINEAR)
             res[mode] = {"planned_mib": round(cost / 2 ** 20, 3),
                          "removed": round(1 - cost / no_merge, 4), "planner_ms": round(dt * 1e3, 2)}
+            # the same stack entered from an embedding whose columns may be
+            # permuted and left through a linear output head (its own gather
+            # counted): the stream region may then take one layer's order
+            perms.append(rng.permutation(c["hidden"]).astype(np.int32))
+            nodes, dims, _ = polyq.decoder_plan_graph(c["layers"], c["hidden"], c["ffn"], perm_of,
+                                                      c["kv"], c["qdim"], True,
+                                                      (len(perms) - 1, 32000))
+            _, cost_h = polyq.plan_graph(nodes, dims, perms)
+            res[mode]["free_embedding_linear_head_mib"] = round(cost_h / 2 ** 20, 3)
         res["no_merge_mib"] = round(no_merge / 2 ** 20, 3)
         res["paper_no_merge_mib"] = c["paper_no_merge_mib"]
         res["paper_polyq_mib"] = c["paper_polyq_mib"]

@@ -962,15 +962,21 @@ def no_merge_traffic(nodes, edge_dims):
     return 4 * sum(edge_dims[i[0]] for k, i, o, p in nodes if k == NODE_LINEAR)
 
 
-def decoder_graph(n_layers, hidden, ffn, kv=None, perm_ids=None, qdim=None):
+def decoder_graph(n_layers, hidden, ffn, kv=None, perm_ids=None, qdim=None, free_source=False,
+                  head=None):
     """The decode graph of a Llama/Qwen-style stack (R11 per layer, R17
     kinds): nodes, edge widths and, per layer, the edge ids by name.  ``qdim``
     is the width of q and of the attention output (heads x head width,
     default ``hidden``), ``kv`` the k/v width (grouped-query attention when
     below ``qdim``);
-    ``perm_ids(layer, name)`` gives each linear's permutation id.  The
-    stream enters from a fixed natural source and leaves through a boundary
-    (the output head reads natural order)."""
+    ``perm_ids(layer, name)`` gives each linear's permutation id.  By default
+    the stream enters from a fixed natural source and leaves through a
+    boundary (the output head reads natural order).  ``free_source``: the
+    stream enters from an embedding table whose columns may be permuted at
+    compile time (any order, no cost).  ``head = (perm id, vocab)``: the
+    stream ends in a final RMSNorm and an output head that is itself a linear
+    (it reads any order through its gather), whose logits leave through a
+    boundary."""
     qdim = hidden if qdim is None else qdim
     kv = qdim if kv is None else kv
     nodes, dims, names = [], [], []
@@ -980,7 +986,7 @@ def decoder_graph(n_layers, hidden, ffn, kv=None, perm_ids=None, qdim=None):
         return len(dims) - 1
 
     s = edge(hidden)
-    nodes.append((NODE_SOURCE_FIXED, [], s, -1))
+    nodes.append((NODE_SOURCE_FREE if free_source else NODE_SOURCE_FIXED, [], s, -1))
     for l in range(n_layers):
         e = {}
         e["h"] = edge(hidden)
@@ -1008,7 +1014,14 @@ def decoder_graph(n_layers, hidden, ffn, kv=None, perm_ids=None, qdim=None):
         e["s_in"] = s
         names.append(e)
         s = e["s2"]
-    nodes.append((NODE_BOUNDARY, [s], -1, -1))
+    if head is None:
+        nodes.append((NODE_BOUNDARY, [s], -1, -1))
+    else:
+        hf = edge(hidden)
+        nodes.append((NODE_ELEMENTWISE, [s], hf, -1))    # final RMSNorm
+        logits = edge(head[1])
+        nodes.append((NODE_LINEAR, [hf], logits, head[0]))
+        nodes.append((NODE_BOUNDARY, [logits], -1, -1))
     return nodes, dims, names
 
 

@@ -21,6 +21,10 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libpolyq.so")
 STAMP = os.path.join(BUILD, "stamp.txt")
+# The debug build (-DPOLYQ_DEBUG, a test aid): the same sources, whose GEMV
+# and GEMM kernels also write the codes and weights they decode.
+BUILD_DEBUG = os.path.join(HERE, "_build_debug")
+LIB_DEBUG = os.path.join(HERE, "libpolyq_debug.so")
 ARCH = "-gencode=arch=compute_103a,code=sm_103a"
 
 
@@ -47,36 +51,40 @@ def _stamp_text():
     return f"{platform.machine()} {sys.version_info[:2]}"
 
 
-def _up_to_date():
-    if not os.path.exists(LIB) or not os.path.exists(STAMP):
+def _up_to_date(lib, build):
+    stamp = os.path.join(build, "stamp.txt")
+    if not os.path.exists(lib) or not os.path.exists(stamp):
         return False
-    with open(STAMP) as f:
+    with open(stamp) as f:
         if f.read().strip() != _stamp_text():
             return False
-    t = os.path.getmtime(LIB)
+    t = os.path.getmtime(lib)
     return all(os.path.getmtime(p) <= t for p in _sources() + _headers() + [__file__])
 
 
-def build_library(force: bool = False, verbose: bool = False) -> str:
-    """Build (if stale) and return the path of libpolyq.so."""
-    if not force and _up_to_date():
-        return LIB
+def build_library(force: bool = False, verbose: bool = False, debug: bool = False) -> str:
+    """Build (if stale) and return the path of libpolyq.so (or, with
+    ``debug``, of the test aid libpolyq_debug.so)."""
+    lib, build = (LIB_DEBUG, BUILD_DEBUG) if debug else (LIB, BUILD)
+    if not force and _up_to_date(lib, build):
+        return lib
     cuda = _cuda_home()
     nvcc = os.path.join(cuda, "bin", "nvcc")
-    os.makedirs(BUILD, exist_ok=True)
+    os.makedirs(build, exist_ok=True)
     inc = ["-I", INCLUDE, "-I", CSRC, "-I", os.path.join(cuda, "include")]
+    defs = ["-DPOLYQ_DEBUG"] if debug else []
     jobs = []
     objs = []
     for src in _sources():
-        obj = os.path.join(BUILD, os.path.basename(src) + ".o")
+        obj = os.path.join(build, os.path.basename(src) + ".o")
         objs.append(obj)
         if src.endswith(".cu"):
             cmd = [nvcc, "-O3", "-std=c++17", ARCH, "-lineinfo", "--expt-relaxed-constexpr",
                    "-Xcompiler", "-fPIC,-ffp-contract=off", "-Xptxas", "-warn-spills",
-                   *inc, "-c", src, "-o", obj]
+                   *defs, *inc, "-c", src, "-o", obj]
         else:
             cmd = ["g++", "-O2", "-std=c++17", "-fPIC", "-ffp-contract=off", "-Wall",
-                   *inc, "-c", src, "-o", obj]
+                   *defs, *inc, "-c", src, "-o", obj]
         jobs.append((cmd, subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.STDOUT)))
     failed = []
     for cmd, p in jobs:
@@ -88,17 +96,17 @@ def build_library(force: bool = False, verbose: bool = False) -> str:
             print(text)
     if failed:
         raise RuntimeError("libpolyq build failed:\n" + "\n".join(failed))
-    tmp = LIB + ".tmp"
+    tmp = lib + ".tmp"
     link = [nvcc, "-shared", ARCH, "-cudart=shared", "-o", tmp, *objs,
             "-Xlinker", "-rpath," + os.path.join(cuda, "lib64"), "-lpthread"]
     p = subprocess.run(link, stdout=subprocess.PIPE, stderr=subprocess.STDOUT)
     if p.returncode != 0:
         raise RuntimeError("libpolyq link failed:\n" + " ".join(link) + "\n"
                            + p.stdout.decode(errors="replace"))
-    os.replace(tmp, LIB)
-    with open(STAMP, "w") as f:
+    os.replace(tmp, lib)
+    with open(os.path.join(build, "stamp.txt"), "w") as f:
         f.write(_stamp_text())
-    return LIB
+    return lib
 
 
 if __name__ == "__main__":

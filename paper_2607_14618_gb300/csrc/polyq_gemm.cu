@@ -39,6 +39,9 @@
 #include <algorithm>
 
 #include "polyq.h"
+#ifdef POLYQ_DEBUG
+#include "polyq_debug.h"
+#endif
 #include "polyq_dev.cuh"
 #include "polyq_internal.h"
 
@@ -415,6 +418,30 @@ __device__ __forceinline__ void dequant_row(int bits, const uint32_t (&w)[8], ui
   }
 }
 
+#ifdef POLYQ_DEBUG
+// Debug build only: every fp16 weight the dequantisers (or, for 16-bit
+// blocks, TMA) place in a B tile is written to g_dbg_w[n][position] (the
+// layer's clustered order), read back from the swizzled tile.
+__device__ uint16_t* g_dbg_w;
+__device__ long long g_dbg_wK;
+
+__device__ __forceinline__ void dbg_row(const uint8_t* btile, int r, int n, int N,
+                                        const GmBlock& B, int hg) {
+  uint16_t* out = g_dbg_w;
+  if (!out || n >= N) return;
+#pragma unroll
+  for (int c = 0; c < 4; ++c) {
+    const uint16_t* src =
+        reinterpret_cast<const uint16_t*>(btile + r * 64 + ((c ^ ((r >> 1) & 3)) << 4));
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      const int w = 32 * hg + slot_code(B.bits, 8 * c + e);
+      if (w < B.n_ch) out[(long long)n * g_dbg_wK + B.pos0 + w] = src[e];
+    }
+  }
+}
+#endif
+
 __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant__ GmParams P) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   // 1024-byte alignment of the operand tiles (128-byte swizzle atoms)
@@ -605,9 +632,19 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
             const uint32_t meta = reinterpret_cast<const uint32_t*>(
                 st + MT * kATile + kBTile + kCodes)[r * 4 + mslot];
             dequant_row(B.bits, w, meta, st + MT * kATile, r);
+#ifdef POLYQ_DEBUG
+            dbg_row(st + MT * kATile, r, un * BN + r, P.N, B, hg);
+#endif
           }
           fence_proxy_async_smem();
         }
+#ifdef POLYQ_DEBUG
+        else {
+          for (int h = 0; h < 2; ++h)
+            dbg_row(stage_ptr(s) + MT * kATile, r0 + 128 * h, un * BN + r0 + 128 * h, P.N, B,
+                    kt - B.kt0);
+        }
+#endif
         __syncwarp();
         if (lane == 0) mbar_arrive(smem_u32(&bar_bready[s]));
       }
@@ -726,6 +763,29 @@ extern "C" int polyq_gemm_workspace_bytes(const polyq_dev_layer* L, int64_t M, s
   *bytes = gemm_workspace(L, M);
   return POLYQ_OK;
 }
+
+#ifdef POLYQ_DEBUG
+// Debug build only: polyq_linear_gemm with every weight placed in a B tile
+// written to w_out [N][K] (fp16 bits, clustered order).
+extern "C" int polyq_debug_gemm_weights(const polyq_dev_layer* L, const void* X, int64_t M,
+                                        float* Y, void* workspace, size_t ws_bytes,
+                                        uint16_t* w_out, void* stream) {
+  polyq_clear_error();
+  cudaStream_t st = (cudaStream_t)stream;
+  const long long K = L ? L->K : 0;
+  cudaError_t e = cudaMemcpyToSymbolAsync(g_dbg_w, &w_out, sizeof w_out, 0,
+                                          cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess)
+    e = cudaMemcpyToSymbolAsync(g_dbg_wK, &K, sizeof K, 0, cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  if (e != cudaSuccess) return polyq_set_error(POLYQ_ECUDA, "debug: %s", cudaGetErrorString(e));
+  const int rc = polyq_linear_gemm(L, X, M, Y, workspace, ws_bytes, stream);
+  uint16_t* none = nullptr;
+  cudaMemcpyToSymbolAsync(g_dbg_w, &none, sizeof none, 0, cudaMemcpyHostToDevice, st);
+  cudaStreamSynchronize(st);
+  return rc;
+}
+#endif
 
 extern "C" int polyq_linear_gemm(const polyq_dev_layer* L, const void* X, int64_t M, float* Y,
                                  void* workspace, size_t ws_bytes, void* stream) {

@@ -40,6 +40,9 @@
 #include <mutex>
 
 #include "polyq.h"
+#ifdef POLYQ_DEBUG
+#include "polyq_debug.h"
+#endif
 #include "polyq_dev.cuh"
 #include "polyq_gemv_dev.cuh"
 #include "polyq_gemv_layout.cuh"
@@ -348,6 +351,11 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) gemv_main(const __grid_c
         d.z = (uint32_t)it.tile;
         d.w = (uint32_t)uvalid2;
         *reinterpret_cast<uint4*>(stages + slot * kStageBytes + kDescOff) = d;
+#ifdef POLYQ_DEBUG
+        *reinterpret_cast<uint4*>(stages + slot * kStageBytes + kDescOff + 16) =
+            make_uint4((uint32_t)(B.pos0 + it.j * B.units), (uint32_t)(it.tile * kRows),
+                       (uint32_t)S.N[it.l], (uint32_t)(B.pos0 + j2 * B.units));
+#endif
       }
       uint32_t bytes = (pair ? 2 : 1) * (nbx * pitch * kRows + RB);
       if (B.bits < 16) bytes += kMetaBytes;
@@ -731,6 +739,29 @@ extern "C" int polyq_linear_gemv(const polyq_dev_layer* L, const void* x, int ba
   return gemv_group("polyq_linear_gemv", one, 1, xs, batch, ys, rs, workspace, ws_bytes,
                     (cudaStream_t)stream);
 }
+
+#ifdef POLYQ_DEBUG
+// Debug build only: polyq_linear_gemv with every code the streaming kernel
+// decodes written to codes_out [N][K] (uint16, clustered order).
+extern "C" int polyq_debug_gemv_codes(const polyq_dev_layer* L, const void* x, int batch, float* y,
+                                      void* workspace, size_t ws_bytes, uint16_t* codes_out,
+                                      void* stream) {
+  polyq_clear_error();
+  cudaStream_t st = (cudaStream_t)stream;
+  const long long K = L ? L->K : 0;
+  cudaError_t e = cudaMemcpyToSymbolAsync(g_dbg_codes, &codes_out, sizeof codes_out, 0,
+                                          cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess)
+    e = cudaMemcpyToSymbolAsync(g_dbg_K, &K, sizeof K, 0, cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  if (e != cudaSuccess) return polyq_set_error(POLYQ_ECUDA, "debug: %s", cudaGetErrorString(e));
+  const int rc = polyq_linear_gemv(L, x, batch, y, nullptr, workspace, ws_bytes, stream);
+  uint16_t* none = nullptr;
+  cudaMemcpyToSymbolAsync(g_dbg_codes, &none, sizeof none, 0, cudaMemcpyHostToDevice, st);
+  cudaStreamSynchronize(st);
+  return rc;
+}
+#endif
 
 extern "C" int polyq_linear_gemv_input(const polyq_dev_layer* const* layers, int n,
                                        const polyq_gemv_input* in, int batch, float* const* ys,

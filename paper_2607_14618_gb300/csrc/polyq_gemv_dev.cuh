@@ -367,6 +367,34 @@ __device__ __forceinline__ void flush_rows(float (&acc)[2], float* y, int N, int
   }
 }
 
+#ifdef POLYQ_DEBUG
+// Debug build only: every code an MMA step decodes is written to
+// g_dbg_codes[row][position] (uint16, the layer's clustered order; for
+// 16-bit weights the fp16 bit pattern), so that tests can compare the hot
+// decoder with the packed bytes bit for bit.  The producer writes the step's
+// first position, first tile row, the layer's N and (paired stages) the
+// second step's first position into the 16 bytes after the descriptor.
+__device__ uint16_t* g_dbg_codes;
+__device__ long long g_dbg_K;
+
+// The two codes of pair register v: (fp16 half - 1024) >> p for each half.
+template <int NB, int BITS>
+__device__ __forceinline__ void dbg_pair(uint32_t v, int jp, int t, int row, int uvalid,
+                                         const uint4& d) {
+  uint16_t* out = g_dbg_codes;
+  if (!out) return;
+  const int r = (int)d.y + row;
+  if (r >= (int)d.z) return;
+  int ulo, plo, uhi, phi;
+  pair_units(BITS, jp, &ulo, &plo, &uhi, &phi);
+  const int u0 = lane_unit(BITS, NB, t, ulo), u1 = lane_unit(BITS, NB, t, uhi);
+  if (u0 < uvalid)
+    out[(long long)r * g_dbg_K + d.x + u0] = (uint16_t)(((v & 0x3FFu) >> plo));
+  if (u1 < uvalid)
+    out[(long long)r * g_dbg_K + d.x + u1] = (uint16_t)((((v >> 16) & 0x3FFu) >> phi));
+}
+#endif
+
 // ---------------------------------------------------------------------------
 // MMA steps
 // ---------------------------------------------------------------------------
@@ -459,6 +487,9 @@ __device__ __forceinline__ void step_mma(uint32_t magic, int batch, int uvalid, 
   const int my_b = g / NGS, my_c = g % NGS;
   const int dc = my_b < batch ? my_c - lane_unit(BITS, NB, t, 0) / 64 : -1000;
   const uint32_t* brow = rec + (my_b * 4 + t) * LW;
+#ifdef POLYQ_DEBUG
+  const uint4 dbg = *reinterpret_cast<const uint4*>(stage + kDescOff + 16);
+#endif
 
   // independent accumulator sets for the step's MMA chain: four for the 32
   // MMAs of a batch-1 step, two for the 8-16 of a batch 2-4 step
@@ -483,6 +514,12 @@ __device__ __forceinline__ void step_mma(uint32_t magic, int batch, int uvalid, 
           const uint32_t a1 = make_pair<BITS>(wb, jp, magic);
           const uint32_t a2 = make_pair<BITS>(wa, jp + 1, magic);
           const uint32_t a3 = make_pair<BITS>(wb, jp + 1, magic);
+#ifdef POLYQ_DEBUG
+          dbg_pair<NB, BITS>(a0, jp, t, rA, uvalid, dbg);
+          dbg_pair<NB, BITS>(a1, jp, t, rB, uvalid, dbg);
+          dbg_pair<NB, BITS>(a2, jp + 1, t, rA, uvalid, dbg);
+          dbg_pair<NB, BITS>(a3, jp + 1, t, rB, uvalid, dbg);
+#endif
           mma_f16_16816(d[(jp / 2) % NACC], a0, a1, a2, a3, hh ? bv.z : bv.x, hh ? bv.w : bv.y);
         }
       }
@@ -549,6 +586,12 @@ __device__ __forceinline__ void step_mma_pair(uint32_t magic, int batch, int g0,
   const int dc = my_b < batch ? my_c - lane_unit(BITS, NB, t, 0) / 64 : -1000;
   const uint32_t* bs[2] = {dc == 0 ? rec0 + (my_b * 4 + t) * LW : zeros,
                            dc == 0 ? rec1 + (my_b * 4 + t) * LW : zeros};
+#ifdef POLYQ_DEBUG
+  const uint4 dbg0 = *reinterpret_cast<const uint4*>(stage + kDescOff + 16);
+  const uint4 dbg1 = make_uint4(dbg0.w, dbg0.y, dbg0.z, 0u);
+  const uint4 dsc = *reinterpret_cast<const uint4*>(stage + kDescOff);
+  const int uv[2] = {(int)(dsc.y & 0xFFFFu), (int)dsc.w};
+#endif
 
   float d[2][2][4];  // per step two accumulator sets: four independent chains
 #pragma unroll
@@ -570,6 +613,15 @@ __device__ __forceinline__ void step_mma_pair(uint32_t magic, int batch, int g0,
           const uint32_t a1 = make_pair<BITS>(wb[k], jp, magic);
           const uint32_t a2 = make_pair<BITS>(wa[k], jp + 1, magic);
           const uint32_t a3 = make_pair<BITS>(wb[k], jp + 1, magic);
+#ifdef POLYQ_DEBUG
+          {
+            const uint4& dg = k ? dbg1 : dbg0;
+            dbg_pair<NB, BITS>(a0, jp, t, rA, uv[k], dg);
+            dbg_pair<NB, BITS>(a1, jp, t, rB, uv[k], dg);
+            dbg_pair<NB, BITS>(a2, jp + 1, t, rA, uv[k], dg);
+            dbg_pair<NB, BITS>(a3, jp + 1, t, rB, uv[k], dg);
+          }
+#endif
           const uint4& bv = k ? bv1 : bv0;
           mma_f16_16816(d[k][(jp / 2) & 1], a0, a1, a2, a3, hh ? bv.z : bv.x, hh ? bv.w : bv.y);
         }
@@ -627,6 +679,21 @@ __device__ __forceinline__ void step_16(int batch, int uvalid,
     const uint4 a0 = pa[0], a1 = pa[1], b0 = pb[0], b1 = pb[1];
     const uint32_t wa[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
     const uint32_t wb[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+#ifdef POLYQ_DEBUG
+    if (g_dbg_codes) {
+      const uint4 dg = *reinterpret_cast<const uint4*>(stage + kDescOff + 16);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        const int u = 64 * h + 16 * t + i;
+        const uint16_t va = (uint16_t)(wa[i / 2] >> (16 * (i & 1)));
+        const uint16_t vb = (uint16_t)(wb[i / 2] >> (16 * (i & 1)));
+        if (u < uvalid && (int)dg.y + rA < (int)dg.z)
+          g_dbg_codes[((long long)dg.y + rA) * g_dbg_K + dg.x + u] = va;
+        if (u < uvalid && (int)dg.y + rB < (int)dg.z)
+          g_dbg_codes[((long long)dg.y + rB) * g_dbg_K + dg.x + u] = vb;
+      }
+    }
+#endif
 #pragma unroll
     for (int m2 = 0; m2 < 2; ++m2) {
       const uint4 bv = *reinterpret_cast<const uint4*>(bsrc + 8 * h + 4 * m2);

@@ -38,7 +38,8 @@ constexpr int kRecMax = 2 * kRecOne;  // a stage may hold two steps' records
 // follow each other).
 constexpr int kRecOff = kCodesBytes + kMetaBytes;
 constexpr int kDescOff = kRecOff + kRecMax;
-constexpr int kStageBytes = ((kDescOff + 16) + 127) / 128 * 128;
+// the descriptor, and 16 bytes that only the debug build writes
+constexpr int kStageBytes = ((kDescOff + 32) + 127) / 128 * 128;
 constexpr uint32_t kMagic = 0x64006400u;  // two fp16 1024.0
 constexpr float kMagicF = 1024.0f;
 

@@ -583,13 +583,17 @@ def gemv_launches_per_call(layer: DeviceLayer, batch: int) -> int:
     return 2
 
 
-def decoder_plan_graph(n_layers, hidden, ffn, perm_of, kv=None, qdim=None):
+def decoder_plan_graph(n_layers, hidden, ffn, perm_of, kv=None, qdim=None, free_source=False,
+                       head=None):
     """Planner input for a decoder stack's decode step: per layer RMSNorm ->
     q, k, v -> attention -> o -> residual add -> RMSNorm -> gate, up ->
-    SiLU * up -> down -> residual add; the stream enters in natural order and
-    leaves through a natural-order boundary.  ``perm_of(layer, name)``
-    returns the permutation id of each linear.  Returns (nodes, edge widths,
-    per-layer edge ids by name)."""
+    SiLU * up -> down -> residual add; by default the stream enters in
+    natural order and leaves through a natural-order boundary.
+    ``free_source``: it enters from an embedding whose columns may be
+    permuted (any order at no cost).  ``head = (perm id, vocab)``: it ends in
+    a final RMSNorm and an output-head linear whose logits leave through a
+    boundary.  ``perm_of(layer, name)`` returns the permutation id of each
+    linear.  Returns (nodes, edge widths, per-layer edge ids by name)."""
     qdim = hidden if qdim is None else qdim
     kv = qdim if kv is None else kv
     nodes, dims, names = [], [], []
@@ -599,7 +603,7 @@ def decoder_plan_graph(n_layers, hidden, ffn, perm_of, kv=None, qdim=None):
         return len(dims) - 1
 
     s = edge(hidden)
-    nodes.append((NODE_SOURCE_FIXED, [], s, -1))
+    nodes.append((NODE_SOURCE_FREE if free_source else NODE_SOURCE_FIXED, [], s, -1))
     for l in range(n_layers):
         e = {"s_in": s, "h": edge(hidden)}
         nodes.append((NODE_ELEMENTWISE, [s], e["h"], -1))
@@ -625,7 +629,14 @@ def decoder_plan_graph(n_layers, hidden, ffn, perm_of, kv=None, qdim=None):
         nodes.append((NODE_ELEMENTWISE, [e["s1"], e["down"]], e["s2"], -1))
         names.append(e)
         s = e["s2"]
-    nodes.append((NODE_BOUNDARY, [s], -1, -1))
+    if head is None:
+        nodes.append((NODE_BOUNDARY, [s], -1, -1))
+    else:
+        hf = edge(hidden)
+        nodes.append((NODE_ELEMENTWISE, [s], hf, -1))  # final RMSNorm
+        logits = edge(head[1])
+        nodes.append((NODE_LINEAR, [hf], logits, head[0]))
+        nodes.append((NODE_BOUNDARY, [logits], -1, -1))
     return nodes, dims, names
 
 

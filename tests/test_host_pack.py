@@ -13,10 +13,25 @@ from paper_2607_14618_gb300 import synth
 HEADER = os.path.join(os.path.dirname(os.path.dirname(__file__)), "include", "polyq.h")
 
 
-def _declared_functions():
-    text = open(HEADER).read()
+def _declared_functions(header=HEADER):
+    text = open(header).read()
     text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
     return sorted(set(re.findall(r"\b(polyq_[a-z0-9_]+)\s*\(", text)))
+
+
+def test_debug_library_exports_its_declared_symbols(polyq_lib):
+    """The debug build (a test aid) exports what include/polyq_debug.h
+    declares, besides everything the product exports; the product library
+    exports none of the debug calls."""
+    from paper_2607_14618_gb300 import build
+    names = _declared_functions(os.path.join(os.path.dirname(HEADER), "polyq_debug.h"))
+    assert names == ["polyq_debug_gemm_weights", "polyq_debug_gemv_codes"]
+    dbg = C.CDLL(build.build_library(debug=True))
+    for n in names + _declared_functions():
+        assert hasattr(dbg, n), n
+    lib = C.CDLL(polyq_lib.LIB_PATH)
+    for n in names:
+        assert not hasattr(lib, n), n
 
 
 def test_library_exports_every_declared_symbol(polyq_lib):

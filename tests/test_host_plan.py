@@ -87,6 +87,14 @@ def test_planner_matches_oracle_on_decoder_graphs(polyq_lib, layers, hidden, ffn
     lo, co = O.plan_graph(nodes, dims, perms)
     lc, cc = polyq_lib.plan_graph(nodes, dims, perms)
     assert list(lc) == lo and cc == co
+    # the same stack entered from a free-order embedding and left through a
+    # linear output head
+    perms.append(rng.permutation(hidden))
+    nodes, dims, _ = O.decoder_graph(layers, hidden, ffn, kv, pid, qdim, True,
+                                     (len(perms) - 1, 32000))
+    lo, co = O.plan_graph(nodes, dims, perms)
+    lc, cc = polyq_lib.plan_graph(nodes, dims, perms)
+    assert list(lc) == lo and cc == co
 
 
 def test_planner_rejects_bad_graphs(polyq_lib):
@@ -110,8 +118,11 @@ def test_planner_rejects_bad_graphs(polyq_lib):
 def test_library_decoder_graph_matches_oracle_graph(polyq_lib):
     def pid(l, nm):
         return 7 * l + ["q", "k", "v", "o", "gate", "up", "down"].index(nm)
-    for args in ((3, 64, 160, None, None), (2, 64, 160, 16, 96)):
-        n1, d1, e1 = polyq_lib.decoder_plan_graph(args[0], args[1], args[2], pid, args[3], args[4])
-        n2, d2, e2 = O.decoder_graph(args[0], args[1], args[2], args[3], pid, args[4])
+    for args in ((3, 64, 160, None, None, False, None), (2, 64, 160, 16, 96, False, None),
+                 (2, 64, 160, None, None, True, (14, 500)), (1, 64, 160, 16, 96, False, (7, 9))):
+        n1, d1, e1 = polyq_lib.decoder_plan_graph(args[0], args[1], args[2], pid, args[3], args[4],
+                                                  args[5], args[6])
+        n2, d2, e2 = O.decoder_graph(args[0], args[1], args[2], args[3], pid, args[4], args[5],
+                                     args[6])
         assert [(k, list(i), o, p) for k, i, o, p in n1] == [(k, list(i), o, p) for k, i, o, p in n2]
         assert list(d1) == list(d2) and e1 == e2

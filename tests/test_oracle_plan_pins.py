@@ -203,3 +203,30 @@ def test_planned_stack_equals_the_unplanned_stack_bit_for_bit():
             if g1 is not None:
                 assert np.array_equal(g1, g2)
     assert np.array_equal(s_plan, s_nat)
+
+
+@pytest.mark.parametrize("free_source,head,shuffles,stream_label", [
+    (False, None, 2, O.NATURAL),     # q/k/v and gate/up gather the natural stream
+    (True, None, 2, O.NATURAL),      # a free source alone changes nothing: the
+                                     # boundary still wants natural order
+    (False, True, 3, O.NATURAL),     # a linear head adds its own gather
+    (True, True, 2, 0),              # the stream takes q/k/v's order from the
+                                     # embedding: q/k/v read it as is, gate/up
+                                     # and the head gather
+])
+def test_free_embedding_and_linear_head_hand_worked(free_source, head, shuffles, stream_label):
+    # One grouped layer: q/k/v share permutation 0, o has 1, gate/up share 2,
+    # down has 3, the head 4.  The residual stream, both RMSNorm outputs and
+    # the o/down outputs form one region (joined by elementwise nodes); every
+    # other region is free.  Each order wanted from that region costs one
+    # shuffle of 64 channels at 4 bytes (Section 5.3); worked by hand.
+    rng = np.random.default_rng(9)
+    perms = [rng.permutation(64), rng.permutation(64), rng.permutation(64),
+             rng.permutation(160), rng.permutation(64)]
+    pid = {"q": 0, "k": 0, "v": 0, "o": 1, "gate": 2, "up": 2, "down": 3}
+    nodes, dims, names = O.decoder_graph(1, 64, 160, None, lambda l, nm: pid[nm], None,
+                                         free_source, (4, 100) if head else None)
+    labels, cost = O.plan_graph(nodes, dims, perms)
+    assert cost == shuffles * 4 * 64
+    assert labels[names[0]["s_in"]] == stream_label
+    assert labels[names[0]["h"]] == stream_label and labels[names[0]["s2"]] == stream_label
