@@ -917,8 +917,11 @@ extern "C" int polyq_linear_gemm(const polyq_dev_layer* L, const void* X, int64_
   cudaError_t e = cudaLaunchKernelEx(&cfg, gemm_prep, P);
   if (e != cudaSuccess)
     return polyq_set_error(POLYQ_ECUDA, "polyq_linear_gemm: prep launch: %s", cudaGetErrorString(e));
-  // no programmatic overlap for the main kernel: it owns all of TMEM on an SM
-  cfg.numAttrs = 0;
+  // The main kernel may launch while the pre-pass runs (programmatic
+  // dependent launch): its set-up overlaps the pre-pass, and its producer
+  // waits for the pre-pass before the first load of Xg.  It allocates all of
+  // an SM's tensor memory, which is safe because two of its CTAs (197 KB of
+  // shared memory each) never share an SM.
   cfg.gridDim = dim3((unsigned)(P.streamk ? sms : std::min(P.units, sms)));
   cfg.blockDim = dim3(kThreadsG);
   cfg.dynamicSmemBytes = smem;
