@@ -677,7 +677,7 @@ def bench_decode_step(polyq, synth, torch, device, stream, args, hbm):
             del chain
         del stack, base, hosts
         torch.cuda.empty_cache()
-    # §5.3 model of activation-reorder traffic per token (A16 read + write of
+    # §5.4 model of activation-reorder traffic per token (A16 read + write of
     # each explicit shuffle): without merges every linear shuffles its input
     no_merge = 4 * L * sum(k for _, _, k in LLAMA)
     for mode in out:
@@ -693,7 +693,7 @@ def bench_decode_step(polyq, synth, torch, device, stream, args, hbm):
 def plan_report(polyq):
     """§4.4 planning of the whole decode graph (host, no GPU) on the
     Llama2-13B and Qwen3-32B shapes: modelled activation-reorder traffic per
-    token (§5.3 model) without merges and with the library planner, for
+    token (§5.4 model) without merges and with the library planner, for
     separately allocated linears and for q/k/v and gate/up allocated jointly.
     Every layer gets its own seeded permutations (distinct allocations)."""
     shapes = {"llama2_13b": dict(layers=40, hidden=5120, ffn=13824, kv=None, qdim=None,

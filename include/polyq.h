@@ -262,7 +262,7 @@ typedef struct {
 
 /* Assign a channel order ("basis") to every edge so that the explicit
  * activation shuffles the graph needs cost the least modelled traffic
- * (Section 4.4; the traffic model is Section 5.3's A16 read + write, 4 bytes
+ * (Section 4.4; the traffic model is Section 5.4's A16 read + write, 4 bytes
  * per channel per shuffle).  Edges joined by elementwise nodes (and by an
  * attention node that keeps v's order) form regions that share one order;
  * each region takes, among the natural order and the permutations of the
@@ -504,7 +504,7 @@ int polyq_workspace_status(const void* workspace, int* status, void* stream);
 int polyq_gemm_workspace_bytes(const polyq_dev_layer* layer, int64_t M,
                                size_t* bytes);
 
-/* Prefill GEMM (the same product for M tokens, Section 5.4 prefill):
+/* Prefill GEMM (the same product for M tokens, Section 5.5 prefill):
  *   Y[m][n] = sum_p X[m][gather[p]] * W'[n][p]
  * X: device bf16 [M][K], any finite values; Y: device fp32 [M][N], 16-byte
  * aligned (else POLYQ_EINVAL); workspace as for the GEMV (its status word in

@@ -22,7 +22,7 @@ What is restated here (PolyQ, arXiv 2607.14618):
 * §4.3  the merge rule ``O' = A (W P^T)(P W')``: the producer emits its
         outputs in the consumer's basis, so the consumer's gather becomes the
         identity.
-* §5.3  the per-token reorder-traffic model (A16 read+write bytes of explicit
+* §5.4  the per-token reorder-traffic model (A16 read+write bytes of explicit
         activation shuffles).
 
 Readings taken where the paper is silent:
@@ -75,7 +75,7 @@ R17 graph planning (§4.4): edges carry a channel basis; linears absorb any
    edges joined by basis-keeping nodes form regions; each region takes the
    candidate basis (natural, or a consuming linear's permutation) with the
    smallest modelled traffic, where one explicit shuffle of an edge into a
-   basis costs 4 bytes per channel (A16 read + write, §5.3) and is shared
+   basis costs 4 bytes per channel (A16 read + write, §5.4) and is shared
    by every consumer of that edge wanting that basis; ties go to natural,
    then to the lowest permutation id.
 R16 bit-specific scaling (§3.4): m_k = a_k / mean(a) (a = the activation
@@ -467,12 +467,12 @@ def permute_rows(layer, row_perm):
 
 
 # ---------------------------------------------------------------------------
-# §5.3: reorder-traffic model
+# §5.4: reorder-traffic model
 # ---------------------------------------------------------------------------
 def reorder_traffic_bytes(gathered_k, n_layers):
     """Per-token A16 read+write bytes of explicit activation shuffles: each
     shuffled activation of K channels costs 2 bytes read + 2 bytes written
-    per channel (§5.3)."""
+    per channel (§5.4)."""
     return 4 * int(sum(gathered_k)) * int(n_layers)
 
 
@@ -958,7 +958,7 @@ def plan_graph(nodes, edge_dims, perms):
 
 
 def no_merge_traffic(nodes, edge_dims):
-    """The per-layer-gather baseline of §5.3: every linear input shuffled."""
+    """The per-layer-gather baseline of §5.4: every linear input shuffled."""
     return 4 * sum(edge_dims[i[0]] for k, i, o, p in nodes if k == NODE_LINEAR)
 
 

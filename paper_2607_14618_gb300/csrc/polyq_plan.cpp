@@ -1,7 +1,7 @@
 // Section 4.4 graph-based permutation planning on the host: channel orders
 // ("bases") for the activation edges of a static operator DAG, chosen so
 // that the explicit activation shuffles cost the least modelled traffic
-// (Section 5.3: A16 read + write, 4 bytes per channel per shuffle).
+// (Section 5.4: A16 read + write, 4 bytes per channel per shuffle).
 //
 // Edges joined by order-keeping nodes form regions; every edge of a region
 // carries the same order.  A region's cost for a candidate order is one

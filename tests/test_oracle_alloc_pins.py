@@ -301,7 +301,7 @@ def test_scaling_never_raises_the_block_error():
 
 
 # ---------------------------------------------------------------------------
-# Section 5.2 (Figure 6 shape): budget kept after snapping, padding removed
+# Section 5.3 (Figure 7): budget kept after snapping, padding removed
 # ---------------------------------------------------------------------------
 @pytest.mark.parametrize("B", [3.0, 3.5, 4.0, 5.0, 6.0])
 def test_snapped_budget_stays_within_the_papers_mismatch(B):

@@ -1,5 +1,5 @@
 """Pins of the oracle's graph planner (Section 4.4, traffic model of
-Section 5.3): the paper's per-layer-gather baselines, hand-worked graphs,
+Section 5.4): the paper's per-layer-gather baselines, hand-worked graphs,
 exhaustive search on small graphs, and execution of a planned stack against
 the unplanned one.  CPU only."""
 import itertools
@@ -29,8 +29,8 @@ def _distinct_perms(hidden, ffn, qdim=None, grouped=False, seed=0):
 
 
 @pytest.mark.parametrize("layers,hidden,ffn,kv,qdim,paper_mib", [
-    (40, 5120, 13824, None, None, 6.80),   # Llama2-13B (§5.3)
-    (64, 5120, 25600, 1024, 8192, 14.50),  # Qwen3-32B (§5.3)
+    (40, 5120, 13824, None, None, 6.80),   # Llama2-13B (§5.4)
+    (64, 5120, 25600, 1024, 8192, 14.50),  # Qwen3-32B (§5.4)
 ])
 def test_no_merge_baseline_reproduces_the_papers_traffic(layers, hidden, ffn, kv, qdim,
                                                          paper_mib):
@@ -219,7 +219,7 @@ def test_free_embedding_and_linear_head_hand_worked(free_source, head, shuffles,
     # down has 3, the head 4.  The residual stream, both RMSNorm outputs and
     # the o/down outputs form one region (joined by elementwise nodes); every
     # other region is free.  Each order wanted from that region costs one
-    # shuffle of 64 channels at 4 bytes (Section 5.3); worked by hand.
+    # shuffle of 64 channels at 4 bytes (Section 5.4); worked by hand.
     rng = np.random.default_rng(9)
     perms = [rng.permutation(64), rng.permutation(64), rng.permutation(64),
              rng.permutation(160), rng.permutation(64)]
