@@ -19,7 +19,10 @@ import bench
 dist.init_process_group("gloo", init_method="env://")
 ws, rank, _ = bench._dist()
 ms = bench.max_over_ranks(10.0 + 5.0 * rank, ws, "cpu")
-print(json.dumps({{"rank": rank, "ms": ms, "tbs": bench.job_tbs(ws, 1000000, 20, ms)}}))
+# per timed window, the slower rank's duration
+win = bench.window_max_over_ranks([1.0 + rank, 3.0 - rank, 2.0], ws, "cpu")
+print(json.dumps({{"rank": rank, "ms": ms, "tbs": bench.job_tbs(ws, 1000000, 20, ms),
+                  "win": win}}))
 dist.destroy_process_group()
 """
 
@@ -46,6 +49,7 @@ def test_two_gloo_ranks_take_the_slowest_time_and_sum_the_replicas():
         outs.append(json.loads(out.strip().splitlines()[-1]))
     for o in outs:
         assert o["ms"] == 15.0  # the slower rank's 15 ms, on every rank
+        assert o["win"] == [2.0, 3.0, 2.0]
         # two replicas of 1 MB per step, 20 steps in 15 ms
         assert abs(o["tbs"] - 2 * 1e6 * 20 / 15e-3 / 1e12) < 1e-12
 
@@ -63,4 +67,5 @@ def test_single_rank_needs_no_process_group():
     sys.path.insert(0, ROOT)
     import bench
     assert bench.max_over_ranks(12.5, 1) == 12.5
+    assert bench.window_max_over_ranks([1.0, 2.0], 1) == [1.0, 2.0]
     assert bench.job_tbs(1, 142208000, 10, 0.5) == 142208000 * 10 / 0.5e-3 / 1e12

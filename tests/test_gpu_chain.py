@@ -205,3 +205,31 @@ def test_record_wait_gives_up_with_a_status(polyq_lib):
     torch.cuda.synchronize()
     assert polyq_lib.workspace_status(chain.workspace) == 0
     check_tolerance(y.cpu().numpy(), O.linear(ref, x), x, K)
+
+
+@pytest.mark.parametrize("batch", [1, 4])
+@pytest.mark.parametrize("scale_exp", [-40, 12, 40])
+def test_chained_phases_at_any_activation_scale(polyq_lib, batch, scale_exp):
+    """The chained launch builds its records with the same per-chunk exponent
+    as the per-call pre-pass: two dependent-free phases of all five widths,
+    with inputs scaled by 2^scale_exp, against the oracle."""
+    phases, refs, xs = [], [], []
+    for i, (N, K) in enumerate(((200, 3001), (96, 1100))):
+        W, a = synth.layer_weights(N, K, 90 + i)
+        bits = synth.random_codes_layer_bits(K, 90 + i)
+        host = polyq_lib.HostLayer.pack(W, a, 3.0, forced_bits=bits)
+        dev = polyq_lib.DeviceLayer(host, "cuda")
+        refs.append(O.pack_layer(W, a, 3.0, bits=bits))
+        _, x = synth.activations(a, batch, 90 + i)
+        x = x * 2.0 ** scale_exp
+        xb = synth.bf16_bits(x.astype(np.float32))
+        assert np.array_equal(synth.bf16_to_f64(xb), x)
+        xs.append(x)
+        y = torch.zeros((batch, N), dtype=torch.float32, device="cuda")
+        phases.append(dict(layers=[dev], kind=polyq_lib.X_BF16, a=_x_dev(xb), ys=[y]))
+    chain = polyq_lib.GemvChain(phases, batch=batch)
+    chain.run()
+    torch.cuda.synchronize()
+    assert polyq_lib.workspace_status(chain.workspace) == 0
+    for ph, ref, x in zip(phases, refs, xs):
+        check_tolerance(ph["ys"][0].cpu().numpy(), O.linear(ref, x), x, x.shape[1])
