@@ -310,7 +310,8 @@ int polyq_gemv_workspace_bytes(const polyq_dev_layer* layer, int batch,
  * copies are exact whatever the activations' absolute scale, except for
  * values more than about 2^20 below their group's largest, which lose low
  * bits as fp16 subnormals (each by at most 2^-31 of that largest value).  batch in 1..4; y: device fp32 [batch][N];
- * residual: device fp32 [batch][N] or NULL (y may alias residual).  y is
+ * residual: device fp32 [batch][N] or NULL (y may alias residual; y must not
+ * overlap x or the workspace).  y is
  * first set to the residual (or zero), then each of the few pieces a row's
  * sum is split into is added with an fp32 atomic addition, so the last bits
  * of y may differ from run to run.  workspace: device scratch of at least

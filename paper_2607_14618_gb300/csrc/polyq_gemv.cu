@@ -227,12 +227,66 @@ __device__ __forceinline__ void fence_proxy_async_global() {
   asm volatile("fence.proxy.async.global;" ::: "memory");
 }
 
+// y starts as the residual (or zero); the main kernel adds its pieces.  Done
+// by CTAs of the pre-pass that build no record (CTA `cta` of `n_cta`), in
+// parallel with those that do.
+__device__ __forceinline__ void init_outputs(const GvParams& P, int cta, int n_cta) {
+  // 16-byte stores (and residual loads) where y and the residual allow them;
+  // a thread's loads of one round are in flight together.
+#pragma unroll
+  for (int q = 0; q < POLYQ_MAX_GROUP; ++q) {
+    if (q >= P.n_layers) break;
+    float* y = P.L[q].y;
+    const float* res = P.L[q].residual;
+    if (y == res) continue;
+    const int total = P.batch * P.L[q].N;
+    const int st = n_cta * blockDim.x;
+    const int t0 = cta * blockDim.x + threadIdx.x;
+    const bool vec = total % 4 == 0 && reinterpret_cast<uintptr_t>(y) % 16 == 0 &&
+                     reinterpret_cast<uintptr_t>(res) % 16 == 0;
+    if (vec) {
+      float4* y4 = reinterpret_cast<float4*>(y);
+      const float4* r4 = reinterpret_cast<const float4*>(res);
+      const int n4 = total / 4;
+      for (int i0 = t0; i0 < n4; i0 += 2 * st) {
+        float4 v[2];
+#pragma unroll
+        for (int u = 0; u < 2; ++u)
+          v[u] = (res && i0 + u * st < n4) ? r4[i0 + u * st] : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int u = 0; u < 2; ++u)
+          if (i0 + u * st < n4) y4[i0 + u * st] = v[u];
+      }
+    } else {
+      for (int i0 = t0; i0 < total; i0 += 4 * st) {
+        float v[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) v[u] = (res && i0 + u * st < total) ? res[i0 + u * st] : 0.f;
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          if (i0 + u * st < total) y[i0 + u * st] = v[u];
+      }
+    }
+  }
+}
+
 // ---------------------------------------------------------------------------
-// pre-pass: one CTA of 128 threads per activation record (layer, step)
+// pre-pass: one CTA of 256 threads per activation record (layer, step); each
+// thread builds at most one (batch, chunk) slot of it, which keeps the chain
+// of dependent instructions between the activation loads and the record
+// stores short.  A few more CTAs initialise the outputs.
 // ---------------------------------------------------------------------------
+constexpr int kPrepWarps = 8;
+constexpr int kPrepThreads = 32 * kPrepWarps;
+
 template <int NB>
-__global__ void __launch_bounds__(kConsumers) gemv_prep(const __grid_constant__ GvParams P) {
+__global__ void __launch_bounds__(kPrepThreads) gemv_prep(const __grid_constant__ GvParams P) {
   pdl_trigger();  // the main kernel may start streaming weights right away
+  if ((int)blockIdx.x >= P.recs) {
+    pdl_wait();  // y may still be in use by earlier kernels
+    init_outputs(P, (int)blockIdx.x - P.recs, (int)gridDim.x - P.recs);
+    return;
+  }
   __shared__ GvShared S;
   __shared__ uint32_t s_p3[16];  // 3-bit pair schedule
   load_shared(P, &S);
@@ -248,30 +302,20 @@ __global__ void __launch_bounds__(kConsumers) gemv_prep(const __grid_constant__ 
   int src[2][2];
   float fac[2][2];
   const XIn in = xin_of(P, l);
-  rec_sources<NB>(in, S.blk[l][bi], j, warp, lane, s_p3, src, fac);  // static layer data
+  rec_sources<NB, kPrepWarps>(in, S.blk[l][bi], j, warp, lane, s_p3, src, fac);  // static layer data
   if (P.xkind == POLYQ_X_RMSNORM) rms_prefetch(P.xa, P.L[0].K, P.batch);
   pdl_wait();  // x comes from the previous kernel; the records and y may still be in use
   // The streaming kernel writes the status only after its own wait for this
   // grid, so clearing it here cannot lose one of its reports.
   if (P.clear_status && blockIdx.x == 0 && threadIdx.x == 0) *P.status = 0;
   float ra[2][2], rb[2][2];
-  rec_load<NB>(in, S.blk[l][bi], j, warp, lane, s_p3, src, ra, rb);
+  rec_load<NB, kPrepWarps>(in, S.blk[l][bi], j, warp, lane, s_p3, src, ra, rb);
   __shared__ float s_rnorm[4];
-  __shared__ float s_part[4][kWarps];
-  if (P.xkind == POLYQ_X_RMSNORM) rms_rnorm(P.xa, P.L[0].K, P.batch, P.eps, s_part, s_rnorm);
-  rec_store<NB>(in, S.blk[l][bi], j, warp, lane, s_p3, src, fac, ra, rb, s_rnorm,
-                reinterpret_cast<uint32_t*>(P.rec + (size_t)r * rec_bytes(NB)));
-  // y starts as the residual (or zero); the main kernel adds its pieces
-#pragma unroll
-  for (int q = 0; q < POLYQ_MAX_GROUP; ++q) {
-    if (q >= P.n_layers) break;
-    float* y = P.L[q].y;
-    const float* res = P.L[q].residual;
-    if (y == res) continue;
-    const int total = P.batch * P.L[q].N;
-    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < total; i += gridDim.x * blockDim.x)
-      y[i] = res ? res[i] : 0.f;
-  }
+  __shared__ float s_part[4][kPrepWarps];
+  if (P.xkind == POLYQ_X_RMSNORM)
+    rms_rnorm<kPrepWarps>(P.xa, P.L[0].K, P.batch, P.eps, s_part, s_rnorm);
+  rec_store<NB, kPrepWarps>(in, S.blk[l][bi], j, warp, lane, s_p3, src, fac, ra, rb, s_rnorm,
+                            reinterpret_cast<uint32_t*>(P.rec + (size_t)r * rec_bytes(NB)));
 }
 
 template <int NB>
@@ -595,8 +639,13 @@ int launch(const GvParams& P, int grid, cudaStream_t st) {
   cfg.stream = st;
   cfg.attrs = at;
   cfg.numAttrs = 1;
-  cfg.gridDim = dim3((unsigned)P.recs);
-  cfg.blockDim = dim3(kConsumers);
+  // record CTAs, then output-initialising CTAs (eight floats per thread)
+  long long init = 0;
+  for (int q = 0; q < P.n_layers; ++q)
+    if (P.L[q].y != P.L[q].residual) init += (long long)P.batch * P.L[q].N;
+  const int n_init = (int)std::min<long long>(64, (init + 8 * kPrepThreads - 1) / (8 * kPrepThreads));
+  cfg.gridDim = dim3((unsigned)(P.recs + n_init));
+  cfg.blockDim = dim3(kPrepThreads);
   cfg.dynamicSmemBytes = 0;
   cudaError_t e = cudaLaunchKernelEx(&cfg, gemv_prep<NB>, P);
   if (e != cudaSuccess)

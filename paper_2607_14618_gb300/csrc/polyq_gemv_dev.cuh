@@ -24,6 +24,9 @@ struct GvBlock {
   int units;           // units per step
 };
 
+// 2^k as a float, for -126 <= k <= 127 (a normal number: exponent field k + 127).
+__device__ __forceinline__ float pow2i(int k) { return __int_as_float((k + 127) << 23); }
+
 __device__ __forceinline__ uint32_t pack_half2(__half lo, __half hi) {
   return (uint32_t)__half_as_ushort(lo) | ((uint32_t)__half_as_ushort(hi) << 16);
 }
@@ -43,12 +46,15 @@ struct SlotGeom {
   int p[2];   // power-of-two scale exponents of the two halves
 };
 
-template <int NB, int BITS>
+// NW warps build a record: a thread has slots s < rec_slots(NW).
+__host__ __device__ constexpr int rec_slots(int nw) { return nw >= 8 ? 1 : 2; }
+
+template <int NB, int BITS, int NW>
 __device__ __forceinline__ SlotGeom slot_geom_t(int warp, int lane, int tid, int s, int j,
                                                 const uint32_t* p3) {
   SlotGeom g;
   if constexpr (BITS == 16) {
-    const int e = tid + kConsumers * s;
+    const int e = tid + 32 * NW * s;
     g.valid = e < NB * 64;
     g.bb = e / 64;
     g.t = (e / 16) % 4;
@@ -60,7 +66,7 @@ __device__ __forceinline__ SlotGeom slot_geom_t(int warp, int lane, int tid, int
   } else {
     constexpr int U = step_units(BITS, NB), NGS = U / 64;
     constexpr int GP = group_pairs(BITS), GU = group_units(BITS);
-    const int bc = warp + kWarps * s;
+    const int bc = warp + NW * s;
     g.valid = bc < NB * NGS;
     g.bb = bc / NGS;
     g.c = bc - g.bb * NGS;
@@ -87,15 +93,15 @@ __device__ __forceinline__ SlotGeom slot_geom_t(int warp, int lane, int tid, int
   return g;
 }
 
-template <int NB>
+template <int NB, int NW>
 __device__ __forceinline__ SlotGeom slot_geom(int bits, int warp, int lane, int tid, int s,
                                               int j, const uint32_t* p3) {
   switch (bits) {
-    case 2: return slot_geom_t<NB, 2>(warp, lane, tid, s, j, p3);
-    case 3: return slot_geom_t<NB, 3>(warp, lane, tid, s, j, p3);
-    case 4: return slot_geom_t<NB, 4>(warp, lane, tid, s, j, p3);
-    case 8: return slot_geom_t<NB, 8>(warp, lane, tid, s, j, p3);
-    default: return slot_geom_t<NB, 16>(warp, lane, tid, s, j, p3);
+    case 2: return slot_geom_t<NB, 2, NW>(warp, lane, tid, s, j, p3);
+    case 3: return slot_geom_t<NB, 3, NW>(warp, lane, tid, s, j, p3);
+    case 4: return slot_geom_t<NB, 4, NW>(warp, lane, tid, s, j, p3);
+    case 8: return slot_geom_t<NB, 8, NW>(warp, lane, tid, s, j, p3);
+    default: return slot_geom_t<NB, 16, NW>(warp, lane, tid, s, j, p3);
   }
 }
 
@@ -121,7 +127,7 @@ __device__ __forceinline__ void prefetch_l2(const void* p) {
 // prefetch of the activations the record will read.  L2 is where writes of
 // earlier kernels land, so prefetching before their completion is safe: the
 // loads after the wait still see the final values.
-template <int NB>
+template <int NB, int NW = kWarps>
 __device__ __forceinline__ void rec_sources(const XIn& in, const GvBlock& B, int j, int warp,
                                             int lane, const uint32_t* p3, int (&src)[2][2],
                                             float (&fac)[2][2]) {
@@ -130,7 +136,8 @@ __device__ __forceinline__ void rec_sources(const XIn& in, const GvBlock& B, int
   for (int s = 0; s < 2; ++s) {
     src[s][0] = src[s][1] = -1;
     fac[s][0] = fac[s][1] = 1.f;
-    const SlotGeom g = slot_geom<NB>(B.bits, warp, lane, threadIdx.x, s, j, p3);
+    if (s >= rec_slots(NW)) continue;
+    const SlotGeom g = slot_geom<NB, NW>(B.bits, warp, lane, threadIdx.x, s, j, p3);
     if (g.valid && g.bb < in.batch) {
 #pragma unroll
       for (int h = 0; h < 2; ++h)
@@ -150,10 +157,11 @@ __device__ __forceinline__ void rec_sources(const XIn& in, const GvBlock& B, int
   }
 }
 
-// Barrier of the 128 consumer threads (named barrier 1; the producer warp of
-// a streaming kernel does not take part).
+// Barrier of the 32 * NW threads that build records (named barrier 1; the
+// producer warp of a streaming kernel does not take part).
+template <int NW = kWarps>
 __device__ __forceinline__ void consumer_sync() {
-  asm volatile("bar.sync 1, %0;" ::"n"(kConsumers) : "memory");
+  asm volatile("bar.sync 1, %0;" ::"n"(32 * NW) : "memory");
 }
 
 // L2 prefetch of the batch rows the RMSNorm factor reads (before a wait).
@@ -168,8 +176,10 @@ __device__ __forceinline__ void rms_prefetch(const float* xa, int K, int batch) 
 // batch x kWarps partial sums.  A thread's loads of up to kRmsBatch float4
 // are issued together (one L2 round trip for rows up to 8192 wide).
 constexpr int kRmsBatch = 16;
+template <int NW = kWarps>
 __device__ __forceinline__ void rms_rnorm(const float* xa, int K, int batch, float eps,
-                                          float (*s_part)[kWarps], float* s_rnorm) {
+                                          float (*s_part)[NW], float* s_rnorm) {
+  constexpr int NT = 32 * NW;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const bool vec = (K % 4 == 0) && (reinterpret_cast<uintptr_t>(xa) % 16 == 0);
   for (int bb = 0; bb < batch; ++bb) {
@@ -177,11 +187,11 @@ __device__ __forceinline__ void rms_rnorm(const float* xa, int K, int batch, flo
     float acc = 0.f;
     if (vec) {
       const int n4 = K / 4;
-      for (int i0 = threadIdx.x; i0 < n4; i0 += kRmsBatch * kConsumers) {
+      for (int i0 = threadIdx.x; i0 < n4; i0 += kRmsBatch * NT) {
         float4 v[kRmsBatch];
 #pragma unroll
         for (int u = 0; u < kRmsBatch; ++u) {
-          const int i = i0 + u * kConsumers;
+          const int i = i0 + u * NT;
           v[u] = i < n4 ? __ldcg(reinterpret_cast<const float4*>(row) + i)
                         : make_float4(0.f, 0.f, 0.f, 0.f);
         }
@@ -194,7 +204,7 @@ __device__ __forceinline__ void rms_rnorm(const float* xa, int K, int batch, flo
         }
       }
     } else {
-      for (int i = threadIdx.x; i < K; i += kConsumers) {
+      for (int i = threadIdx.x; i < K; i += NT) {
         const float v = __ldcg(row + i);
         acc = fmaf(v, v, acc);
       }
@@ -203,28 +213,29 @@ __device__ __forceinline__ void rms_rnorm(const float* xa, int K, int batch, flo
     for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
     if (lane == 0) s_part[bb][warp] = acc;
   }
-  consumer_sync();
+  consumer_sync<NW>();
   if (threadIdx.x < batch) {
     float t = 0.f;
-    for (int w = 0; w < kWarps; ++w) t += s_part[threadIdx.x][w];
+    for (int w = 0; w < NW; ++w) t += s_part[threadIdx.x][w];
     s_rnorm[threadIdx.x] = rsqrtf(t / (float)K + eps);
   }
-  consumer_sync();
+  consumer_sync<NW>();
 }
 
 // Pass 2 of a record: load the thread's raw inputs (bf16 x, or the fp32
 // inputs of the transform).  Loads go through L2 (ld.global.cg) because in
 // the chained kernel the inputs are written during the same launch.
-template <int NB>
+template <int NB, int NW = kWarps>
 __device__ __forceinline__ void rec_load(const XIn& in, const GvBlock& B, int j, int warp,
                                          int lane, const uint32_t* p3, const int (&src)[2][2],
                                          float (&ra)[2][2], float (&rb)[2][2]) {
 #pragma unroll
   for (int s = 0; s < 2; ++s) {
-    const SlotGeom g = slot_geom<NB>(B.bits, warp, lane, threadIdx.x, s, j, p3);
+    ra[s][0] = ra[s][1] = rb[s][0] = rb[s][1] = 0.f;
+    if (s >= rec_slots(NW)) continue;
+    const SlotGeom g = slot_geom<NB, NW>(B.bits, warp, lane, threadIdx.x, s, j, p3);
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
-      ra[s][h] = rb[s][h] = 0.f;
       if (src[s][h] < 0) continue;
       const size_t o = (size_t)g.bb * in.K + src[s][h];
       if (in.kind == POLYQ_X_BF16) {
@@ -242,7 +253,7 @@ __device__ __forceinline__ void rec_load(const XIn& in, const GvBlock& B, int j,
 // bf16 copy, multiply by the activation factor, scale each value by the power
 // of two its code carries, round to fp16 and store the pairs and (b < 16)
 // the per-chunk sums C1 = 1024 * sum x' and X = sum x' * 2^p.
-template <int NB>
+template <int NB, int NW = kWarps>
 __device__ __forceinline__ void rec_store(const XIn& in, const GvBlock& B, int j, int warp,
                                           int lane, const uint32_t* p3, const int (&src)[2][2],
                                           const float (&fac)[2][2], const float (&ra)[2][2],
@@ -251,10 +262,11 @@ __device__ __forceinline__ void rec_store(const XIn& in, const GvBlock& B, int j
   constexpr int LW = rec_lane_words(NB);
   constexpr int PW = rec_pair_words(NB);
   constexpr int NGM = 8 / NB;
+  constexpr int SL = rec_slots(NW);
   float xv[2][2];
 #pragma unroll
-  for (int s = 0; s < 2; ++s) {
-    const SlotGeom g = slot_geom<NB>(B.bits, warp, lane, threadIdx.x, s, j, p3);
+  for (int s = 0; s < SL; ++s) {
+    const SlotGeom g = slot_geom<NB, NW>(B.bits, warp, lane, threadIdx.x, s, j, p3);
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
       if (src[s][h] < 0) {
@@ -283,38 +295,41 @@ __device__ __forceinline__ void rec_store(const XIn& in, const GvBlock& B, int j
   // exactly one chunk; a 16-bit batch row spans warps w and w ^ 1, which
   // exchange their maxima through shared memory (the width is uniform over
   // the record, so every consumer thread takes the same branch).
-  uint32_t mx[2];
+  uint32_t mx[2] = {0u, 0u};
 #pragma unroll
-  for (int s = 0; s < 2; ++s)
+  for (int s = 0; s < SL; ++s)
     mx[s] = __reduce_max_sync(0xffffffffu, max(__float_as_uint(fabsf(xv[s][0])),
                                                __float_as_uint(fabsf(xv[s][1]))));
   if (B.bits == 16) {
-    __shared__ uint32_t s_wmax[kWarps][2];
-    consumer_sync();  // an earlier record's readers are done with s_wmax
+    __shared__ uint32_t s_wmax[NW][2];
+    consumer_sync<NW>();  // an earlier record's readers are done with s_wmax
     if (lane == 0) {
       s_wmax[warp][0] = mx[0];
       s_wmax[warp][1] = mx[1];
     }
-    consumer_sync();
+    consumer_sync<NW>();
     mx[0] = max(mx[0], s_wmax[warp ^ 1][0]);
     mx[1] = max(mx[1], s_wmax[warp ^ 1][1]);
   }
   float* recf = reinterpret_cast<float*>(rec);
 #pragma unroll
-  for (int s = 0; s < 2; ++s) {
-    const SlotGeom g = slot_geom<NB>(B.bits, warp, lane, threadIdx.x, s, j, p3);
+  for (int s = 0; s < SL; ++s) {
+    const SlotGeom g = slot_geom<NB, NW>(B.bits, warp, lane, threadIdx.x, s, j, p3);
     if (!g.valid) continue;  // uniform over the warp
     // e: floor(log2(max)) - kRecExp (an fp32 subnormal maximum counts as 2^-127)
     const int e = mx[s] ? max((int)(mx[s] >> 23) - 127 - kRecExp, kRecExpMin) : 0;
-    const __half hlo = __float2half_rn(ldexpf(xv[s][0], -g.p[0] - e));
-    const __half hhi = __float2half_rn(ldexpf(xv[s][1], -g.p[1] - e));
+    // 2^(-p-e) lies in [2^-121, 2^126] (p <= 8, -126 <= e <= 113): a
+    // normal float, so the products are exact scalings (rounded like any
+    // product where they fall below the normal range)
+    const __half hlo = __float2half_rn(xv[s][0] * pow2i(-g.p[0] - e));
+    const __half hhi = __float2half_rn(xv[s][1] * pow2i(-g.p[1] - e));
     rec[(g.bb * 4 + g.t) * LW + g.jp] = pack_half2(hlo, hhi);
     if (B.bits != 16) {
       // X sums the values the MMA multiplies (fp16 times 2^p), so that the
       // zero-point term removes exactly what the codes' z adds; with
       // activation factors these differ from the fp32 products x * t
       float s1 = __half2float(hlo) + __half2float(hhi);
-      float s2 = ldexpf(__half2float(hlo), g.p[0]) + ldexpf(__half2float(hhi), g.p[1]);
+      float s2 = __half2float(hlo) * pow2i(g.p[0]) + __half2float(hhi) * pow2i(g.p[1]);
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) {
         s1 += __shfl_xor_sync(0xffffffffu, s1, o);
@@ -323,10 +338,10 @@ __device__ __forceinline__ void rec_store(const XIn& in, const GvBlock& B, int j
       if (lane == 0) {
         recf[PW + g.bb * NGM + g.c] = kMagicF * s1;
         recf[PW + NB * NGM + g.bb * NGM + g.c] = s2;
-        recf[PW + 2 * NB * NGM + g.bb * NGM + g.c] = ldexpf(1.f, e);
+        recf[PW + 2 * NB * NGM + g.bb * NGM + g.c] = pow2i(e);
       }
     } else if (g.jp == 0 && g.t == 0) {
-      recf[PW + 2 * NB * NGM + g.bb * NGM] = ldexpf(1.f, e);
+      recf[PW + 2 * NB * NGM + g.bb * NGM] = pow2i(e);
     }
   }
 }

@@ -32,8 +32,10 @@ def test_gemm_matches_oracle(polyq_lib, M, N, K, B, seed, forced):
     host = polyq_lib.HostLayer.pack(W, a, B, forced_bits=bits)
     dev = polyq_lib.DeviceLayer(host, "cuda")
     ref = O.pack_layer(W, a, B, bits=bits)
-    Y = polyq_lib.linear_gemm(dev, _x_dev(Xb))
+    ws = torch.zeros(polyq_lib.gemm_workspace_bytes(dev, M), dtype=torch.uint8, device="cuda")
+    Y = polyq_lib.linear_gemm(dev, _x_dev(Xb), workspace=ws)
     torch.cuda.synchronize()
+    assert polyq_lib.workspace_status(ws[-256:]) == 0  # no bounded wait gave up
     check_tolerance(Y.cpu().numpy(), O.linear(ref, X), X, K)
 
 
