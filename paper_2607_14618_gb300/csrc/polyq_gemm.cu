@@ -197,6 +197,7 @@ constexpr int kRowExp = 14;       // a row's largest magnitude becomes [2^14, 2^
 constexpr int kRowExpMin = -126;  // 2^e stays a normal float
 constexpr int kPrepThreads = 256;
 constexpr int kPrepMaxSmem = 200 * 1024;
+constexpr int kRowVec = 8;  // 16-byte pieces of a row a thread holds (rows up to 16384 wide)
 
 // Clustered K slot k of a row: the position p it takes its value from, or -1
 // past the end of a block.
@@ -237,8 +238,8 @@ __global__ void __launch_bounds__(kPrepThreads) gemm_prep(const __grid_constant_
   uint16_t* s_row = reinterpret_cast<uint16_t*>(psm + (size_t)Kp * 4 * (P.xscale ? 2 : 1));
   if (staged) {
     // static layer data, built before the wait for the previous kernel; a
-    // thread's loads of 8 slots are issued together
-    constexpr int U = 8;
+    // thread's loads of 16 slots are issued together
+    constexpr int U = 16;
     for (int k0 = threadIdx.x; k0 < Kp; k0 += kPrepThreads * U) {
       int pos[U], src[U];
       float fac[U];
@@ -289,6 +290,75 @@ __global__ void __launch_bounds__(kPrepThreads) gemm_prep(const __grid_constant_
     return __uint_as_float((uint32_t)b << 16) * f;
   };
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // Row scale of row m from its largest magnitude bits mx (fp32 bit pattern,
+  // per thread): e_m = floor(log2(max)) - kRowExp, an fp32 subnormal maximum
+  // counting as 2^-127.  2^e and 2^-e are normal floats (-126 <= e <= 113),
+  // so the products with 2^-e are exact scalings (rounded like any product
+  // where they fall below the normal range).  Returns 2^-e_m.
+  auto row_scale = [&](int m, uint32_t mx) -> float {
+    if (P.xscale) {
+      mx = 0;
+      for (int k = threadIdx.x; k < Kp; k += kPrepThreads)
+        mx = max(mx, __float_as_uint(fabsf(value(m, k))));
+    }
+    mx = __reduce_max_sync(0xffffffffu, mx);
+    if (lane == 0) s_wmax[warp] = mx;
+    __syncthreads();
+#pragma unroll
+    for (int w = 0; w < kPrepThreads / 32; ++w) mx = max(mx, s_wmax[w]);
+    const int e = mx ? max((int)(mx >> 23) - 127 - kRowExp, kRowExpMin) : 0;
+    if (threadIdx.x == 0) P.rowscale[m] = __int_as_float((127 + e) << 23);
+    return __int_as_float((127 - e) << 23);
+  };
+  const int n8 = P.K / 8;  // 16-byte pieces of a row
+  const bool vec = staged && (P.K & 7) == 0 && (reinterpret_cast<uintptr_t>(P.x) & 15) == 0 &&
+                   n8 <= kRowVec * kPrepThreads;
+  if (vec) {
+    // A thread holds its pieces of a row in registers: the next row's loads
+    // are issued before the current row is gathered, so they are in flight
+    // meanwhile.  Each thread writes 8 consecutive slots with one 16-byte
+    // store.
+    auto load_row = [&](int m, uint4 (&v)[kRowVec]) {
+      const uint4* row = reinterpret_cast<const uint4*>(P.x) + (size_t)m * n8;
+#pragma unroll
+      for (int u = 0; u < kRowVec; ++u) {
+        const int i = threadIdx.x + u * kPrepThreads;
+        v[u] = i < n8 ? __ldg(row + i) : make_uint4(0u, 0u, 0u, 0u);
+      }
+    };
+    uint4 v[kRowVec];
+    if ((int)blockIdx.x < P.M) load_row(blockIdx.x, v);
+    for (int m = blockIdx.x; m < P.M; m += gridDim.x) {
+      uint32_t mx = 0;
+#pragma unroll
+      for (int u = 0; u < kRowVec; ++u) {
+        const int i = threadIdx.x + u * kPrepThreads;
+        if (i < n8) {
+          reinterpret_cast<uint4*>(s_row)[i] = v[u];
+          const uint32_t w[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
+#pragma unroll
+          for (int q = 0; q < 4; ++q) mx = max(mx, max(w[q] & 0x7FFFu, (w[q] >> 16) & 0x7FFFu));
+        }
+      }
+      mx <<= 16;  // bf16 magnitude bits -> fp32 bits
+      __syncthreads();  // the staged row (and, on the first row, the map) is complete
+      const float inv = row_scale(m, mx);
+      if (m + (int)gridDim.x < P.M) load_row(m + gridDim.x, v);
+      uint4* dst = reinterpret_cast<uint4*>(P.xg + (size_t)m * Kp);
+      for (int i = threadIdx.x; i < Kp / 8; i += kPrepThreads) {
+        uint32_t w[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const __half2 h = __halves2half2(__float2half_rn(value(m, 8 * i + 2 * q) * inv),
+                                           __float2half_rn(value(m, 8 * i + 2 * q + 1) * inv));
+          w[q] = *reinterpret_cast<const uint32_t*>(&h);
+        }
+        dst[i] = make_uint4(w[0], w[1], w[2], w[3]);
+      }
+      __syncthreads();  // the row buffer and s_wmax are reused by the next row
+    }
+    return;
+  }
   for (int m = blockIdx.x; m < P.M; m += gridDim.x) {
     // largest magnitude of the row's values (bit patterns of non-negative
     // floats order as integers); without activation factors that is the
@@ -312,23 +382,11 @@ __global__ void __launch_bounds__(kPrepThreads) gemm_prep(const __grid_constant_
     }
     mx <<= 16;  // bf16 magnitude bits -> fp32 bits
     __syncthreads();  // the staged row (and, on the first row, the map) is complete
-    if (P.xscale) {
-      mx = 0;
-      for (int k = threadIdx.x; k < Kp; k += kPrepThreads)
-        mx = max(mx, __float_as_uint(fabsf(value(m, k))));
-    }
-    mx = __reduce_max_sync(0xffffffffu, mx);
-    if (lane == 0) s_wmax[warp] = mx;
-    __syncthreads();
-#pragma unroll
-    for (int w = 0; w < kPrepThreads / 32; ++w) mx = max(mx, s_wmax[w]);
-    // e_m = floor(log2(max)) - kRowExp (an fp32 subnormal maximum counts as 2^-127)
-    const int e = mx ? max((int)(mx >> 23) - 127 - kRowExp, kRowExpMin) : 0;
-    if (threadIdx.x == 0) P.rowscale[m] = ldexpf(1.f, e);
+    const float inv = row_scale(m, mx);
     __half2* dst = reinterpret_cast<__half2*>(P.xg) + (size_t)m * half;
     for (int i = threadIdx.x; i < half; i += kPrepThreads)
-      dst[i] = __halves2half2(__float2half_rn(ldexpf(value(m, 2 * i), -e)),
-                              __float2half_rn(ldexpf(value(m, 2 * i + 1), -e)));
+      dst[i] = __halves2half2(__float2half_rn(value(m, 2 * i) * inv),
+                              __float2half_rn(value(m, 2 * i + 1) * inv));
     __syncthreads();  // the row buffer and s_wmax are reused by the next row
   }
 }
@@ -897,14 +955,6 @@ extern "C" int polyq_linear_gemm(const polyq_dev_layer* L, const void* X, int64_
   cfg.numAttrs = 1;
   const size_t prep_smem = prep_smem_bytes(P.K, KT * BK, P.xscale != nullptr);
   P.prep_staged = prep_smem > 0;
-  {
-    // as many CTAs as fit at once, each taking rows m = b, b + grid, ...
-    const int by_smem = prep_smem ? std::max(1, (int)((228 * 1024) / (prep_smem + 2048))) : 8;
-    const int per_sm = std::min(8, by_smem);
-    cfg.gridDim = dim3((unsigned)std::min<long long>(M, (long long)sms * per_sm));
-  }
-  cfg.blockDim = dim3(kPrepThreads);
-  cfg.dynamicSmemBytes = prep_smem;
   static bool prep_attr_done[8] = {false};
   if (!prep_attr_done[dev & 7]) {
     cudaError_t ea = cudaFuncSetAttribute(gemm_prep, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -914,6 +964,20 @@ extern "C" int polyq_linear_gemm(const polyq_dev_layer* L, const void* X, int64_
                              cudaGetErrorString(ea));
     prep_attr_done[dev & 7] = true;
   }
+  {
+    // as many CTAs as are resident at once (registers and shared memory),
+    // each taking rows m = b, b + grid, ...
+    int per_sm = 0;
+    cudaError_t eo =
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, gemm_prep, kPrepThreads, prep_smem);
+    if (eo != cudaSuccess || per_sm < 1)
+      return polyq_set_error(POLYQ_ECUDA, "polyq_linear_gemm: prep occupancy: %s",
+                             cudaGetErrorString(eo));
+    per_sm = std::min(8, per_sm);
+    cfg.gridDim = dim3((unsigned)std::min<long long>(M, (long long)sms * per_sm));
+  }
+  cfg.blockDim = dim3(kPrepThreads);
+  cfg.dynamicSmemBytes = prep_smem;
   cudaError_t e = cudaLaunchKernelEx(&cfg, gemm_prep, P);
   if (e != cudaSuccess)
     return polyq_set_error(POLYQ_ECUDA, "polyq_linear_gemm: prep launch: %s", cudaGetErrorString(e));
