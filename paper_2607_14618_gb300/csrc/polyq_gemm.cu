@@ -316,8 +316,7 @@ __global__ void __launch_bounds__(kPrepThreads) gemm_prep(const __grid_constant_
   if (vec) {
     // A thread holds its pieces of a row in registers: the next row's loads
     // are issued before the current row is gathered, so they are in flight
-    // meanwhile.  Each thread writes 8 consecutive slots with one 16-byte
-    // store.
+    // meanwhile.
     auto load_row = [&](int m, uint4 (&v)[kRowVec]) {
       const uint4* row = reinterpret_cast<const uint4*>(P.x) + (size_t)m * n8;
 #pragma unroll
@@ -344,16 +343,18 @@ __global__ void __launch_bounds__(kPrepThreads) gemm_prep(const __grid_constant_
       __syncthreads();  // the staged row (and, on the first row, the map) is complete
       const float inv = row_scale(m, mx);
       if (m + (int)gridDim.x < P.M) load_row(m + gridDim.x, v);
-      uint4* dst = reinterpret_cast<uint4*>(P.xg + (size_t)m * Kp);
-      for (int i = threadIdx.x; i < Kp / 8; i += kPrepThreads) {
-        uint32_t w[4];
+      // four consecutive slots per thread and 8-byte store (with eight, the
+      // row reads of a warp's threads collide in shared-memory banks more)
+      uint2* dst = reinterpret_cast<uint2*>(P.xg + (size_t)m * Kp);
+      for (int i = threadIdx.x; i < Kp / 4; i += kPrepThreads) {
+        uint32_t w[2];
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          const __half2 h = __halves2half2(__float2half_rn(value(m, 8 * i + 2 * q) * inv),
-                                           __float2half_rn(value(m, 8 * i + 2 * q + 1) * inv));
+        for (int q = 0; q < 2; ++q) {
+          const __half2 h = __halves2half2(__float2half_rn(value(m, 4 * i + 2 * q) * inv),
+                                           __float2half_rn(value(m, 4 * i + 2 * q + 1) * inv));
           w[q] = *reinterpret_cast<const uint32_t*>(&h);
         }
-        dst[i] = make_uint4(w[0], w[1], w[2], w[3]);
+        dst[i] = make_uint2(w[0], w[1]);
       }
       __syncthreads();  // the row buffer and s_wmax are reused by the next row
     }
