@@ -188,10 +188,12 @@ __host__ __device__ inline int slot_code(int bits, int s) {
 // builds, in shared memory, the map from a clustered slot to the source
 // channel it reads (and its activation factor); then, one row at a time, it
 // copies the row of X into shared memory with 16-byte loads (finding the
-// row's largest magnitude on the way) and gathers from there.  Global reads
-// and writes are so coalesced whatever the permutation.  Layers too wide for
-// that (see prep_smem_bytes) gather from global memory instead.  Y is zeroed
-// when the K range is split over CTAs.
+// row's largest magnitude on the way) and gathers from there.  Rows up to
+// 16384 wide are held in registers, the next row's loads in flight while the
+// current row is gathered.  Global reads and writes are so coalesced whatever
+// the permutation.  Layers too wide for shared memory (see prep_smem_bytes)
+// gather from global memory instead.  Y is zeroed when the K range is split
+// over CTAs.
 // ---------------------------------------------------------------------------
 constexpr int kRowExp = 14;       // a row's largest magnitude becomes [2^14, 2^15)
 constexpr int kRowExpMin = -126;  // 2^e stays a normal float

@@ -7,11 +7,13 @@
 // (t = the Section 3.4 activation factors of a scaled layer, else 1.)
 //
 // Two kernels per call, chained with programmatic dependent launch:
-//  * gemv_prep, one CTA per (layer, step): gathers x through `gather`, scales
-//    each value by the power of two that the decoder leaves on its code,
-//    rounds it to fp16 and stores the step's activation record together with
-//    per-chunk sums for the magic-number and zero-point corrections.  The
-//    gather indices are loaded before the wait for the previous kernel.
+//  * gemv_prep, one 256-thread CTA per (layer, step) and a few more CTAs
+//    that set y to the residual (or zero): gathers x through `gather`,
+//    scales each value by the power of two that the decoder leaves on its
+//    code (and by its chunk's exponent), rounds it to fp16 and stores the
+//    step's activation record together with per-chunk sums for the
+//    magic-number and zero-point corrections.  The gather indices are loaded
+//    before the wait for the previous kernel.
 //  * gemv_main, persistent, 160 threads per CTA, 3 CTAs per SM.  The (layer,
 //    64-row tile, step) work items of all layers of the call form one list;
 //    each CTA takes a contiguous range of it.  Warp 4 (one thread) streams
