@@ -24,6 +24,7 @@ def _x_dev(xb):
     (96, 96, 640, 2.0, 57, False),       # all 2-bit
     (300, 520, 2100, 3.0, 60, True),     # stream-K: ~3 K tiles per CTA, cut across tiles
     (64, 2000, 4000, 3.0, 61, False),    # uniform K split into 8 ranges
+    (2000, 320, 1600, 3.0, 62, True),    # more rows than pre-pass CTAs (rows held in registers)
 ])
 def test_gemm_matches_oracle(polyq_lib, M, N, K, B, seed, forced):
     W, a = synth.layer_weights(N, K, seed)

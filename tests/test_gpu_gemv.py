@@ -116,6 +116,24 @@ def test_gemv_full_size_sampled_rows(polyq_lib, name, N, K, B, batch):
 
 
 @pytest.mark.parametrize("batch", [1, 4])
+def test_gemv_residual_not_16_byte_aligned(polyq_lib, batch):
+    """The outputs are set to the residual by CTAs of the pre-pass with
+    16-byte loads and stores where the pointers allow; a residual at a 4-byte
+    offset takes the scalar path."""
+    N, K = 200, 1024
+    W, a = synth.layer_weights(N, K, 37)
+    host = polyq_lib.HostLayer.pack(W, a, 3.0)
+    dev = polyq_lib.DeviceLayer(host, "cuda")
+    ref = O.pack_layer(W, a, 3.0)
+    xb, x = synth.activations(a, batch, 37)
+    res = torch.randn(batch * N + 1, device="cuda")[1:].view(batch, N)
+    assert res.data_ptr() % 16 != 0
+    y = polyq_lib.linear_gemv(dev, _x_dev(xb), residual=res)
+    torch.cuda.synchronize()
+    check_tolerance(y.cpu().numpy(), O.linear(ref, x) + res.cpu().numpy().astype(np.float64), x, K)
+
+
+@pytest.mark.parametrize("batch", [1, 4])
 def test_gemv_group_matches_oracle(polyq_lib, batch):
     """Several layers in one launch (q/k/v-like: shared input, own widths and
     gathers; plus a layer of another shape and forced widths)."""

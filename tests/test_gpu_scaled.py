@@ -91,6 +91,7 @@ def test_scaled_gemv_with_fused_rmsnorm(polyq_lib):
 @pytest.mark.parametrize("M,N,K,seed,forced", [
     (256, 256, 1100, 61, True),
     (512, 640, 2048, 62, False),
+    (2000, 320, 2048, 63, True),  # more rows than pre-pass CTAs: the next row loads while one is gathered
 ])
 def test_scaled_gemm_matches_oracle(polyq_lib, M, N, K, seed, forced):
     W, a = synth.layer_weights(N, K, seed)
