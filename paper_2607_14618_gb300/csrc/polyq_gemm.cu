@@ -169,6 +169,32 @@ __device__ __forceinline__ int find_kblock(const GmBlock* blk, int nblk, int kt)
   return b;
 }
 
+// The block of the current K tile with its fields in registers.  K tiles
+// only increase within a piece, so after a seek at the piece's first tile the
+// cursor advances with one comparison per tile instead of a search through
+// the block table in shared memory.
+struct BlockCursor {
+  int bi, kt0, next_kt0, bits, seg_off, grp_off;
+  __device__ __forceinline__ void load(const GmBlock* sblk, int nblk) {
+    const GmBlock& B = sblk[bi];
+    kt0 = B.kt0;
+    bits = B.bits;
+    seg_off = B.seg_off;
+    grp_off = B.grp_off;
+    next_kt0 = bi + 1 < nblk ? sblk[bi + 1].kt0 : 0x7FFFFFFF;
+  }
+  __device__ __forceinline__ void seek(const GmBlock* sblk, int nblk, int kt) {
+    bi = find_kblock(sblk, nblk, kt);
+    load(sblk, nblk);
+  }
+  __device__ __forceinline__ void advance(const GmBlock* sblk, int nblk, int kt) {
+    while (kt >= next_kt0) {
+      ++bi;
+      load(sblk, nblk);
+    }
+  }
+};
+
 // Position inside a 32-code half group of the code that fills K slot `s`
 // (0..31) of a tile (the order in which the dequantiser emits its fp16 pairs).
 __host__ __device__ inline int slot_code(int bits, int s) {
@@ -564,14 +590,16 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
       Pieces pc;
       pc.init(P);
       int um, un, kt_lo, kt_hi;
+      BlockCursor B;
       while (!s_abort && pc.next(P, um, un, kt_lo, kt_hi)) {
+        B.seek(sblk, nblk, kt_lo);
         for (int kt = kt_lo; kt < kt_hi && !s_abort; ++kt, ++kg) {
           const int s = kg % kStagesG, use = kg / kStagesG;
           if (use > 0 && !mbar_wait_sleep(smem_u32(&bar_sfree[s]), (use - 1) & 1)) {
             fail(kStatusTimeoutEmpty);
             break;
           }
-          const GmBlock& B = sblk[find_kblock(sblk, nblk, kt)];
+          B.advance(sblk, nblk, kt);
           const int hg = kt - B.kt0;  // half group
           uint8_t* st = stage_ptr(s);
           const uint32_t bar = smem_u32(&bar_full[s]);
@@ -643,16 +671,20 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
     Pieces pc;
     pc.init(P);
     int um, un, kt_lo, kt_hi;
+    BlockCursor B;
     for (; !s_abort && pc.next(P, um, un, kt_lo, kt_hi); ++uc) {
+      B.seek(sblk, nblk, kt_lo);
       for (int kt = kt_lo; kt < kt_hi && !s_abort; ++kt, ++kg) {
         if ((kg & 1) != grp) continue;
         const int s = kg % kStagesG, use = kg / kStagesG;
-        if (!mbar_wait(smem_u32(&bar_full[s]), use & 1) ||
-            (use > 0 && !mbar_wait(smem_u32(&bar_sfree[s]), (use - 1) & 1))) {
+        // The producer issues a slot's copies only after the MMAs of its
+        // previous use are done, so once they have landed the weight tile
+        // may be overwritten too.
+        if (!mbar_wait(smem_u32(&bar_full[s]), use & 1)) {
           fail(kStatusTimeoutFull);
           break;
         }
-        const GmBlock& B = sblk[find_kblock(sblk, nblk, kt)];
+        B.advance(sblk, nblk, kt);
         if (B.bits != 16) {
           const int hg = kt - B.kt0;
           uint8_t* st = stage_ptr(s);
@@ -694,7 +726,7 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
                 st + MT * kATile + kBTile + kCodes)[r * 4 + mslot];
             dequant_row(B.bits, w, meta, st + MT * kATile, r);
 #ifdef POLYQ_DEBUG
-            dbg_row(st + MT * kATile, r, un * BN + r, P.N, B, hg);
+            dbg_row(st + MT * kATile, r, un * BN + r, P.N, sblk[B.bi], hg);
 #endif
           }
           fence_proxy_async_smem();
@@ -702,8 +734,8 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
 #ifdef POLYQ_DEBUG
         else {
           for (int h = 0; h < 2; ++h)
-            dbg_row(stage_ptr(s) + MT * kATile, r0 + 128 * h, un * BN + r0 + 128 * h, P.N, B,
-                    kt - B.kt0);
+            dbg_row(stage_ptr(s) + MT * kATile, r0 + 128 * h, un * BN + r0 + 128 * h, P.N,
+                    sblk[B.bi], kt - B.kt0);
         }
 #endif
         __syncwarp();
