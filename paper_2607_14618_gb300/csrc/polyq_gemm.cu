@@ -54,9 +54,10 @@ constexpr int MT = 2;             // M tiles per work unit (share one weight til
 constexpr int BN = 256;           // weight rows per work unit
 constexpr int BK = 32;            // K per tile: half a quantisation group
 constexpr int kStagesG = 4;
-constexpr int kCodeBox = 48;      // code bytes per row loaded per tile: an odd
-                                  // number of 16-byte chunks keeps row reads
-                                  // conflict-free; covers offset (<= 12) + 32
+constexpr int kCodeBox = 32;      // code bytes per row loaded per tile: the tile's codes from a
+                                  // 16-byte aligned start (offset <= 12 with at most 16 bytes of
+                                  // codes, or 32 bytes of 8-bit codes at offset 0), one TMA
+                                  // row request each (48-byte rows take two)
 constexpr int kATile = BM * BK * 2;             // 8 KB (64-byte rows)
 constexpr int kBTile = BN * BK * 2;             // 16 KB
 constexpr int kCodes = BN * kCodeBox;           // 12 KB
