@@ -25,7 +25,7 @@
 //                   2-5 take the even stages and 6-9 the odd ones, two weight
 //                   rows per thread; afterwards all eight drain the
 //                   accumulator with tcgen05.ld and store fp32 Y.
-//     Four pipeline stages.  When the (M, N) tiles cannot fill the GPU the K
+//     Five pipeline stages.  When the (M, N) tiles cannot fill the GPU the K
 //     range is split, uniformly or stream-K (each CTA an equal contiguous
 //     share of all (tile, K tile) pairs), and the pieces are added into a
 //     zeroed Y (so the order of those additions varies); otherwise Y is
@@ -53,16 +53,16 @@ constexpr int BM = 128;           // rows per MMA
 constexpr int MT = 2;             // M tiles per work unit (share one weight tile)
 constexpr int BN = 256;           // weight rows per work unit
 constexpr int BK = 32;            // K per tile: half a quantisation group
-constexpr int kStagesG = 4;
+constexpr int kStagesG = 5;
 constexpr int kCodeBox = 32;      // code bytes per row loaded per tile: the tile's codes from a
                                   // 16-byte aligned start (offset <= 12 with at most 16 bytes of
                                   // codes, or 32 bytes of 8-bit codes at offset 0), one TMA
                                   // row request each (48-byte rows take two)
 constexpr int kATile = BM * BK * 2;             // 8 KB (64-byte rows)
 constexpr int kBTile = BN * BK * 2;             // 16 KB
-constexpr int kCodes = BN * kCodeBox;           // 12 KB
+constexpr int kCodes = BN * kCodeBox;           // 8 KB
 constexpr int kMeta = BN * 16;                  // 4 KB
-constexpr int kStageG = MT * kATile + kBTile + kCodes + kMeta;  // 48 KB
+constexpr int kStageG = MT * kATile + kBTile + kCodes + kMeta;  // 44 KB
 constexpr int kThreadsG = 320;
 constexpr int kDqWarps = 8;
 constexpr double kUnitCostTiles = 12.0;  // per-piece overhead, in K-tile stages, of the split model
