@@ -18,13 +18,16 @@
 //                   bytes and meta of 256 weight rows, or for 16-bit blocks the
 //                   fp16 weights straight into the operand buffer;
 //       warp 1      allocates 512 TMEM columns and issues tcgen05.mma
-//                   (M=128, N=256, K=16, fp16 in, fp32 accumulate), two
-//                   M tiles per weight tile;
+//                   (M=128, N=256, K=16, fp16 in, fp32 accumulate): the
+//                   weights are the A operand, 128 rows per MMA, and the
+//                   256 tokens of an M pair the B operand, so a TMEM lane
+//                   holds one output column;
 //       warps 2..9  dequantise: (q - z) * s in fp16 via magic-number decode,
 //                   written in the UMMA 64-byte-swizzle K-major layout.  Warps
 //                   2-5 take the even stages and 6-9 the odd ones, two weight
 //                   rows per thread; afterwards all eight drain the
-//                   accumulator with tcgen05.ld and store fp32 Y.
+//                   accumulator with tcgen05.ld and store fp32 Y, each warp
+//                   store covering 32 consecutive columns of one row.
 //     Five pipeline stages.  When the (M, N) tiles cannot fill the GPU the K
 //     range is split, uniformly or stream-K (each CTA an equal contiguous
 //     share of all (tile, K tile) pairs), and the pieces are added into a
@@ -432,10 +435,8 @@ __device__ __forceinline__ void store_pairs_sw64(uint8_t* btile, int r, int chun
   *reinterpret_cast<uint4*>(dst) = make_uint4(p[0], p[1], p[2], p[3]);
 }
 
-__device__ __forceinline__ void red_add_v4(float* p, float a, float b, float c, float d) {
-  asm volatile("red.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(p), "f"(a), "f"(b), "f"(c),
-               "f"(d)
-               : "memory");
+__device__ __forceinline__ void red_add_f32(float* p, float a) {
+  asm volatile("red.global.add.f32 [%0], %1;" ::"l"(p), "f"(a) : "memory");
 }
 
 __device__ __forceinline__ uint32_t dq_pair(uint32_t raw, __half2 zz, __half2 ss) {
@@ -643,13 +644,16 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
           }
           tc_fence_after();
           uint8_t* st = stage_ptr(s);
-          const uint32_t b0 = smem_u32(st + MT * kATile);
+          // A: 128 of the tile's 256 weight rows; B: all 256 tokens of the M
+          // pair (one 256-row box).  Accumulator t holds weight rows 128 t..
+          // in its TMEM lanes and the tokens in its 256 columns.
+          const uint32_t x0 = smem_u32(st);
 #pragma unroll
           for (int t = 0; t < MT; ++t) {
-            const uint32_t a0 = smem_u32(st + t * kATile);
+            const uint32_t w0 = smem_u32(st + MT * kATile + t * (BM * BK * 2));
 #pragma unroll
             for (int kk = 0; kk < BK / 16; ++kk)
-              tc_mma_f16(tmem + t * BN, umma_desc_sw64(a0 + 32 * kk), umma_desc_sw64(b0 + 32 * kk),
+              tc_mma_f16(tmem + t * BN, umma_desc_sw64(w0 + 32 * kk), umma_desc_sw64(x0 + 32 * kk),
                          kIdesc, (kt > kt_lo || kk > 0) ? 1u : 0u);
           }
           tc_commit(smem_u32(&bar_sfree[s]));
@@ -743,48 +747,45 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
         if (lane == 0) mbar_arrive(smem_u32(&bar_bready[s]));
       }
       if (s_abort) break;
-      // epilogue: rows 32q + lane of each M tile, columns [128 half, +128)
+      // epilogue: lane i of a warp owns output column n = weight row
+      // 128 t + 32 q + i of the tile, and each TMEM column one token of the
+      // M pair, so every store of a warp writes 32 consecutive floats of one
+      // row of Y.  Tokens [128 half, +128) of the pair, 32 at a time.
       if (!mbar_wait(smem_u32(&bar_accf), uc & 1)) {
         fail(kStatusTimeoutFull);
         break;
       }
       tc_fence_after();
+      const bool add = P.ksplit > 1 || P.streamk;  // Y was zeroed by the pre-pass
+#pragma unroll 1
+      for (int c4 = 0; c4 < 4; ++c4) {
+        const int col = 128 * half + 32 * c4;
+        const int m0 = um * (MT * BM) + col;
+        const int jn = min(32, P.M - m0);  // tokens of this chunk inside M
+        if (jn <= 0) break;
+        // 2^e_m of the pre-pass, one token per lane, broadcast below
+        const float rs_l = lane < jn ? P.rowscale[m0 + lane] : 0.f;
+        float rs[32];
 #pragma unroll
-      for (int t = 0; t < MT; ++t) {
-        const int m = um * (MT * BM) + t * BM + 32 * q + lane;
-        const float rs = m < P.M ? P.rowscale[m] : 0.f;  // 2^e_m of the pre-pass
+        for (int j = 0; j < 32; ++j) rs[j] = __shfl_sync(0xffffffffu, rs_l, j);
 #pragma unroll
-        for (int c4 = 0; c4 < 4; ++c4) {
-          const int col = 128 * half + 32 * c4;
+        for (int t = 0; t < MT; ++t) {
           uint32_t v[32];
           tc_ld_32x32b_x32(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(t * BN + col), v);
           tc_wait_ld();
-          float f[32];
+          const int n = un * BN + t * BM + 32 * q + lane;
+          if (n < P.N) {
+            float* dst = P.y + (size_t)m0 * P.N + n;
 #pragma unroll
-          for (int j = 0; j < 32; ++j) f[j] = __uint_as_float(v[j]) * rs;
-          const int n0 = un * BN + col;
-          if (m < P.M) {
-            float* dst = P.y + (size_t)m * P.N + n0;
-            const bool vec = n0 + 32 <= P.N && (P.N % 4) == 0;
-            if (P.ksplit > 1 || P.streamk) {  // Y was zeroed by the pre-pass: add this K range
-              if (vec) {
-#pragma unroll
-                for (int j = 0; j < 8; ++j)
-                  red_add_v4(dst + 4 * j, f[4 * j], f[4 * j + 1], f[4 * j + 2], f[4 * j + 3]);
-              } else {
-#pragma unroll
-                for (int j = 0; j < 32; ++j)
-                  if (n0 + j < P.N) atomicAdd(dst + j, f[j]);
+            for (int j = 0; j < 32; ++j) {
+              if (j < jn) {
+                const float f = __uint_as_float(v[j]) * rs[j];
+                if (add)
+                  red_add_f32(dst, f);
+                else
+                  *dst = f;
               }
-            } else if (vec) {
-#pragma unroll
-              for (int j = 0; j < 8; ++j)
-                reinterpret_cast<float4*>(dst)[j] =
-                    make_float4(f[4 * j], f[4 * j + 1], f[4 * j + 2], f[4 * j + 3]);
-            } else {
-#pragma unroll
-              for (int j = 0; j < 32; ++j)
-                if (n0 + j < P.N) dst[j] = f[j];
+              dst += P.N;
             }
           }
         }
@@ -887,7 +888,7 @@ extern "C" int polyq_linear_gemm(const polyq_dev_layer* L, const void* X, int64_
   int rc = polyq_check_dev_layer(L, "polyq_linear_gemm");
   if (rc) return rc;
   if (!X || !Y) return polyq_set_error(POLYQ_EINVAL, "polyq_linear_gemm: X or Y is NULL");
-  if ((uintptr_t)Y % 16)  // Y is written (and zeroed for split K) with 16-byte stores
+  if ((uintptr_t)Y % 16)  // Y is zeroed for split K with 16-byte stores
     return polyq_set_error(POLYQ_EINVAL, "polyq_linear_gemm: Y must be 16-byte aligned");
   if (M < 1 || M > (1 << 24))
     return polyq_set_error(POLYQ_EINVAL, "polyq_linear_gemm: M=%lld", (long long)M);
