@@ -750,44 +750,51 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
       // epilogue: lane i of a warp owns output column n = weight row
       // 128 t + 32 q + i of the tile, and each TMEM column one token of the
       // M pair, so every store of a warp writes 32 consecutive floats of one
-      // row of Y.  Tokens [128 half, +128) of the pair, 32 at a time.
+      // row of Y.  Tokens [128 half, +128) of the pair, 32 at a time.  The
+      // 2^e_m of the pre-pass (one token per lane, broadcast by shuffles) are
+      // loaded together, and both accumulators' TMEM loads of a chunk share
+      // one wait.  (The loads follow the accumulator's barrier, which orders
+      // them after the pre-pass even for a warp that took no stage.)
       if (!mbar_wait(smem_u32(&bar_accf), uc & 1)) {
         fail(kStatusTimeoutFull);
         break;
       }
       tc_fence_after();
+      const int mh = um * (MT * BM) + 128 * half;
+      float rs_l[4];
+#pragma unroll
+      for (int c4 = 0; c4 < 4; ++c4)
+        rs_l[c4] = mh + 32 * c4 + lane < P.M ? P.rowscale[mh + 32 * c4 + lane] : 0.f;
       const bool add = P.ksplit > 1 || P.streamk;  // Y was zeroed by the pre-pass
-#pragma unroll 1
+      const int n0 = un * BN + 32 * q + lane;       // + BM for the second accumulator
+#pragma unroll
       for (int c4 = 0; c4 < 4; ++c4) {
-        const int col = 128 * half + 32 * c4;
-        const int m0 = um * (MT * BM) + col;
+        const int m0 = mh + 32 * c4;
         const int jn = min(32, P.M - m0);  // tokens of this chunk inside M
         if (jn <= 0) break;
-        // 2^e_m of the pre-pass, one token per lane, broadcast below
-        const float rs_l = lane < jn ? P.rowscale[m0 + lane] : 0.f;
-        float rs[32];
+        uint32_t v0[32], v1[32];
+        const uint32_t ta = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(128 * half + 32 * c4);
+        tc_ld_32x32b_x32(ta, v0);
+        tc_ld_32x32b_x32(ta + BN, v1);
+        tc_wait_ld();
+        tc_regs_ready(v0);
+        tc_regs_ready(v1);
+        float* dst = P.y + (size_t)m0 * P.N + n0;
+        const bool ok0 = n0 < P.N, ok1 = n0 + BM < P.N;
 #pragma unroll
-        for (int j = 0; j < 32; ++j) rs[j] = __shfl_sync(0xffffffffu, rs_l, j);
-#pragma unroll
-        for (int t = 0; t < MT; ++t) {
-          uint32_t v[32];
-          tc_ld_32x32b_x32(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(t * BN + col), v);
-          tc_wait_ld();
-          const int n = un * BN + t * BM + 32 * q + lane;
-          if (n < P.N) {
-            float* dst = P.y + (size_t)m0 * P.N + n;
-#pragma unroll
-            for (int j = 0; j < 32; ++j) {
-              if (j < jn) {
-                const float f = __uint_as_float(v[j]) * rs[j];
-                if (add)
-                  red_add_f32(dst, f);
-                else
-                  *dst = f;
-              }
-              dst += P.N;
+        for (int j = 0; j < 32; ++j) {
+          const float rs = __shfl_sync(0xffffffffu, rs_l[c4], j);
+          if (j < jn) {
+            const float f0 = __uint_as_float(v0[j]) * rs, f1 = __uint_as_float(v1[j]) * rs;
+            if (add) {
+              if (ok0) red_add_f32(dst, f0);
+              if (ok1) red_add_f32(dst + BM, f1);
+            } else {
+              if (ok0) dst[0] = f0;
+              if (ok1) dst[BM] = f1;
             }
           }
+          dst += P.N;
         }
       }
       tc_fence_before();
