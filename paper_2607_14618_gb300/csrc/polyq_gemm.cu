@@ -625,7 +625,10 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
   } else if (warp == 1) {
     // ---------------- MMA issuer ----------------
     if (lane == 0) {
-      int kg = 0, uc = 0;
+      int uc = 0, s = 0;
+      uint32_t ph = 0;
+      const uint64_t dx0 = umma_desc_sw64(smem_u32(smem));
+      const uint64_t dw0 = umma_desc_sw64(smem_u32(smem + MT * kATile));
       Pieces pc;
       pc.init(P);
       int um, un, kt_lo, kt_hi;
@@ -635,28 +638,32 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
           break;
         }
         tc_fence_after();
-        for (int kt = kt_lo; kt < kt_hi && !s_abort; ++kt, ++kg) {
-          const int s = kg % kStagesG, use = kg / kStagesG;
-          if (!mbar_wait_sleep(smem_u32(&bar_full[s]), use & 1) ||
-              !mbar_wait_sleep(smem_u32(&bar_bready[s]), use & 1)) {
+        for (int kt = kt_lo; kt < kt_hi && !s_abort; ++kt) {
+          // Every dequantiser warp of the stage's group waits for the
+          // stage's copies (bar_full) before it arrives on bar_bready, so
+          // bar_bready alone orders the MMAs after the X tile and the weights.
+          if (!mbar_wait_sleep(smem_u32(&bar_bready[s]), ph)) {
             fail(kStatusTimeoutFull);
             break;
           }
           tc_fence_after();
-          uint8_t* st = stage_ptr(s);
           // A: 128 of the tile's 256 weight rows; B: all 256 tokens of the M
           // pair (one 256-row box).  Accumulator t holds weight rows 128 t..
-          // in its TMEM lanes and the tokens in its 256 columns.
-          const uint32_t x0 = smem_u32(st);
+          // in its TMEM lanes and the tokens in its 256 columns.  The slot's
+          // descriptors are those of slot 0 plus its offset (address >> 4).
+          const uint64_t so = (uint64_t)((s * kStageG) >> 4);
+          const uint64_t dx = dx0 + so, dw = dw0 + so;
 #pragma unroll
-          for (int t = 0; t < MT; ++t) {
-            const uint32_t w0 = smem_u32(st + MT * kATile + t * (BM * BK * 2));
+          for (int t = 0; t < MT; ++t)
 #pragma unroll
             for (int kk = 0; kk < BK / 16; ++kk)
-              tc_mma_f16(tmem + t * BN, umma_desc_sw64(w0 + 32 * kk), umma_desc_sw64(x0 + 32 * kk),
+              tc_mma_f16(tmem + t * BN, dw + (uint64_t)((t * BM * BK * 2) >> 4) + 2 * kk, dx + 2 * kk,
                          kIdesc, (kt > kt_lo || kk > 0) ? 1u : 0u);
-          }
           tc_commit(smem_u32(&bar_sfree[s]));
+          if (++s == kStagesG) {
+            s = 0;
+            ph ^= 1u;
+          }
         }
         tc_commit(smem_u32(&bar_accf));
       }
