@@ -114,16 +114,30 @@ __device__ __forceinline__ bool mbar_try_wait_hint(uint32_t bar, uint32_t parity
   return ok != 0;
 }
 
-// Bounded wait for the lone producer and MMA threads: each poll may sleep up
-// to 1 us, so that their polling does not take issue slots from the
-// dequantisation warps that share their schedulers.  At most 2^22 polls, a
-// few seconds.
+// Bounded waits that also give up once another role of the CTA has failed:
+// 0 when the phase completed, 1 on a timeout, 2 when `abort` was raised.  The
+// flag is read only after a poll has failed, so that a stage whose barrier
+// has already completed costs one poll and no shared load.  The lone producer
+// and MMA threads poll with a suspend hint of up to 1 us, so that their
+// polling does not take issue slots from the dequantisation warps that share
+// their schedulers: at most 2^22 such polls, a few seconds.
 constexpr uint32_t kWaitLimitSleep = 1u << 22;
 constexpr uint32_t kSuspendHintNs = 1000;
-__device__ __forceinline__ bool mbar_wait_sleep(uint32_t bar, uint32_t parity) {
-  for (uint32_t it = 0; it < kWaitLimitSleep; ++it)
-    if (mbar_try_wait_hint(bar, parity, kSuspendHintNs)) return true;
-  return false;
+constexpr int kWaitOk = 0, kWaitTimeout = 1, kWaitAborted = 2;
+__device__ __forceinline__ int wait_ab(uint32_t bar, uint32_t parity, const volatile int* abort) {
+  for (uint32_t it = 0; it < kWaitLimit; ++it) {
+    if (mbar_try_wait(bar, parity)) return kWaitOk;
+    if (*abort) return kWaitAborted;
+  }
+  return kWaitTimeout;
+}
+__device__ __forceinline__ int wait_sleep_ab(uint32_t bar, uint32_t parity,
+                                             const volatile int* abort) {
+  for (uint32_t it = 0; it < kWaitLimitSleep; ++it) {
+    if (mbar_try_wait_hint(bar, parity, kSuspendHintNs)) return kWaitOk;
+    if (*abort) return kWaitAborted;
+  }
+  return kWaitTimeout;
 }
 
 // The pieces of work a CTA takes, in order: an output tile (um, un) and a
@@ -595,11 +609,14 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
       BlockCursor B;
       while (!s_abort && pc.next(P, um, un, kt_lo, kt_hi)) {
         B.seek(sblk, nblk, kt_lo);
-        for (int kt = kt_lo; kt < kt_hi && !s_abort; ++kt, ++kg) {
+        for (int kt = kt_lo; kt < kt_hi; ++kt, ++kg) {
           const int s = kg % kStagesG, use = kg / kStagesG;
-          if (use > 0 && !mbar_wait_sleep(smem_u32(&bar_sfree[s]), (use - 1) & 1)) {
-            fail(kStatusTimeoutEmpty);
-            break;
+          if (use > 0) {
+            const int w = wait_sleep_ab(smem_u32(&bar_sfree[s]), (use - 1) & 1, &s_abort);
+            if (w != kWaitOk) {
+              if (w == kWaitTimeout) fail(kStatusTimeoutEmpty);
+              break;
+            }
           }
           B.advance(sblk, nblk, kt);
           const int hg = kt - B.kt0;  // half group
@@ -633,17 +650,21 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
       pc.init(P);
       int um, un, kt_lo, kt_hi;
       for (; !s_abort && pc.next(P, um, un, kt_lo, kt_hi); ++uc) {
-        if (uc > 0 && !mbar_wait_sleep(smem_u32(&bar_acce), (uc - 1) & 1)) {
-          fail(kStatusTimeoutEmpty);
-          break;
+        if (uc > 0) {
+          const int w = wait_sleep_ab(smem_u32(&bar_acce), (uc - 1) & 1, &s_abort);
+          if (w != kWaitOk) {
+            if (w == kWaitTimeout) fail(kStatusTimeoutEmpty);
+            break;
+          }
         }
         tc_fence_after();
-        for (int kt = kt_lo; kt < kt_hi && !s_abort; ++kt) {
+        for (int kt = kt_lo; kt < kt_hi; ++kt) {
           // Every dequantiser warp of the stage's group waits for the
           // stage's copies (bar_full) before it arrives on bar_bready, so
           // bar_bready alone orders the MMAs after the X tile and the weights.
-          if (!mbar_wait_sleep(smem_u32(&bar_bready[s]), ph)) {
-            fail(kStatusTimeoutFull);
+          const int w = wait_sleep_ab(smem_u32(&bar_bready[s]), ph, &s_abort);
+          if (w != kWaitOk) {
+            if (w == kWaitTimeout) fail(kStatusTimeoutFull);
             break;
           }
           tc_fence_after();
@@ -686,14 +707,15 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
     BlockCursor B;
     for (; !s_abort && pc.next(P, um, un, kt_lo, kt_hi); ++uc) {
       B.seek(sblk, nblk, kt_lo);
-      for (int kt = kt_lo; kt < kt_hi && !s_abort; ++kt, ++kg) {
+      for (int kt = kt_lo; kt < kt_hi; ++kt, ++kg) {
         if ((kg & 1) != grp) continue;
         const int s = kg % kStagesG, use = kg / kStagesG;
         // The producer issues a slot's copies only after the MMAs of its
         // previous use are done, so once they have landed the weight tile
         // may be overwritten too.
-        if (!mbar_wait(smem_u32(&bar_full[s]), use & 1)) {
-          fail(kStatusTimeoutFull);
+        const int w = wait_ab(smem_u32(&bar_full[s]), use & 1, &s_abort);
+        if (w != kWaitOk) {
+          if (w == kWaitTimeout) fail(kStatusTimeoutFull);
           break;
         }
         B.advance(sblk, nblk, kt);
@@ -762,9 +784,12 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
       // loaded together, and both accumulators' TMEM loads of a chunk share
       // one wait.  (The loads follow the accumulator's barrier, which orders
       // them after the pre-pass even for a warp that took no stage.)
-      if (!mbar_wait(smem_u32(&bar_accf), uc & 1)) {
-        fail(kStatusTimeoutFull);
-        break;
+      {
+        const int w = wait_ab(smem_u32(&bar_accf), uc & 1, &s_abort);
+        if (w != kWaitOk) {
+          if (w == kWaitTimeout) fail(kStatusTimeoutFull);
+          break;
+        }
       }
       tc_fence_after();
       const int mh = um * (MT * BM) + 128 * half;
