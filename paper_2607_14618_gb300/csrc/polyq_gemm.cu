@@ -6,15 +6,18 @@
 // The contraction runs over 32-wide K tiles (half a quantisation group); every
 // tile lies inside one bit block (Section 4.2) and one group, so each weight
 // row of a tile has one (scale, zero).
-//  1. gemm_prep gathers X through `gather` into a clustered fp16 matrix
-//     Xg[M][KT*32] (workspace), zero-padded at block ends, with the K order
-//     inside each tile permuted the same way the dequantiser emits codes.
+//  1. gemm_prep gathers X through `gather` into a clustered fp16 matrix Xg
+//     (workspace), zero-padded at block ends, with the K order inside each
+//     tile permuted the same way the dequantiser emits codes.  Xg is stored
+//     as the shared-memory images of the producer's copies: one 16 KB block
+//     per (pair of M tiles, K tile), 256 rows of 64 bytes in the 64-byte
+//     swizzle, so that one contiguous bulk copy fetches a stage's X.
 //     Each row m is scaled by the power of two 2^-e_m that brings its largest
 //     |x * t| into [2^14, 2^15), so that any finite bf16 row rounds to fp16
 //     without overflow and without dropping small values into subnormals;
 //     the epilogue multiplies row m of Y by 2^e_m.
 //  2. gemm_main: one persistent CTA per SM, 10 warps.
-//       warp 0      TMA producer: Xg tiles (64-byte swizzle), packed code
+//       warp 0      TMA producer: Xg blocks (bulk copies), packed code
 //                   bytes and meta of 256 weight rows, or for 16-bit blocks the
 //                   fp16 weights straight into the operand buffer;
 //       warp 1      allocates 512 TMEM columns and issues tcgen05.mma
@@ -80,7 +83,6 @@ struct GmBlock {
 };
 
 struct GmParams {
-  CUtensorMap tm_x;      // Xg [M][KT*32] fp16, box {32, 256} (both M tiles), 64B swizzle
   CUtensorMap tm_codes;  // packed [N][S] u8, box {48, 256}
   CUtensorMap tm_meta;   // meta [N][meta_stride] u32, box {4, 256}
   CUtensorMap tm_w16;    // packed [N][S/2] u16, box {32, 256}, 64B swizzle
@@ -226,7 +228,7 @@ __host__ __device__ inline int slot_code(int bits, int s) {
 }
 
 // ---------------------------------------------------------------------------
-// pre-pass: Xg[m][kt*32 + s] = fp16(X[m][gather[p]] * xscale[p] * 2^-e_m) with
+// pre-pass: Xg(m, kt*32 + s) = fp16(X[m][gather[p]] * xscale[p] * 2^-e_m) with
 // p = pos0 + 32 h + slot_code(s)
 // for the h-th 32-code half group of the block (tile kt).  Each CTA first
 // builds, in shared memory, the map from a clustered slot to the source
@@ -244,6 +246,15 @@ constexpr int kRowExpMin = -126;  // 2^e stays a normal float
 constexpr int kPrepThreads = 256;
 constexpr int kPrepMaxSmem = 200 * 1024;
 constexpr int kRowVec = 8;  // 16-byte pieces of a row a thread holds (rows up to 16384 wide)
+
+// Element offset of Xg(m, k) in the blocked layout: block (m / 256, k / 32)
+// of 256 rows x 32 fp16, row m % 256 at 64 bytes each, its 16-byte chunks
+// in the 64-byte swizzle (chunk index XOR bits 7..8 of the byte address).
+__device__ __forceinline__ size_t xg_off(int m, int k, int KT) {
+  const int r = m & (MT * BM - 1), c = (k >> 3) & 3;
+  return (((size_t)(m / (MT * BM)) * KT + (k >> 5)) * (MT * BM) + r) * BK +
+         ((c ^ ((r >> 1) & 3)) << 3) + (k & 7);
+}
 
 // Clustered K slot k of a row: the position p it takes its value from, or -1
 // past the end of a block.
@@ -341,6 +352,14 @@ __global__ void __launch_bounds__(kPrepThreads) gemm_prep(const __grid_constant_
   // counting as 2^-127.  2^e and 2^-e are normal floats (-126 <= e <= 113),
   // so the products with 2^-e are exact scalings (rounded like any product
   // where they fall below the normal range).  Returns 2^-e_m.
+  // The rows of the last M pair past M are zero (their MMA columns are not
+  // stored, but they must be finite).
+  auto zero_pad_rows = [&]() {
+    const int Mp = P.units_m * (MT * BM);
+    for (int m = P.M + blockIdx.x; m < Mp; m += gridDim.x)
+      for (int i = threadIdx.x; i < Kp / 4; i += kPrepThreads)
+        *reinterpret_cast<uint2*>(P.xg + xg_off(m, 4 * i, P.KT)) = make_uint2(0u, 0u);
+  };
   auto row_scale = [&](int m, uint32_t mx) -> float {
     if (P.xscale) {
       mx = 0;
@@ -391,7 +410,6 @@ __global__ void __launch_bounds__(kPrepThreads) gemm_prep(const __grid_constant_
       if (m + (int)gridDim.x < P.M) load_row(m + gridDim.x, v);
       // four consecutive slots per thread and 8-byte store (with eight, the
       // row reads of a warp's threads collide in shared-memory banks more)
-      uint2* dst = reinterpret_cast<uint2*>(P.xg + (size_t)m * Kp);
       for (int i = threadIdx.x; i < Kp / 4; i += kPrepThreads) {
         uint32_t w[2];
 #pragma unroll
@@ -400,10 +418,11 @@ __global__ void __launch_bounds__(kPrepThreads) gemm_prep(const __grid_constant_
                                            __float2half_rn(value(m, 4 * i + 2 * q + 1) * inv));
           w[q] = *reinterpret_cast<const uint32_t*>(&h);
         }
-        dst[i] = make_uint2(w[0], w[1]);
+        *reinterpret_cast<uint2*>(P.xg + xg_off(m, 4 * i, P.KT)) = make_uint2(w[0], w[1]);
       }
       __syncthreads();  // the row buffer and s_wmax are reused by the next row
     }
+    zero_pad_rows();
     return;
   }
   for (int m = blockIdx.x; m < P.M; m += gridDim.x) {
@@ -430,12 +449,13 @@ __global__ void __launch_bounds__(kPrepThreads) gemm_prep(const __grid_constant_
     mx <<= 16;  // bf16 magnitude bits -> fp32 bits
     __syncthreads();  // the staged row (and, on the first row, the map) is complete
     const float inv = row_scale(m, mx);
-    __half2* dst = reinterpret_cast<__half2*>(P.xg) + (size_t)m * half;
     for (int i = threadIdx.x; i < half; i += kPrepThreads)
-      dst[i] = __halves2half2(__float2half_rn(value(m, 2 * i) * inv),
-                              __float2half_rn(value(m, 2 * i + 1) * inv));
+      *reinterpret_cast<__half2*>(P.xg + xg_off(m, 2 * i, P.KT)) =
+          __halves2half2(__float2half_rn(value(m, 2 * i) * inv),
+                         __float2half_rn(value(m, 2 * i + 1) * inv));
     __syncthreads();  // the row buffer and s_wmax are reused by the next row
   }
+  zero_pad_rows();
 }
 
 // ---------------------------------------------------------------------------
@@ -597,7 +617,6 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
   if (warp == 0) {
     // ---------------- TMA producer ----------------
     if (lane == 0) {
-      prefetch_tmap(&P.tm_x);
       prefetch_tmap(&P.tm_codes);
       if (P.has_meta) prefetch_tmap(&P.tm_meta);
       prefetch_tmap(&P.tm_w16);
@@ -624,8 +643,10 @@ __global__ void __launch_bounds__(kThreadsG, 1) gemm_main(const __grid_constant_
           const uint32_t bar = smem_u32(&bar_full[s]);
           const bool w16 = B.bits == 16;
           mbar_expect_tx(bar, MT * kATile + (w16 ? kBTile : kCodes + kMeta));
-          // both M tiles in one box: 256 rows, the second at + kATile
-          tma_load_2d(smem_u32(st), &P.tm_x, kt * BK, um * (MT * BM), bar);
+          // both M tiles of X: one 16 KB block of Xg, already in the
+          // swizzled shared-memory layout
+          bulk_load(smem_u32(st), P.xg + ((size_t)um * P.KT + kt) * (MT * BM * BK), MT * kATile,
+                    bar);
           if (w16) {
             tma_load_2d(smem_u32(st + MT * kATile), &P.tm_w16, (B.seg_off + 64 * hg) / 2, un * BN,
                         bar);
@@ -876,10 +897,12 @@ int k_tiles(const polyq_dev_layer* L, GmBlock* blk) {
   return kt;
 }
 
-// Workspace: Xg [M][KT*32] fp16, the row scales [M] fp32, then 256 bytes
-// holding the status word; each part starts on a 256-byte boundary.
+// Workspace: Xg (16 KB blocks, M rounded up to a pair of M tiles) fp16, the
+// row scales [M] fp32, then 256 bytes holding the status word; each part
+// starts on a 256-byte boundary.
 size_t gemm_xg_bytes(const polyq_dev_layer* L, int64_t M) {
-  return ((size_t)M * k_tiles(L, nullptr) * BK * 2 + 255) / 256 * 256;
+  const size_t Mp = (size_t)((M + MT * BM - 1) / (MT * BM)) * (MT * BM);
+  return (Mp * k_tiles(L, nullptr) * BK * 2 + 255) / 256 * 256;
 }
 size_t gemm_workspace(const polyq_dev_layer* L, int64_t M) {
   return gemm_xg_bytes(L, M) + ((size_t)M * 4 + 255) / 256 * 256 + 256;
@@ -957,9 +980,6 @@ extern "C" int polyq_linear_gemm(const polyq_dev_layer* L, const void* X, int64_
   P.rowscale = (float*)((uint8_t*)workspace + gemm_xg_bytes(L, M));
   P.y = Y;
   P.status = (int*)((uint8_t*)workspace + need - 256);
-  rc = polyq_tensor_map_2d(&P.tm_x, P.xg, 2, (uint64_t)KT * BK, (uint64_t)M, (uint64_t)KT * BK * 2,
-                           BK, MT * BM, 64);
-  if (rc) return rc;
   rc = polyq_tensor_map_2d(&P.tm_codes, L->packed, 1, (uint64_t)L->row_stride, (uint64_t)L->N,
                            (uint64_t)L->row_stride, kCodeBox, BN);
   if (rc) return rc;
