@@ -56,6 +56,19 @@ using namespace polyq;
 using namespace polyq::gv;
 
 constexpr int kCtasPerSm = 3;
+
+// Bounded wait that also gives up once another warp of the CTA has failed
+// (`abort` set): true when the phase completed.  The flag is read only after
+// a poll has failed, so a stage whose barrier has already completed costs one
+// poll and no shared load.
+__device__ __forceinline__ bool wait_or_abort(uint32_t bar, uint32_t parity,
+                                              const volatile int* abort) {
+  for (uint32_t it = 0; it < kWaitLimit; ++it) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (*abort) return false;
+  }
+  return false;
+}
 constexpr int kMaxGrid = 1024;  // persistent CTAs at most
 constexpr uint32_t kDescEnd = 0x200u;   // descriptor flag: no more items
 constexpr uint32_t kDescPair = 0x400u;  // descriptor flag: the stage holds two steps
@@ -447,7 +460,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) gemv_main(const __grid_c
     bool ok = true;
     while (item < hi) {
       const int slot = ks % kStages;
-      if (s_abort || (ks >= kStages && !mbar_wait(empty0 + 8 * slot, ((ks / kStages) - 1) & 1))) {
+      if (ks >= kStages && !wait_or_abort(empty0 + 8 * slot, ((ks / kStages) - 1) & 1, &s_abort)) {
         if (!s_abort) atomicExch(P.status, kStatusTimeoutEmpty);
         s_abort = 1;
         ok = false;
@@ -481,7 +494,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) gemv_main(const __grid_c
   int slot = 0;
   uint32_t phase = 0;
   for (;;) {
-    if (s_abort || !mbar_wait(full0 + 8 * slot, phase)) {
+    if (!wait_or_abort(full0 + 8 * slot, phase, &s_abort)) {
       if (lane == 0 && !s_abort) atomicExch(P.status, kStatusTimeoutFull);
       s_abort = 1;
       break;
