@@ -377,10 +377,21 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) gemv_main(const __grid_c
     int item = lo;
     if (lo < hi) it.init(S, nl, lo);
     int rec_a[kStages], rec_b[kStages];  // records of each stage's steps (-1: none)
-    // Weights of the next stage: one item, or at batch 2-4 two consecutive
-    // steps of one block and tile whose codes take one box each.
-    auto issue_stage = [&](int k) {
-      const int slot = k % kStages;
+    // Weights of a stage: one item, or at batch 2-4 two consecutive steps of
+    // one block and tile whose codes take one box each.  A stage is planned
+    // (its descriptor and copy coordinates, from the shared layer tables)
+    // before the wait for its slot, and issued after it.
+    struct Plan {
+      uint4 d;
+#ifdef POLYQ_DEBUG
+      uint4 dbg;
+#endif
+      const CUtensorMap* tm;
+      const CUtensorMap* tm_meta;
+      int nbx, pitch, x0, xstep, x2, xmeta, y, pair, rec_a;
+      uint32_t bytes;
+    };
+    auto plan_stage = [&](Plan& p) {
       const GvBlock& B = S.blk[it.l][it.bi];
       int sb, nbx, pitch;
       switch (B.bits) {
@@ -392,51 +403,59 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) gemv_main(const __grid_c
       }
       const bool pair = NB > 1 && nbx == 1 && item + 1 < hi && it.j + 1 < B.n_steps;
       const int j2 = it.j + 1;
-      const uint32_t dst = smem_u32(stages + slot * kStageBytes);
-      const uint32_t bar = full0 + 8 * slot;
-      {
-        // what the consumers need: width, whether the stage ends a tile
-        // piece, pairing, layer, valid units of each step, first meta entry,
-        // tile
-        const int uvalid = min(B.units, B.n_ch - it.j * B.units);
-        const int uvalid2 = pair ? min(B.units, B.n_ch - j2 * B.units) : 0;
-        const int g0 = (B.grp_off + it.j * (B.units / 64)) & 3;
-        const int last_s = it.s + (pair ? 1 : 0);
-        const bool flush = last_s == S.steps[it.l] - 1 || item + (pair ? 2 : 1) == hi;
-        uint4 d;
-        d.x = (uint32_t)B.bits | ((uint32_t)flush << 8) | ((uint32_t)pair << 10) |
+      // what the consumers need: width, whether the stage ends a tile
+      // piece, pairing, layer, valid units of each step, first meta entry,
+      // tile
+      const int uvalid = min(B.units, B.n_ch - it.j * B.units);
+      const int uvalid2 = pair ? min(B.units, B.n_ch - j2 * B.units) : 0;
+      const int g0 = (B.grp_off + it.j * (B.units / 64)) & 3;
+      const int last_s = it.s + (pair ? 1 : 0);
+      const bool flush = last_s == S.steps[it.l] - 1 || item + (pair ? 2 : 1) == hi;
+      p.d.x = (uint32_t)B.bits | ((uint32_t)flush << 8) | ((uint32_t)pair << 10) |
               ((uint32_t)it.l << 16);
-        d.y = (uint32_t)uvalid | ((uint32_t)g0 << 16);
-        d.z = (uint32_t)it.tile;
-        d.w = (uint32_t)uvalid2;
-        *reinterpret_cast<uint4*>(stages + slot * kStageBytes + kDescOff) = d;
+      p.d.y = (uint32_t)uvalid | ((uint32_t)g0 << 16);
+      p.d.z = (uint32_t)it.tile;
+      p.d.w = (uint32_t)uvalid2;
 #ifdef POLYQ_DEBUG
-        *reinterpret_cast<uint4*>(stages + slot * kStageBytes + kDescOff + 16) =
-            make_uint4((uint32_t)(B.pos0 + it.j * B.units), (uint32_t)(it.tile * kRows),
-                       (uint32_t)S.N[it.l], (uint32_t)(B.pos0 + j2 * B.units));
+      p.dbg = make_uint4((uint32_t)(B.pos0 + it.j * B.units), (uint32_t)(it.tile * kRows),
+                         (uint32_t)S.N[it.l], (uint32_t)(B.pos0 + j2 * B.units));
 #endif
-      }
-      uint32_t bytes = (pair ? 2 : 1) * (nbx * pitch * kRows + RB);
-      if (B.bits < 16) bytes += kMetaBytes;
-      mbar_expect_tx(bar, bytes);
-      const CUtensorMap* tm = &P.L[it.l].tm_codes[it.bi];
-      for (int h = 0; h < nbx; ++h)
-        tma_load_2d(dst + h * kRows * pitch, tm, B.seg_off + it.j * sb + h * (sb / nbx),
-                    it.tile * kRows, bar);
-      if (pair) tma_load_2d(dst + kRows * pitch, tm, B.seg_off + j2 * sb, it.tile * kRows, bar);
-      if (B.bits < 16) {
-        // one box of kMetaBox groups covers both steps of a pair
-        const int x0 = (B.grp_off + it.j * (B.units / 64)) & ~3;
-        tma_load_2d(dst + kCodesBytes, &P.L[it.l].tm_meta, x0, it.tile * kRows, bar);
-      }
-      rec_a[slot] = S.rec0[it.l] + it.s;
-      rec_b[slot] = pair ? rec_a[slot] + 1 : -1;
+      p.bytes = (pair ? 2 : 1) * (nbx * pitch * kRows + RB);
+      if (B.bits < 16) p.bytes += kMetaBytes;
+      p.tm = &P.L[it.l].tm_codes[it.bi];
+      p.tm_meta = B.bits < 16 ? &P.L[it.l].tm_meta : nullptr;
+      p.nbx = nbx;
+      p.pitch = pitch;
+      p.x0 = B.seg_off + it.j * sb;
+      p.xstep = sb / nbx;
+      p.x2 = B.seg_off + j2 * sb;
+      // one box of kMetaBox groups covers both steps of a pair
+      p.xmeta = (B.grp_off + it.j * (B.units / 64)) & ~3;
+      p.y = it.tile * kRows;
+      p.pair = pair;
+      p.rec_a = S.rec0[it.l] + it.s;
       it.next(S, nl);
       ++item;
       if (pair) {
         it.next(S, nl);
         ++item;
       }
+    };
+    auto issue_stage = [&](int k, const Plan& p) {
+      const int slot = k % kStages;
+      const uint32_t dst = smem_u32(stages + slot * kStageBytes);
+      const uint32_t bar = full0 + 8 * slot;
+      *reinterpret_cast<uint4*>(stages + slot * kStageBytes + kDescOff) = p.d;
+#ifdef POLYQ_DEBUG
+      *reinterpret_cast<uint4*>(stages + slot * kStageBytes + kDescOff + 16) = p.dbg;
+#endif
+      mbar_expect_tx(bar, p.bytes);
+      for (int h = 0; h < p.nbx; ++h)
+        tma_load_2d(dst + h * kRows * p.pitch, p.tm, p.x0 + h * p.xstep, p.y, bar);
+      if (p.pair) tma_load_2d(dst + kRows * p.pitch, p.tm, p.x2, p.y, bar);
+      if (p.tm_meta) tma_load_2d(dst + kCodesBytes, p.tm_meta, p.xmeta, p.y, bar);
+      rec_a[slot] = p.rec_a;
+      rec_b[slot] = p.pair ? p.rec_a + 1 : -1;
     };
     auto issue_records = [&](int k) {
       const int slot = k % kStages;
@@ -451,14 +470,25 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) gemv_main(const __grid_c
         for (int b = 0; b < S.n_blocks[l]; ++b) prefetch_tmap(&P.L[l].tm_codes[b]);
         prefetch_tmap(&P.L[l].tm_meta);
       }
-      if (item < hi) issue_stage(ks++);
+      if (item < hi) {
+        Plan p0;
+        plan_stage(p0);
+        issue_stage(ks++, p0);
+      }
     }
     pdl_wait();  // the records come from the pre-pass of this call
     fence_proxy_async_global();  // it wrote them through the generic proxy
     if (lane != 0) return;
     if (ks > 0) issue_records(0);
+    // At batch 2-4, where the producer's per-stage work is on the ring's
+    // critical path, the next stage is planned while its slot is still in
+    // use; at batch 1 after the wait (measured 0.7% faster there).
+    constexpr bool kPlanAhead = NB > 1;
     bool ok = true;
-    while (item < hi) {
+    Plan pn;
+    bool have = item < hi;
+    if (kPlanAhead && have) plan_stage(pn);
+    while (have) {
       const int slot = ks % kStages;
       if (ks >= kStages && !wait_or_abort(empty0 + 8 * slot, ((ks / kStages) - 1) & 1, &s_abort)) {
         if (!s_abort) atomicExch(P.status, kStatusTimeoutEmpty);
@@ -466,9 +496,12 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) gemv_main(const __grid_c
         ok = false;
         break;
       }
-      issue_stage(ks);
+      if (!kPlanAhead) plan_stage(pn);
+      issue_stage(ks, pn);
       issue_records(ks);
       ++ks;
+      have = item < hi;
+      if (kPlanAhead && have) plan_stage(pn);
     }
     // wait (bounded) for the copies still in flight, then mark the end of
     // the items in the next stage
