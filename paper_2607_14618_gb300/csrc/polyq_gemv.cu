@@ -460,9 +460,9 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) gemv_main(const __grid_c
     auto issue_records = [&](int k) {
       const int slot = k % kStages;
       const uint32_t dst = smem_u32(stages + slot * kStageBytes + kRecOff);
-      bulk_load(dst, P.rec + (size_t)rec_a[slot] * RB, RB, full0 + 8 * slot);
-      if (rec_b[slot] >= 0)
-        bulk_load(dst + RB, P.rec + (size_t)rec_b[slot] * RB, RB, full0 + 8 * slot);
+      // a paired stage's two records are consecutive: one copy
+      bulk_load(dst, P.rec + (size_t)rec_a[slot] * RB, (rec_b[slot] >= 0 ? 2 : 1) * RB,
+                full0 + 8 * slot);
     };
     int ks = 0;  // stages issued
     if (lane == 0) {
