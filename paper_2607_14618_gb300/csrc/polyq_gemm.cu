@@ -83,7 +83,7 @@ struct GmBlock {
 };
 
 struct GmParams {
-  CUtensorMap tm_codes;  // packed [N][S] u8, box {48, 256}
+  CUtensorMap tm_codes;  // packed [N][S] u8, box {kCodeBox, 256}
   CUtensorMap tm_meta;   // meta [N][meta_stride] u32, box {4, 256}
   CUtensorMap tm_w16;    // packed [N][S/2] u16, box {32, 256}, 64B swizzle
   GmBlock blk[POLYQ_MAX_BLOCKS];
