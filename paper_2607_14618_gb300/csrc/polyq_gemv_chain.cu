@@ -261,7 +261,7 @@ __global__ void __launch_bounds__(kThreads, kChCtasPerSm) gemv_chain(const __gri
       uint32_t it = 0;
       while ((int)(target - ld_acquire_gpu(P.ready + p)) > 0) {
         if (++it > kGridWaitLimit || s_abort) return false;
-        __nanosleep(128);
+        __nanosleep(32);
       }
       fence_proxy_async_global();  // the builders wrote through the generic proxy
       return true;
@@ -416,7 +416,7 @@ __global__ void __launch_bounds__(kThreads, kChCtasPerSm) gemv_chain(const __gri
             s_abort = 1;
             break;
           }
-          __nanosleep(256);
+          __nanosleep(32);
         }
         __threadfence();
       }
